@@ -1,0 +1,183 @@
+/*
+ * cm.h - C ABI of the GB300 CanonicalMerge / LatentFragmentSet library (libcm.so).
+ *
+ * The library implements the data-parallel hot path of "Cache Merging as a
+ * Convergent Replicated State for Multi-Agent Latent Reasoning":
+ *
+ *   Id(C)        content address of a KV-cache fragment          (Section 4.3; Algorithm 2, Id)
+ *   Ingest(S,C)  S u {(Id(C), C)}, duplicates absorbed            (Algorithm 2, Ingest)
+ *   Merge(S1,S2) set union                                        (Eq. setunion; Algorithm 2, Merge)
+ *   Render(S)    CanonicalMerge of the set's fragments            (Algorithm 1; Algorithm 2, Render)
+ *
+ * Data layout. A fragment is one agent's legacy KV cache with the batch
+ * dimension (always 1) dropped: K and V are two DEVICE buffers, each
+ * [num_layers][num_kv_heads][seq_len][head_dim] bf16, contiguous, row-major,
+ * K stored post-RoPE (the key at position t already rotated by R(t)).
+ * A rendered cache is two caller-owned DEVICE buffers
+ * [num_layers][num_kv_heads][capacity_tokens][head_dim] bf16 (row stride =
+ * capacity_tokens); positions >= the rendered length are left untouched.
+ *
+ * Conventions fixed by this library where the paper leaves a choice:
+ *   - content address: BLAKE2s tree hash (RFC 7693; 1024-byte leaves, fanout 128,
+ *     16-byte digests, shapes and dtype in the salt, seq_len in the personalisation)
+ *     of the byte stream K[0],V[0],...,K[L-1],V[L-1];
+ *   - routing layer l* 0-indexed, default floor(L/2); the K-norm score is carried
+ *     as an exact integer key (per-row fp64 norm, quantised to 2^-20);
+ *   - canonical order: descending score, ties by descending id read big-endian;
+ *   - RoPE re-encoding uses the rotate-half pairing (j, j + head_dim/2),
+ *     frequency theta^(-2j/head_dim); the slot at offset 0 is a byte copy; V is a
+ *     byte copy. Re-rotated K is the fp64 rotation rounded once to bf16, bit for bit.
+ *
+ * Errors. Every call validates all arguments before it enqueues any GPU work and
+ * returns a cm_status; no C++ exception crosses this boundary and nothing aborts.
+ * cm_last_error_message() gives a thread-local description of the last failure.
+ *
+ * Threading. Calls on one context are serialised by a lock inside the context.
+ * A set must not be modified (ingest, union, destroy) while another thread uses it.
+ */
+#ifndef CM_H_
+#define CM_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define CM_ABI_VERSION 1
+
+/* Same type as cudaStream_t (a CUDA runtime stream handle); NULL is the legacy default stream. */
+typedef struct CUstream_st *cm_stream_t;
+
+typedef enum cm_status {
+    CM_OK = 0,
+    CM_ERR_INVALID_ARG = 1,     /* null pointer, non-positive size, unsupported head_dim, bad routing layer */
+    CM_ERR_SHAPE_MISMATCH = 2,  /* (layers, kv_heads, head_dim) differ from the set's */
+    CM_ERR_CAPACITY = 3,        /* rendered length exceeds capacity_tokens */
+    CM_ERR_ALIGNMENT = 4,       /* a device buffer is not 16-byte aligned */
+    CM_ERR_COLLISION = 5,       /* verify_bytes_on_hit: equal id, different bytes */
+    CM_ERR_CUDA = 6,            /* a CUDA runtime call failed (message has the CUDA error text) */
+    CM_ERR_OOM = 7,             /* host or device allocation failed */
+    CM_ERR_TIMEOUT = 8,         /* reserved: a bounded device-side wait ran out (no such wait exists yet) */
+    CM_ERR_UNSUPPORTED = 9      /* too many fragments for one render launch group, or shape beyond limits */
+} cm_status;
+
+/* 16-byte content address: the BLAKE2s tree root digest, in digest byte order. */
+typedef struct cm_id {
+    uint8_t b[16];
+} cm_id;
+
+/* One KV-cache fragment. k and v are DEVICE pointers, 16-byte aligned, each
+ * [num_layers][num_kv_heads][seq_len][head_dim] bf16 contiguous. Limits:
+ * 1 <= num_layers, num_kv_heads <= 65535; seq_len >= 1; head_dim a power of two
+ * in [16, 512]. The library only reads them. */
+typedef struct cm_fragment {
+    int32_t num_layers;
+    int32_t num_kv_heads;
+    int32_t seq_len;
+    int32_t head_dim;
+    const void *k;
+    const void *v;
+} cm_fragment;
+
+typedef struct cm_context cm_context;
+typedef struct cm_set cm_set;
+
+/* Library and ABI version (CM_ABI_VERSION). */
+int32_t cm_abi_version(void);
+
+/* Create a context on CUDA device `device`.
+ *   rope_theta          RoPE base theta (> 0), e.g. 1e6 for Qwen3 (Section 4.1)
+ *   routing_layer       l* (0-indexed); < 0 selects floor(num_layers / 2) per fragment (Section 4.3)
+ *   verify_bytes_on_hit nonzero: when an ingested fragment's id is already in the set,
+ *                       compare its bytes with the stored fragment on the device and
+ *                       return CM_ERR_COLLISION if they differ (the paper assumes a
+ *                       collision-resistant hash, Section 4.3, so this never fires)
+ * The context owns device scratch for hashing, grown on demand and freed by
+ * cm_context_destroy. *out receives the handle. */
+cm_status cm_context_create(int32_t device, double rope_theta, int32_t routing_layer,
+                            int32_t verify_bytes_on_hit, cm_context **out);
+
+/* Destroy a context. All sets created from it must have been destroyed. NULL is a no-op. */
+cm_status cm_context_destroy(cm_context *ctx);
+
+/* Create an empty LatentFragmentSet bound to ctx (Section 4.4). */
+cm_status cm_set_create(cm_context *ctx, cm_set **out);
+
+/* Destroy a set (NULL is a no-op). Fragment buffers are borrowed, never freed here. */
+cm_status cm_set_destroy(cm_set *set);
+
+/* Id(C) of Algorithm 2 and the routing-layer norm key of Eq. rho, without a set.
+ * Runs the hash kernels on `stream` and returns after the result reached the host
+ * (the stream is synchronised).
+ *   out_id        receives the 16-byte content address (required)
+ *   out_norm_key  nullable HOST array of frag->seq_len uint64: Q[t] = sum over kv heads of
+ *                 round-half-even(2^20 * ||K[l*][h][t][:]||_2), each term saturated at 2^44-1 */
+cm_status cm_fragment_id(cm_context *ctx, const cm_fragment *frag, cm_stream_t stream,
+                         cm_id *out_id, uint64_t *out_norm_key);
+
+/* Ingest(S, C) of Algorithm 2: content-address the fragment (one pass over its
+ * bytes on `stream`, which is synchronised before return, because membership is
+ * decided on the host) and insert it keyed by its id. A fragment whose id is
+ * already present is absorbed (*out_absorbed = 1) and the set is unchanged.
+ * The set BORROWS frag->k and frag->v: they must stay allocated and unmodified
+ * while the set (or any set it was unioned into) holds the id. The first
+ * fragment fixes the set's (num_layers, num_kv_heads, head_dim); later ones must
+ * match (CM_ERR_SHAPE_MISMATCH); seq_len may differ.
+ *   out_id, out_absorbed  nullable */
+cm_status cm_ingest(cm_set *set, const cm_fragment *frag, cm_stream_t stream, cm_id *out_id,
+                    int32_t *out_absorbed);
+
+/* Merge of Algorithm 2 (Eq. setunion): dst := dst u src. Host only, no GPU work.
+ * Both sets must come from the same context (CM_ERR_INVALID_ARG otherwise) and have
+ * the same shape unless one is empty (CM_ERR_SHAPE_MISMATCH). On equal ids dst keeps
+ * its record (the bytes are equal). dst == src is allowed (idempotent). */
+cm_status cm_union(cm_set *dst, const cm_set *src);
+
+/* Number of distinct fragments in the set. */
+cm_status cm_set_size(const cm_set *set, int64_t *out);
+
+/* Rendered length of the set: the sum of its fragments' seq_len (0 if empty). */
+cm_status cm_set_seq_len(const cm_set *set, int64_t *out);
+
+/* The set's ids in ascending order (bytes compared as a big-endian integer).
+ * Writes min(size, capacity) ids to the HOST array out. */
+cm_status cm_set_ids(const cm_set *set, cm_id *out, int64_t capacity);
+
+/* Render(S) of Algorithm 2 = CanonicalMerge (Algorithm 1) of the set's fragments:
+ * order them by descending routing-layer mean K-norm over the last T* = min seq_len
+ * positions (Eq. rho), ties by descending id; place them along the sequence axis
+ * at offsets s = exclusive prefix sums of seq_len (Section 4.2); copy V; copy K of
+ * the slot at offset 0; rotate every other slot's K by R(s) (Eq. bagmerge-k).
+ * The kernel is enqueued on `stream` and the call returns without waiting.
+ *   k_out, v_out     DEVICE, 16-byte aligned, [L][H][capacity_tokens][d] bf16
+ *   capacity_tokens  must be >= the rendered length (CM_ERR_CAPACITY)
+ *   out_seq_len      nullable; receives the rendered length
+ *   out_order        nullable HOST array of set-size ids: the canonical order
+ * The output bytes are a pure function of the set: identical for every delivery
+ * order and re-delivery. An empty set renders to length 0 and launches nothing
+ * (k_out and v_out may then be NULL). */
+cm_status cm_render(const cm_set *set, void *k_out, void *v_out, int64_t capacity_tokens,
+                    cm_stream_t stream, int64_t *out_seq_len, cm_id *out_order);
+
+/* BagMerge (Section 4.2, Eq. bagmerge-k / bagmerge-v) in the caller's order:
+ * frags[0] at offset 0 (byte copy), frags[i] at the sum of the previous seq_len,
+ * K rotated by R(offset), V copied. No content address, no dedup: passing the same
+ * fragment twice renders it twice (the naive multiset re-render of Section 5.9).
+ * All fragments must share (L, H, d). Enqueued on `stream`; returns without waiting.
+ *   frags  HOST array of n >= 1 descriptors;  other arguments as in cm_render */
+cm_status cm_bagmerge(cm_context *ctx, const cm_fragment *frags, int32_t n, void *k_out,
+                      void *v_out, int64_t capacity_tokens, cm_stream_t stream,
+                      int64_t *out_seq_len);
+
+/* Static name of a status code. */
+const char *cm_status_string(cm_status status);
+
+/* Thread-local text of the last error raised on this thread ("" if none). */
+const char *cm_last_error_message(void);
+
+#ifdef __cplusplus
+}  /* extern "C" */
+#endif
+
+#endif  /* CM_H_ */

@@ -1,0 +1,20 @@
+"""GB300-native CanonicalMerge / LatentFragmentSet (arxiv 2607.01308).
+
+The compute path is libcm.so: hand-written CUDA for sm_103a behind the C ABI of
+include/cm.h. This package is its Python binding (ctypes). Importing it fails
+loudly if the library has not been built; nothing here computes on the CPU.
+
+    import paper_2607_01308_gb300 as cm
+    ctx = cm.Context(device=0, rope_theta=1e6)
+    S = cm.FragmentSet(ctx)
+    fid, absorbed = S.ingest(K, V)          # Algorithm 2, Ingest
+    n, order = S.render(k_out, v_out)       # Algorithm 2, Render (= Algorithm 1)
+"""
+from ._binding import (  # noqa: F401
+    CMError, Status, cm_id, cm_fragment, lib, LIB_PATH, EXPORTED,
+    cm_abi_version, cm_status_string, cm_last_error_message,
+    cm_context_create, cm_context_destroy, cm_set_create, cm_set_destroy,
+    cm_fragment_id, cm_ingest, cm_union, cm_set_size, cm_set_seq_len, cm_set_ids,
+    cm_render, cm_bagmerge,
+    fragment_from_tensors, Context, FragmentSet,
+)

@@ -1,0 +1,290 @@
+"""ctypes binding of libcm.so (include/cm.h): argument marshalling only.
+
+Every function of the C ABI is exposed under its own name, taking plain ints for
+pointers and handles and raising CMError when the call returns a status other
+than CM_OK. Context / FragmentSet wrap the handles for use with torch CUDA
+tensors (torch is used for device memory and streams only).
+"""
+from __future__ import annotations
+
+import ctypes
+import enum
+import os
+from typing import List, Optional, Sequence, Tuple
+
+PKG_DIR = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG_DIR, "libcm.so")
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError(f"{LIB_PATH} is not built: run `python -c \"import __graft_entry__ as g; "
+                      f"g.build()\"` (nvcc, sm_103a) first; there is no fallback implementation")
+
+lib = ctypes.CDLL(LIB_PATH)
+
+
+class Status(enum.IntEnum):
+    OK = 0
+    ERR_INVALID_ARG = 1
+    ERR_SHAPE_MISMATCH = 2
+    ERR_CAPACITY = 3
+    ERR_ALIGNMENT = 4
+    ERR_COLLISION = 5
+    ERR_CUDA = 6
+    ERR_OOM = 7
+    ERR_TIMEOUT = 8
+    ERR_UNSUPPORTED = 9
+
+
+class CMError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        self.status = Status(status) if status in Status._value2member_map_ else status
+        super().__init__(f"{cm_status_string(status)}: {message}")
+
+
+class cm_id(ctypes.Structure):
+    _fields_ = [("b", ctypes.c_uint8 * 16)]
+
+    def to_bytes(self) -> bytes:
+        return bytes(self.b)
+
+
+class cm_fragment(ctypes.Structure):
+    _fields_ = [("num_layers", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
+                ("seq_len", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("k", ctypes.c_void_p), ("v", ctypes.c_void_p)]
+
+
+_c = ctypes
+_P = ctypes.c_void_p
+_SIGS = {
+    "cm_abi_version": (_c.c_int32, []),
+    "cm_status_string": (_c.c_char_p, [_c.c_int]),
+    "cm_last_error_message": (_c.c_char_p, []),
+    "cm_context_create": (_c.c_int, [_c.c_int32, _c.c_double, _c.c_int32, _c.c_int32,
+                                     _c.POINTER(_P)]),
+    "cm_context_destroy": (_c.c_int, [_P]),
+    "cm_set_create": (_c.c_int, [_P, _c.POINTER(_P)]),
+    "cm_set_destroy": (_c.c_int, [_P]),
+    "cm_fragment_id": (_c.c_int, [_P, _c.POINTER(cm_fragment), _P, _c.POINTER(cm_id),
+                                  _c.POINTER(_c.c_uint64)]),
+    "cm_ingest": (_c.c_int, [_P, _c.POINTER(cm_fragment), _P, _c.POINTER(cm_id),
+                             _c.POINTER(_c.c_int32)]),
+    "cm_union": (_c.c_int, [_P, _P]),
+    "cm_set_size": (_c.c_int, [_P, _c.POINTER(_c.c_int64)]),
+    "cm_set_seq_len": (_c.c_int, [_P, _c.POINTER(_c.c_int64)]),
+    "cm_set_ids": (_c.c_int, [_P, _c.POINTER(cm_id), _c.c_int64]),
+    "cm_render": (_c.c_int, [_P, _P, _P, _c.c_int64, _P, _c.POINTER(_c.c_int64),
+                             _c.POINTER(cm_id)]),
+    "cm_bagmerge": (_c.c_int, [_P, _c.POINTER(cm_fragment), _c.c_int32, _P, _P, _c.c_int64, _P,
+                               _c.POINTER(_c.c_int64)]),
+}
+for _name, (_res, _args) in _SIGS.items():
+    _f = getattr(lib, _name)
+    _f.restype = _res
+    _f.argtypes = _args
+
+EXPORTED = tuple(_SIGS)
+
+
+def cm_abi_version() -> int:
+    return lib.cm_abi_version()
+
+
+def cm_status_string(status: int) -> str:
+    return lib.cm_status_string(int(status)).decode()
+
+
+def cm_last_error_message() -> str:
+    return lib.cm_last_error_message().decode()
+
+
+def _check(status: int) -> None:
+    if status != 0:
+        raise CMError(status, cm_last_error_message())
+
+
+def _stream_handle(stream) -> Optional[int]:
+    """None -> torch's current stream if torch is loaded with CUDA, else the legacy default."""
+    if stream is None:
+        try:
+            import torch
+            if torch.cuda.is_available():
+                return torch.cuda.current_stream().cuda_stream or None
+        except ImportError:
+            pass
+        return None
+    if isinstance(stream, int):
+        return stream or None
+    return stream.cuda_stream or None
+
+
+def cm_context_create(device: int = 0, rope_theta: float = 1.0e6, routing_layer: int = -1,
+                      verify_bytes_on_hit: bool = False) -> int:
+    out = _P()
+    _check(lib.cm_context_create(device, rope_theta, routing_layer, int(verify_bytes_on_hit),
+                                 ctypes.byref(out)))
+    return out.value
+
+
+def cm_context_destroy(ctx: Optional[int]) -> None:
+    _check(lib.cm_context_destroy(ctx))
+
+
+def cm_set_create(ctx: int) -> int:
+    out = _P()
+    _check(lib.cm_set_create(ctx, ctypes.byref(out)))
+    return out.value
+
+
+def cm_set_destroy(s: Optional[int]) -> None:
+    _check(lib.cm_set_destroy(s))
+
+
+def cm_fragment_id(ctx: int, frag: cm_fragment, stream=None,
+                   want_norm_key: bool = True) -> Tuple[bytes, Optional[List[int]]]:
+    out = cm_id()
+    q = (ctypes.c_uint64 * frag.seq_len)() if want_norm_key else None
+    _check(lib.cm_fragment_id(ctx, ctypes.byref(frag), _stream_handle(stream), ctypes.byref(out),
+                              q))
+    return out.to_bytes(), (list(q) if q is not None else None)
+
+
+def cm_ingest(s: int, frag: cm_fragment, stream=None) -> Tuple[bytes, bool]:
+    out = cm_id()
+    absorbed = ctypes.c_int32(0)
+    _check(lib.cm_ingest(s, ctypes.byref(frag), _stream_handle(stream), ctypes.byref(out),
+                         ctypes.byref(absorbed)))
+    return out.to_bytes(), bool(absorbed.value)
+
+
+def cm_union(dst: int, src: int) -> None:
+    _check(lib.cm_union(dst, src))
+
+
+def cm_set_size(s: int) -> int:
+    out = ctypes.c_int64()
+    _check(lib.cm_set_size(s, ctypes.byref(out)))
+    return out.value
+
+
+def cm_set_seq_len(s: int) -> int:
+    out = ctypes.c_int64()
+    _check(lib.cm_set_seq_len(s, ctypes.byref(out)))
+    return out.value
+
+
+def cm_set_ids(s: int) -> List[bytes]:
+    n = cm_set_size(s)
+    arr = (cm_id * max(n, 1))()
+    _check(lib.cm_set_ids(s, arr, n))
+    return [arr[i].to_bytes() for i in range(n)]
+
+
+def cm_render(s: int, k_out: int, v_out: int, capacity_tokens: int,
+              stream=None) -> Tuple[int, List[bytes]]:
+    n = cm_set_size(s)
+    order = (cm_id * max(n, 1))()
+    seq = ctypes.c_int64()
+    _check(lib.cm_render(s, k_out, v_out, capacity_tokens, _stream_handle(stream),
+                         ctypes.byref(seq), order))
+    return seq.value, [order[i].to_bytes() for i in range(n)]
+
+
+def cm_bagmerge(ctx: int, frags: Sequence[cm_fragment], k_out: int, v_out: int,
+                capacity_tokens: int, stream=None) -> int:
+    arr = (cm_fragment * max(len(frags), 1))(*frags)
+    seq = ctypes.c_int64()
+    _check(lib.cm_bagmerge(ctx, arr, len(frags), k_out, v_out, capacity_tokens,
+                           _stream_handle(stream), ctypes.byref(seq)))
+    return seq.value
+
+
+# ---------------------------------------------------------------- torch-facing helpers
+
+def fragment_from_tensors(K, V) -> cm_fragment:
+    """Descriptor of a fragment held in two bf16 CUDA tensors [L, H, T, d] (contiguous)."""
+    import torch
+    if K.shape != V.shape or K.dim() != 4:
+        raise ValueError("K and V must both be [layers, kv_heads, seq_len, head_dim]")
+    for t in (K, V):
+        if t.dtype != torch.bfloat16 or not t.is_cuda or not t.is_contiguous():
+            raise ValueError("K and V must be contiguous bf16 CUDA tensors")
+    L, H, T, d = K.shape
+    return cm_fragment(L, H, T, d, K.data_ptr(), V.data_ptr())
+
+
+class Context:
+    """A libcm context on one CUDA device."""
+
+    def __init__(self, device: int = 0, rope_theta: float = 1.0e6, routing_layer: int = -1,
+                 verify_bytes_on_hit: bool = False):
+        self.handle = cm_context_create(device, rope_theta, routing_layer, verify_bytes_on_hit)
+        self.device = device
+        self.rope_theta = rope_theta
+
+    def close(self):
+        if self.handle:
+            cm_context_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def fragment_id(self, K, V, stream=None):
+        return cm_fragment_id(self.handle, fragment_from_tensors(K, V), stream)
+
+    def bagmerge(self, fragments, k_out, v_out, stream=None) -> int:
+        """BagMerge in the given order; fragments = [(K, V), ...] tensors."""
+        frags = [fragment_from_tensors(K, V) for K, V in fragments]
+        return cm_bagmerge(self.handle, frags, k_out.data_ptr(), v_out.data_ptr(),
+                           k_out.shape[2], stream)
+
+
+class FragmentSet:
+    """A LatentFragmentSet. Holds a reference to every ingested tensor pair it keeps,
+    because the library borrows fragment memory."""
+
+    def __init__(self, ctx: Context):
+        self.ctx = ctx
+        self.handle = cm_set_create(ctx.handle)
+        self._keep = {}
+
+    def close(self):
+        if self.handle:
+            cm_set_destroy(self.handle)
+            self.handle = None
+            self._keep.clear()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def ingest(self, K, V, stream=None) -> Tuple[bytes, bool]:
+        fid, absorbed = cm_ingest(self.handle, fragment_from_tensors(K, V), stream)
+        if not absorbed:
+            self._keep[fid] = (K, V)
+        return fid, absorbed
+
+    def union(self, other: "FragmentSet") -> None:
+        cm_union(self.handle, other.handle)
+        for fid, kv in other._keep.items():
+            self._keep.setdefault(fid, kv)
+
+    def __len__(self) -> int:
+        return cm_set_size(self.handle)
+
+    def ids(self) -> List[bytes]:
+        return cm_set_ids(self.handle)
+
+    def seq_len(self) -> int:
+        return cm_set_seq_len(self.handle)
+
+    def render(self, k_out, v_out, stream=None) -> Tuple[int, List[bytes]]:
+        return cm_render(self.handle, k_out.data_ptr() if k_out is not None else 0,
+                         v_out.data_ptr() if v_out is not None else 0,
+                         k_out.shape[2] if k_out is not None else 0, stream)

@@ -1,0 +1,300 @@
+// Content address Id(C) (Section 4.3; Algorithm 2, Id) and the routing-layer
+// norm key (Eq. rho), computed in one pass over the fragment's bytes.
+//
+// Id is a BLAKE2s tree hash (RFC 7693 compression function; tree parameters of
+// the BLAKE2 paper, Section 2.10) of the byte stream K[0] V[0] ... K[L-1] V[L-1]:
+// 1024-byte leaves (depth 0), inner nodes over 128 child digests, 16-byte
+// digests, shapes and dtype in the salt, seq_len in the personalisation.
+//
+// Level 0 runs one thread per leaf: 16 compressions of 64-byte blocks, loaded as
+// 128-bit vectors straight from the fragment buffers. A thread whose leaf lies in
+// K[l*] also accumulates, row by row, the squared norm of each key in fp64 in
+// ascending element order, and adds the quantised norm of every finished row
+// (round-half-even of 2^20 * sqrt, saturated at 2^44 - 1) into Q[t] with a 64-bit
+// integer atomic: integer addition is associative, so Q does not depend on the
+// order the atomics land in. Rows never straddle leaves because head_dim is a
+// power of two with rows of at most 1024 bytes.
+#include "cm_kernels.h"
+
+namespace cm {
+namespace {
+
+constexpr uint32_t kIV0 = 0x6A09E667u, kIV1 = 0xBB67AE85u, kIV2 = 0x3C6EF372u, kIV3 = 0xA54FF53Au;
+constexpr uint32_t kIV4 = 0x510E527Fu, kIV5 = 0x9B05688Cu, kIV6 = 0x1F83D9ABu, kIV7 = 0x5BE0CD19u;
+constexpr unsigned long long kQMax = (1ull << 44) - 1;
+
+__device__ __forceinline__ uint32_t rotr16(uint32_t x) { return __byte_perm(x, 0, 0x1032); }
+__device__ __forceinline__ uint32_t rotr8(uint32_t x) { return __byte_perm(x, 0, 0x0321); }
+__device__ __forceinline__ uint32_t rotr12(uint32_t x) { return __funnelshift_r(x, x, 12); }
+__device__ __forceinline__ uint32_t rotr7(uint32_t x) { return __funnelshift_r(x, x, 7); }
+
+// The G mixing function of RFC 7693, Section 3.1 (rotation distances 16, 12, 8, 7).
+#define CM_G(a, b, c, d, x, y)      \
+    a = a + b + (x);                \
+    d = rotr16(d ^ a);              \
+    c = c + d;                      \
+    b = rotr12(b ^ c);              \
+    a = a + b + (y);                \
+    d = rotr8(d ^ a);               \
+    c = c + d;                      \
+    b = rotr7(b ^ c);
+
+// One round: four column mixes, then four diagonal mixes, message words taken in
+// the order of that round's SIGMA row (RFC 7693, Section 2.7).
+#define CM_ROUND(s0, s1, s2, s3, s4, s5, s6, s7, s8, s9, s10, s11, s12, s13, s14, s15) \
+    CM_G(v0, v4, v8, v12, m[s0], m[s1])                                                \
+    CM_G(v1, v5, v9, v13, m[s2], m[s3])                                                \
+    CM_G(v2, v6, v10, v14, m[s4], m[s5])                                               \
+    CM_G(v3, v7, v11, v15, m[s6], m[s7])                                               \
+    CM_G(v0, v5, v10, v15, m[s8], m[s9])                                               \
+    CM_G(v1, v6, v11, v12, m[s10], m[s11])                                             \
+    CM_G(v2, v7, v8, v13, m[s12], m[s13])                                              \
+    CM_G(v3, v4, v9, v14, m[s14], m[s15])
+
+// Compression function F (RFC 7693, Section 3.2), 10 rounds. t = bytes hashed
+// so far including this block; the last-node flag is applied together with the
+// last-block flag, on the node's final compression.
+__device__ __forceinline__ void compress(uint32_t h[8], const uint32_t m[16], uint64_t t,
+                                         bool last_block, bool last_node) {
+    uint32_t v0 = h[0], v1 = h[1], v2 = h[2], v3 = h[3];
+    uint32_t v4 = h[4], v5 = h[5], v6 = h[6], v7 = h[7];
+    uint32_t v8 = kIV0, v9 = kIV1, v10 = kIV2, v11 = kIV3;
+    uint32_t v12 = kIV4 ^ (uint32_t)t, v13 = kIV5 ^ (uint32_t)(t >> 32);
+    uint32_t v14 = last_block ? ~kIV6 : kIV6;
+    uint32_t v15 = (last_block && last_node) ? ~kIV7 : kIV7;
+    CM_ROUND(0, 1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 11, 12, 13, 14, 15)
+    CM_ROUND(14, 10, 4, 8, 9, 15, 13, 6, 1, 12, 0, 2, 11, 7, 5, 3)
+    CM_ROUND(11, 8, 12, 0, 5, 2, 15, 13, 10, 14, 3, 6, 7, 1, 9, 4)
+    CM_ROUND(7, 9, 3, 1, 13, 12, 11, 14, 2, 6, 5, 10, 4, 0, 15, 8)
+    CM_ROUND(9, 0, 5, 7, 2, 4, 10, 15, 14, 1, 11, 12, 6, 8, 3, 13)
+    CM_ROUND(2, 12, 6, 10, 0, 11, 8, 3, 4, 13, 7, 5, 15, 14, 1, 9)
+    CM_ROUND(12, 5, 1, 15, 14, 13, 4, 10, 0, 7, 6, 3, 9, 2, 8, 11)
+    CM_ROUND(13, 11, 7, 14, 12, 1, 3, 9, 5, 0, 15, 4, 8, 6, 2, 10)
+    CM_ROUND(6, 15, 14, 9, 11, 3, 0, 8, 12, 2, 13, 7, 1, 4, 10, 5)
+    CM_ROUND(10, 2, 8, 4, 7, 6, 1, 5, 15, 11, 9, 14, 3, 12, 13, 0)
+    h[0] ^= v0 ^ v8;
+    h[1] ^= v1 ^ v9;
+    h[2] ^= v2 ^ v10;
+    h[3] ^= v3 ^ v11;
+    h[4] ^= v4 ^ v12;
+    h[5] ^= v5 ^ v13;
+    h[6] ^= v6 ^ v14;
+    h[7] ^= v7 ^ v15;
+}
+
+#undef CM_ROUND
+#undef CM_G
+
+// Chaining value of node (offset, depth): the base words with the 48-bit node
+// offset (parameter bytes 8..13) and the node depth (byte 14) xored in.
+__device__ __forceinline__ void node_init(uint32_t h[8], const TreeParams &tp, uint64_t offset,
+                                          uint32_t depth) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) h[i] = tp.h_base[i];
+    h[2] ^= (uint32_t)offset;
+    h[3] ^= ((uint32_t)(offset >> 32) & 0xFFFFu) | (depth << 16);
+}
+
+__device__ __forceinline__ uint4 load_nc(const uint8_t *p) {
+    return __ldg(reinterpret_cast<const uint4 *>(p));
+}
+
+__device__ __forceinline__ void store_digest(uint8_t *dst, const uint32_t h[8]) {
+    *reinterpret_cast<uint4 *>(dst) = make_uint4(h[0], h[1], h[2], h[3]);
+}
+
+// Squared-norm accumulation of one 16-byte vector (8 bf16, ascending element
+// order) at stream offset pos; finishes the row on its last vector.
+struct NormState {
+    double ss;
+};
+
+__device__ __forceinline__ void norm_vector(const LeafLaunch &a, NormState &st, uint4 w,
+                                            uint64_t pos) {
+    if (pos < a.norm_begin || pos >= a.norm_begin + a.plane_bytes) return;
+    const uint32_t words[4] = {w.x, w.y, w.z, w.w};
+    double ss = st.ss;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const double lo = (double)__uint_as_float(words[i] << 16);
+        const double hi = (double)__uint_as_float(words[i] & 0xFFFF0000u);
+        ss = __fma_rn(lo, lo, ss);   // x*x is exact in fp64, so this is fl(ss + x^2)
+        ss = __fma_rn(hi, hi, ss);
+    }
+    const uint64_t rel = pos - a.norm_begin;
+    if ((rel & (uint64_t)(a.row_bytes - 1)) == (uint64_t)(a.row_bytes - 16)) {
+        const uint32_t row = (uint32_t)(rel / a.row_bytes);
+        const uint32_t t = row % a.seq_len;
+        const double scaled = __dsqrt_rn(ss) * 1048576.0;     // exact scaling by 2^20
+        const unsigned long long q =
+            (scaled < (double)kQMax) ? __double2ull_rn(scaled) : kQMax;   // NaN saturates too
+        atomicAdd(a.norm_key + t, q);
+        ss = 0.0;
+    }
+    st.ss = ss;
+}
+
+// Cursor over the fragment's byte stream K[0] V[0] K[1] V[1] ...: every segment
+// (one layer of K or of V) is plane_bytes long, a multiple of 32, so a 16-byte
+// vector never straddles two segments.
+struct StreamCursor {
+    const uint8_t *ptr;
+    uint64_t left;       // bytes left in the current segment
+    uint32_t layer;
+    bool in_v;
+};
+
+__device__ __forceinline__ StreamCursor cursor_at(const LeafLaunch &a, uint64_t pos) {
+    StreamCursor c;
+    const uint64_t two_p = 2 * a.plane_bytes;
+    c.layer = (uint32_t)(pos / two_p);
+    const uint64_t within = pos - (uint64_t)c.layer * two_p;
+    c.in_v = within >= a.plane_bytes;
+    const uint64_t seg_off = c.in_v ? within - a.plane_bytes : within;
+    c.ptr = (c.in_v ? a.v : a.k) + (uint64_t)c.layer * a.plane_bytes + seg_off;
+    c.left = a.plane_bytes - seg_off;
+    return c;
+}
+
+__device__ __forceinline__ const uint8_t *cursor_next(const LeafLaunch &a, StreamCursor &c) {
+    if (c.left == 0) {
+        if (c.in_v) {
+            c.in_v = false;
+            ++c.layer;
+        } else {
+            c.in_v = true;
+        }
+        c.ptr = (c.in_v ? a.v : a.k) + (uint64_t)c.layer * a.plane_bytes;
+        c.left = a.plane_bytes;
+    }
+    const uint8_t *p = c.ptr;
+    c.ptr += 16;
+    c.left -= 16;
+    return p;
+}
+
+constexpr int kLeafThreads = 128;
+
+__global__ void __launch_bounds__(kLeafThreads)
+leaf_hash_kernel(const __grid_constant__ LeafLaunch a) {
+    const uint64_t leaf = (uint64_t)blockIdx.x * kLeafThreads + threadIdx.x;
+    if (leaf >= a.num_leaves) return;
+    const uint64_t begin = leaf * kLeafBytes;
+    const uint64_t rem = a.stream_bytes - begin;
+    const uint32_t len = rem < (uint64_t)kLeafBytes ? (uint32_t)rem : (uint32_t)kLeafBytes;
+    const uint32_t nblocks = (len + 63) / 64;
+    const bool last_node = leaf + 1 == a.num_leaves;
+    const bool norm_leaf = begin < a.norm_begin + a.plane_bytes && begin + len > a.norm_begin;
+
+    uint32_t h[8];
+    node_init(h, a.tree, leaf, 0);
+    StreamCursor cur = cursor_at(a, begin);
+    NormState ns{0.0};
+
+    // Two 64-byte blocks (one 128-byte line) per step: eight 16-byte loads in flight.
+    for (uint32_t b = 0; b < nblocks; b += 2) {
+        uint4 w[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            const uint32_t off = b * 64 + q * 16;
+            w[q] = off < len ? load_nc(cursor_next(a, cur)) : make_uint4(0, 0, 0, 0);
+        }
+        if (norm_leaf) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const uint32_t off = b * 64 + q * 16;
+                if (off < len) norm_vector(a, ns, w[q], begin + off);
+            }
+        }
+        {
+            const uint32_t m[16] = {w[0].x, w[0].y, w[0].z, w[0].w, w[1].x, w[1].y, w[1].z, w[1].w,
+                                    w[2].x, w[2].y, w[2].z, w[2].w, w[3].x, w[3].y, w[3].z, w[3].w};
+            const uint32_t end = (b + 1) * 64 < len ? (b + 1) * 64 : len;
+            compress(h, m, end, b + 1 == nblocks, last_node);
+        }
+        if (b + 1 < nblocks) {
+            const uint32_t m[16] = {w[4].x, w[4].y, w[4].z, w[4].w, w[5].x, w[5].y, w[5].z, w[5].w,
+                                    w[6].x, w[6].y, w[6].z, w[6].w, w[7].x, w[7].y, w[7].z, w[7].w};
+            const uint32_t end = (b + 2) * 64 < len ? (b + 2) * 64 : len;
+            compress(h, m, end, b + 2 == nblocks, last_node);
+        }
+    }
+    store_digest(a.digests + leaf * kDigestBytes, h);
+}
+
+constexpr int kInnerThreads = 32;
+
+__global__ void __launch_bounds__(kInnerThreads)
+inner_hash_kernel(const uint8_t *__restrict__ children, uint64_t num_children,
+                  uint8_t *__restrict__ out, uint64_t num_nodes, uint32_t depth,
+                  const __grid_constant__ TreeParams tp) {
+    const uint64_t j = (uint64_t)blockIdx.x * kInnerThreads + threadIdx.x;
+    if (j >= num_nodes) return;
+    const uint64_t first = j * kFanout;
+    const uint64_t nc64 = num_children - first;
+    const uint32_t nc = nc64 < (uint64_t)kFanout ? (uint32_t)nc64 : (uint32_t)kFanout;
+    const uint32_t len = nc * kDigestBytes;
+    const uint32_t nblocks = (len + 63) / 64;
+    const bool last_node = j + 1 == num_nodes;
+    const uint8_t *src = children + first * kDigestBytes;
+
+    uint32_t h[8];
+    node_init(h, tp, j, depth);
+    for (uint32_t b = 0; b < nblocks; ++b) {
+        uint4 w[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const uint32_t off = b * 64 + q * 16;
+            w[q] = off < len ? load_nc(src + off) : make_uint4(0, 0, 0, 0);
+        }
+        const uint32_t m[16] = {w[0].x, w[0].y, w[0].z, w[0].w, w[1].x, w[1].y, w[1].z, w[1].w,
+                                w[2].x, w[2].y, w[2].z, w[2].w, w[3].x, w[3].y, w[3].z, w[3].w};
+        const uint32_t end = (b + 1) * 64 < len ? (b + 1) * 64 : len;
+        compress(h, m, end, b + 1 == nblocks, last_node);
+    }
+    store_digest(out + j * kDigestBytes, h);
+}
+
+__global__ void compare_kernel(const uint4 *__restrict__ a, const uint4 *__restrict__ b,
+                               uint64_t n, unsigned int *flag) {
+    uint32_t diff = 0;
+    for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (uint64_t)gridDim.x * blockDim.x) {
+        const uint4 x = __ldg(a + i), y = __ldg(b + i);
+        diff |= (x.x ^ y.x) | (x.y ^ y.y) | (x.z ^ y.z) | (x.w ^ y.w);
+    }
+    if (__any_sync(0xFFFFFFFFu, diff != 0) && (threadIdx.x & 31) == 0) atomicOr(flag, 1u);
+}
+
+}  // namespace
+
+cudaError_t launch_leaf_hash(const LeafLaunch &a, cudaStream_t stream) {
+    if (a.num_leaves == 0) return cudaSuccess;
+    const uint64_t blocks = (a.num_leaves + kLeafThreads - 1) / kLeafThreads;
+    if (blocks > 0x7FFFFFFFull) return cudaErrorInvalidValue;
+    leaf_hash_kernel<<<(unsigned)blocks, kLeafThreads, 0, stream>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_inner_hash(const uint8_t *children, uint64_t num_children, uint8_t *out,
+                              uint64_t num_nodes, uint32_t depth, const TreeParams &tree,
+                              cudaStream_t stream) {
+    if (num_nodes == 0) return cudaSuccess;
+    const uint64_t blocks = (num_nodes + kInnerThreads - 1) / kInnerThreads;
+    inner_hash_kernel<<<(unsigned)blocks, kInnerThreads, 0, stream>>>(children, num_children, out,
+                                                                    num_nodes, depth, tree);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_compare(const void *a, const void *b, uint64_t bytes, unsigned int *flag,
+                           cudaStream_t stream) {
+    const uint64_t n = bytes / 16;
+    if (n == 0) return cudaSuccess;
+    uint64_t blocks = (n + 255) / 256;
+    if (blocks > 4096) blocks = 4096;
+    compare_kernel<<<(unsigned)blocks, 256, 0, stream>>>(static_cast<const uint4 *>(a),
+                                                         static_cast<const uint4 *>(b), n, flag);
+    return cudaGetLastError();
+}
+
+}  // namespace cm

@@ -1,0 +1,676 @@
+// Host core of libcm: contexts, LatentFragmentSet state, canonical order and
+// launch orchestration behind the C ABI of include/cm.h.
+//
+//   cm_fragment_id / cm_ingest   Id(C) and the norm key on the GPU, then the set
+//                                insert on the host (Algorithm 2, Id / Ingest)
+//   cm_union                     set union over 16-byte ids (Eq. setunion)
+//   cm_render                    canonical order (Algorithm 1) on the host, then
+//                                one fused copy-and-rotate launch (Eq. bagmerge-k/v)
+//   cm_bagmerge                  the same launch in a caller-given order (Section 4.2)
+#include "cm.h"
+
+#include <algorithm>
+#include <array>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <memory>
+#include <mutex>
+#include <new>
+#include <string>
+#include <vector>
+
+#include <cuda_runtime.h>
+
+#include "cm_kernels.h"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+cm_status fail(cm_status st, const std::string &msg) {
+    g_last_error = msg;
+    return st;
+}
+
+cm_status cuda_fail(cudaError_t e, const char *what) {
+    return fail(CM_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+#define CM_CUDA_TRY(expr, what)                              \
+    do {                                                      \
+        cudaError_t e_ = (expr);                              \
+        if (e_ != cudaSuccess) return cuda_fail(e_, (what));  \
+    } while (0)
+
+// Makes `device` current for the scope of a call and restores the caller's device.
+class DeviceScope {
+  public:
+    explicit DeviceScope(int device) {
+        ok_ = cudaGetDevice(&prev_) == cudaSuccess;
+        if (ok_ && prev_ != device) ok_ = cudaSetDevice(device) == cudaSuccess;
+        changed_ = ok_ && prev_ != device;
+    }
+    ~DeviceScope() {
+        if (changed_) cudaSetDevice(prev_);
+    }
+    bool ok() const { return ok_; }
+
+  private:
+    int prev_ = 0;
+    bool ok_ = false;
+    bool changed_ = false;
+};
+
+using IdKey = std::array<uint8_t, 16>;   // operator< is lexicographic = big-endian numeric
+
+IdKey key_of(const cm_id &id) {
+    IdKey k;
+    std::memcpy(k.data(), id.b, 16);
+    return k;
+}
+
+struct Record {
+    cm_id id;
+    int32_t L, H, T, d;
+    const void *k;
+    const void *v;
+    std::vector<uint64_t> Q;   // routing-layer norm key Q[t]
+};
+
+bool is_pow2(int64_t x) { return x > 0 && (x & (x - 1)) == 0; }
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+cm_status validate_fragment(const cm_fragment *f) {
+    if (!f) return fail(CM_ERR_INVALID_ARG, "fragment descriptor is NULL");
+    if (f->num_layers < 1 || f->num_layers > 65535 || f->num_kv_heads < 1 ||
+        f->num_kv_heads > 65535 || f->seq_len < 1)
+        return fail(CM_ERR_INVALID_ARG, "fragment sizes out of range (layers and kv heads in "
+                                        "[1, 65535], seq_len >= 1)");
+    if (!is_pow2(f->head_dim) || f->head_dim < 16 || f->head_dim > 512)
+        return fail(CM_ERR_INVALID_ARG, "head_dim must be a power of two in [16, 512]");
+    if (!f->k || !f->v) return fail(CM_ERR_INVALID_ARG, "fragment k or v pointer is NULL");
+    if (!aligned16(f->k) || !aligned16(f->v))
+        return fail(CM_ERR_ALIGNMENT, "fragment k and v must be 16-byte aligned");
+    const long double bytes = (long double)f->num_layers * f->num_kv_heads * f->seq_len *
+                              f->head_dim * 2.0L * 2.0L;
+    if (bytes > 9.0e15L) return fail(CM_ERR_UNSUPPORTED, "fragment too large");
+    return CM_OK;
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------ context
+
+struct cm_context {
+    int device = 0;
+    double theta = 1e6;
+    int32_t routing_layer = -1;
+    bool verify = false;
+    int num_sms = 0;
+    int render_blocks_per_sm = 1;
+    std::mutex mu;
+    // hashing scratch (device): leaf digests, inner levels, Q[t], compare flag
+    uint8_t *d_scratch = nullptr;
+    size_t scratch_bytes = 0;
+    // pinned host staging for the root digest, Q[t] and the compare flag
+    uint8_t *h_pinned = nullptr;
+    size_t pinned_bytes = 0;
+    int live_sets = 0;
+};
+
+struct cm_set {
+    cm_context *ctx = nullptr;
+    bool has_shape = false;
+    int32_t L = 0, H = 0, d = 0;
+    std::map<IdKey, std::shared_ptr<const Record>> items;
+};
+
+namespace {
+
+int32_t routing_layer_for(const cm_context *ctx, int32_t L) {
+    return ctx->routing_layer < 0 ? L / 2 : ctx->routing_layer;
+}
+
+cm_status ensure_scratch(cm_context *ctx, size_t dev_bytes, size_t host_bytes) {
+    if (dev_bytes > ctx->scratch_bytes) {
+        if (ctx->d_scratch) cudaFree(ctx->d_scratch);
+        ctx->d_scratch = nullptr;
+        ctx->scratch_bytes = 0;
+        const size_t want = std::max(dev_bytes, (size_t)1 << 20);
+        cudaError_t e = cudaMalloc(&ctx->d_scratch, want);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return fail(CM_ERR_OOM, std::string("device scratch allocation failed: ") +
+                                        cudaGetErrorString(e));
+        }
+        ctx->scratch_bytes = want;
+    }
+    if (host_bytes > ctx->pinned_bytes) {
+        if (ctx->h_pinned) cudaFreeHost(ctx->h_pinned);
+        ctx->h_pinned = nullptr;
+        ctx->pinned_bytes = 0;
+        const size_t want = std::max(host_bytes, (size_t)1 << 16);
+        cudaError_t e = cudaHostAlloc(reinterpret_cast<void **>(&ctx->h_pinned), want,
+                                      cudaHostAllocDefault);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return fail(CM_ERR_OOM, std::string("pinned host allocation failed: ") +
+                                        cudaGetErrorString(e));
+        }
+        ctx->pinned_bytes = want;
+    }
+    return CM_OK;
+}
+
+// BLAKE2s parameter block (32 bytes) of the tree, node offset and depth zero,
+// xored into the IV: digest 16, no key, fanout 128, depth 255 (unlimited),
+// leaf 1024, inner 16, salt = <L, H, d, 1 (bf16)> as little-endian uint16,
+// personalisation = <T> as a little-endian uint64.
+cm::TreeParams tree_params(int32_t L, int32_t H, int32_t d, int32_t T) {
+    static const uint32_t iv[8] = {0x6A09E667u, 0xBB67AE85u, 0x3C6EF372u, 0xA54FF53Au,
+                                   0x510E527Fu, 0x9B05688Cu, 0x1F83D9ABu, 0x5BE0CD19u};
+    uint8_t p[32];
+    std::memset(p, 0, sizeof p);
+    p[0] = cm::kDigestBytes;
+    p[1] = 0;
+    p[2] = cm::kFanout;
+    p[3] = 255;
+    const uint32_t leaf = cm::kLeafBytes;
+    for (int i = 0; i < 4; ++i) p[4 + i] = (uint8_t)(leaf >> (8 * i));
+    p[15] = cm::kDigestBytes;   // inner length
+    const uint16_t salt[4] = {(uint16_t)L, (uint16_t)H, (uint16_t)d, 1};
+    for (int i = 0; i < 4; ++i) {
+        p[16 + 2 * i] = (uint8_t)(salt[i] & 0xFF);
+        p[17 + 2 * i] = (uint8_t)(salt[i] >> 8);
+    }
+    const uint64_t person = (uint64_t)T;
+    for (int i = 0; i < 8; ++i) p[24 + i] = (uint8_t)(person >> (8 * i));
+    cm::TreeParams tp;
+    for (int i = 0; i < 8; ++i) {
+        const uint32_t w = (uint32_t)p[4 * i] | ((uint32_t)p[4 * i + 1] << 8) |
+                           ((uint32_t)p[4 * i + 2] << 16) | ((uint32_t)p[4 * i + 3] << 24);
+        tp.h_base[i] = iv[i] ^ w;
+    }
+    return tp;
+}
+
+uint64_t ceil_div(uint64_t a, uint64_t b) { return (a + b - 1) / b; }
+
+// Id(C) and Q[t] of one fragment; caller holds ctx->mu and the device scope.
+cm_status fragment_digest(cm_context *ctx, const cm_fragment *f, cudaStream_t stream, cm_id *id,
+                          std::vector<uint64_t> *Q) {
+    const int32_t L = f->num_layers, H = f->num_kv_heads, T = f->seq_len, d = f->head_dim;
+    const int32_t rl = routing_layer_for(ctx, L);
+    if (rl >= L) return fail(CM_ERR_INVALID_ARG, "routing layer >= num_layers");
+    const uint64_t plane = (uint64_t)H * T * d * 2;
+    const uint64_t stream_bytes = 2ull * L * plane;
+    std::vector<uint64_t> sizes{ceil_div(stream_bytes, cm::kLeafBytes)};
+    while (sizes.size() == 1 || sizes.back() > 1) sizes.push_back(ceil_div(sizes.back(), cm::kFanout));
+    // device layout: [Q: T x 8][level 0][level 1]... (each level 16-byte aligned)
+    const size_t q_bytes = ((size_t)T * 8 + 255) & ~(size_t)255;
+    std::vector<size_t> level_off;
+    size_t off = q_bytes;
+    for (uint64_t n : sizes) {
+        level_off.push_back(off);
+        off += ((size_t)n * cm::kDigestBytes + 255) & ~(size_t)255;
+    }
+    const size_t host_bytes = 16 + (size_t)T * 8;
+    cm_status st = ensure_scratch(ctx, off, host_bytes);
+    if (st != CM_OK) return st;
+    uint8_t *base = ctx->d_scratch;
+    auto *dq = reinterpret_cast<unsigned long long *>(base);
+    const cm::TreeParams tp = tree_params(L, H, d, T);
+
+    CM_CUDA_TRY(cudaMemsetAsync(dq, 0, (size_t)T * 8, stream), "zeroing the norm key");
+    cm::LeafLaunch a;
+    a.k = static_cast<const uint8_t *>(f->k);
+    a.v = static_cast<const uint8_t *>(f->v);
+    a.plane_bytes = plane;
+    a.stream_bytes = stream_bytes;
+    a.num_leaves = sizes[0];
+    a.norm_begin = 2ull * (uint64_t)rl * plane;
+    a.row_bytes = (uint32_t)d * 2;
+    a.seq_len = (uint32_t)T;
+    a.norm_key = dq;
+    a.digests = base + level_off[0];
+    a.tree = tp;
+    CM_CUDA_TRY(cm::launch_leaf_hash(a, stream), "leaf hash launch");
+    for (size_t k = 1; k < sizes.size(); ++k) {
+        CM_CUDA_TRY(cm::launch_inner_hash(base + level_off[k - 1], sizes[k - 1], base + level_off[k],
+                                          sizes[k], (uint32_t)k, tp, stream),
+                    "inner hash launch");
+    }
+    CM_CUDA_TRY(cudaMemcpyAsync(ctx->h_pinned, base + level_off.back(), 16, cudaMemcpyDeviceToHost,
+                                stream),
+                "digest copy");
+    CM_CUDA_TRY(cudaMemcpyAsync(ctx->h_pinned + 16, dq, (size_t)T * 8, cudaMemcpyDeviceToHost,
+                                stream),
+                "norm key copy");
+    CM_CUDA_TRY(cudaStreamSynchronize(stream), "ingest synchronisation");
+    std::memcpy(id->b, ctx->h_pinned, 16);
+    if (Q) {
+        Q->resize((size_t)T);
+        std::memcpy(Q->data(), ctx->h_pinned + 16, (size_t)T * 8);
+    }
+    return CM_OK;
+}
+
+// Byte comparison of a new fragment against a stored record with the same id.
+cm_status bytes_equal(cm_context *ctx, const cm_fragment *f, const Record &r, cudaStream_t stream,
+                      bool *equal) {
+    const uint64_t bytes = (uint64_t)f->num_layers * f->num_kv_heads * f->seq_len * f->head_dim * 2;
+    if (r.L != f->num_layers || r.H != f->num_kv_heads || r.T != f->seq_len || r.d != f->head_dim) {
+        *equal = false;
+        return CM_OK;
+    }
+    cm_status st = ensure_scratch(ctx, 256, 16);
+    if (st != CM_OK) return st;
+    auto *flag = reinterpret_cast<unsigned int *>(ctx->d_scratch);
+    CM_CUDA_TRY(cudaMemsetAsync(flag, 0, sizeof(unsigned int), stream), "flag reset");
+    CM_CUDA_TRY(cm::launch_compare(f->k, r.k, bytes, flag, stream), "compare launch");
+    CM_CUDA_TRY(cm::launch_compare(f->v, r.v, bytes, flag, stream), "compare launch");
+    CM_CUDA_TRY(cudaMemcpyAsync(ctx->h_pinned, flag, sizeof(unsigned int), cudaMemcpyDeviceToHost,
+                                stream),
+                "flag copy");
+    CM_CUDA_TRY(cudaStreamSynchronize(stream), "compare synchronisation");
+    unsigned int h;
+    std::memcpy(&h, ctx->h_pinned, sizeof h);
+    *equal = h == 0;
+    return CM_OK;
+}
+
+// One slot of a render: a fragment and its output offset.
+struct Slot {
+    const void *k;
+    const void *v;
+    int64_t T;
+    int64_t offset;
+};
+
+// Fused copy-and-rotate of slots already in order (offsets set), in launch groups
+// of at most kMaxSlots slots and kMaxTablePairs (cos, sin) pairs.
+cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t L, int32_t H,
+                       int32_t d, void *k_out, void *v_out, int64_t capacity, cudaStream_t stream) {
+    const int rows_per_chunk = cm::kChunkBytes / (2 * d);
+    const int half = d / 2;
+    const int max_group = std::min<int>(cm::kMaxSlots, cm::kMaxTablePairs / half);
+    const uint64_t planes = 2ull * L * H;
+    int log2_pairs = 0;
+    while ((1 << log2_pairs) < d / 16) ++log2_pairs;
+    std::unique_ptr<cm::RenderParams> p(new cm::RenderParams);
+    for (size_t g0 = 0; g0 < slots.size(); g0 += (size_t)max_group) {
+        const size_t n = std::min(slots.size() - g0, (size_t)max_group);
+        std::memset(p.get(), 0, sizeof(cm::RenderParams));
+        p->k_out = k_out;
+        p->v_out = v_out;
+        p->capacity = capacity;
+        p->num_layers = L;
+        p->num_heads = H;
+        p->head_dim = d;
+        p->num_slots = (int32_t)n;
+        p->rows_per_chunk = rows_per_chunk;
+        p->log2_pairs_per_row = log2_pairs;
+        uint64_t chunk = 0;
+        for (size_t i = 0; i < n; ++i) {
+            const Slot &s = slots[g0 + i];
+            cm::RenderSlot &rs = p->slot[i];
+            rs.k = s.k;
+            rs.v = s.v;
+            rs.seq_len = s.T;
+            rs.offset = s.offset;
+            rs.rotate = s.offset != 0;
+            rs.table_base = (int32_t)i * half;
+            const uint64_t cpp = ceil_div((uint64_t)s.T, (uint64_t)rows_per_chunk);
+            rs.chunk_begin = (uint32_t)chunk;
+            rs.chunks_per_plane = (uint32_t)cpp;
+            chunk += cpp * planes;
+            // delta angle a_j = s * theta^(-2j/d) in fp64 (Section 2.3 / Eq. bagmerge-k)
+            for (int j = 0; j < half; ++j) {
+                const double w = std::pow(ctx->theta, -(2.0 * j) / d);
+                const double a = (double)s.offset * w;
+                p->cs[2 * (i * half + j)] = std::cos(a);
+                p->cs[2 * (i * half + j) + 1] = std::sin(a);
+            }
+        }
+        if (chunk > 0xFFFFFFFFull)
+            return fail(CM_ERR_UNSUPPORTED, "render launch group exceeds 2^32 work items");
+        p->total_chunks = (uint32_t)chunk;
+        const uint64_t resident = (uint64_t)ctx->num_sms * ctx->render_blocks_per_sm;
+        const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(chunk, resident));
+        CM_CUDA_TRY(cm::launch_render(*p, grid, stream), "render launch");
+    }
+    return CM_OK;
+}
+
+cm_status validate_outputs(void *k_out, void *v_out, int64_t capacity, int64_t total) {
+    if (capacity < total)
+        return fail(CM_ERR_CAPACITY, "rendered length " + std::to_string(total) +
+                                         " exceeds capacity_tokens " + std::to_string(capacity));
+    if (total == 0) return CM_OK;
+    if (!k_out || !v_out) return fail(CM_ERR_INVALID_ARG, "k_out or v_out is NULL");
+    if (!aligned16(k_out) || !aligned16(v_out))
+        return fail(CM_ERR_ALIGNMENT, "k_out and v_out must be 16-byte aligned");
+    return CM_OK;
+}
+
+// Canonical order of Algorithm 1: descending tail sum of the norm key over the
+// last T* = min T positions (the integer form of rho, Eq. rho), ties by
+// descending id read big-endian.
+std::vector<std::shared_ptr<const Record>> canonical_order(const cm_set *set) {
+    std::vector<std::shared_ptr<const Record>> recs;
+    recs.reserve(set->items.size());
+    int64_t t_star = INT64_MAX;
+    for (const auto &kv : set->items) {
+        recs.push_back(kv.second);
+        t_star = std::min<int64_t>(t_star, kv.second->T);
+    }
+    struct Keyed {
+        unsigned __int128 S;
+        IdKey id;
+        std::shared_ptr<const Record> r;
+    };
+    std::vector<Keyed> keyed;
+    keyed.reserve(recs.size());
+    for (auto &r : recs) {
+        unsigned __int128 S = 0;
+        for (int64_t t = r->T - t_star; t < r->T; ++t) S += r->Q[(size_t)t];
+        keyed.push_back({S, key_of(r->id), r});
+    }
+    std::sort(keyed.begin(), keyed.end(), [](const Keyed &a, const Keyed &b) {
+        if (a.S != b.S) return a.S > b.S;
+        return a.id > b.id;
+    });
+    std::vector<std::shared_ptr<const Record>> out;
+    out.reserve(keyed.size());
+    for (auto &k : keyed) out.push_back(k.r);
+    return out;
+}
+
+template <class F>
+cm_status guarded(F &&f) {
+    try {
+        return f();
+    } catch (const std::bad_alloc &) {
+        return fail(CM_ERR_OOM, "host allocation failed");
+    } catch (...) {
+        return fail(CM_ERR_INVALID_ARG, "unexpected internal error");
+    }
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t cm_abi_version(void) { return CM_ABI_VERSION; }
+
+const char *cm_status_string(cm_status s) {
+    switch (s) {
+        case CM_OK: return "CM_OK";
+        case CM_ERR_INVALID_ARG: return "CM_ERR_INVALID_ARG";
+        case CM_ERR_SHAPE_MISMATCH: return "CM_ERR_SHAPE_MISMATCH";
+        case CM_ERR_CAPACITY: return "CM_ERR_CAPACITY";
+        case CM_ERR_ALIGNMENT: return "CM_ERR_ALIGNMENT";
+        case CM_ERR_COLLISION: return "CM_ERR_COLLISION";
+        case CM_ERR_CUDA: return "CM_ERR_CUDA";
+        case CM_ERR_OOM: return "CM_ERR_OOM";
+        case CM_ERR_TIMEOUT: return "CM_ERR_TIMEOUT";
+        case CM_ERR_UNSUPPORTED: return "CM_ERR_UNSUPPORTED";
+    }
+    return "CM_ERR_UNKNOWN";
+}
+
+const char *cm_last_error_message(void) { return g_last_error.c_str(); }
+
+cm_status cm_context_create(int32_t device, double rope_theta, int32_t routing_layer,
+                            int32_t verify_bytes_on_hit, cm_context **out) {
+    return guarded([&]() -> cm_status {
+        if (!out) return fail(CM_ERR_INVALID_ARG, "out is NULL");
+        *out = nullptr;
+        if (device < 0) return fail(CM_ERR_INVALID_ARG, "device must be >= 0");
+        if (!(rope_theta > 0.0) || !std::isfinite(rope_theta))
+            return fail(CM_ERR_INVALID_ARG, "rope_theta must be finite and > 0");
+        int count = 0;
+        CM_CUDA_TRY(cudaGetDeviceCount(&count), "cudaGetDeviceCount");
+        if (device >= count) return fail(CM_ERR_INVALID_ARG, "no such CUDA device");
+        DeviceScope scope(device);
+        if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
+        std::unique_ptr<cm_context> ctx(new cm_context);
+        ctx->device = device;
+        ctx->theta = rope_theta;
+        ctx->routing_layer = routing_layer;
+        ctx->verify = verify_bytes_on_hit != 0;
+        CM_CUDA_TRY(cudaDeviceGetAttribute(&ctx->num_sms, cudaDevAttrMultiProcessorCount, device),
+                    "multiprocessor count");
+        CM_CUDA_TRY(cm::render_blocks_per_sm(&ctx->render_blocks_per_sm), "render occupancy");
+        if (ctx->render_blocks_per_sm < 1) ctx->render_blocks_per_sm = 1;
+        *out = ctx.release();
+        return CM_OK;
+    });
+}
+
+cm_status cm_context_destroy(cm_context *ctx) {
+    if (!ctx) return CM_OK;
+    return guarded([&]() -> cm_status {
+        if (ctx->live_sets != 0)
+            return fail(CM_ERR_INVALID_ARG, "context still has live sets");
+        DeviceScope scope(ctx->device);
+        if (ctx->d_scratch) cudaFree(ctx->d_scratch);
+        if (ctx->h_pinned) cudaFreeHost(ctx->h_pinned);
+        delete ctx;
+        return CM_OK;
+    });
+}
+
+cm_status cm_set_create(cm_context *ctx, cm_set **out) {
+    return guarded([&]() -> cm_status {
+        if (!out) return fail(CM_ERR_INVALID_ARG, "out is NULL");
+        *out = nullptr;
+        if (!ctx) return fail(CM_ERR_INVALID_ARG, "context is NULL");
+        std::lock_guard<std::mutex> lock(ctx->mu);
+        cm_set *s = new cm_set;
+        s->ctx = ctx;
+        ++ctx->live_sets;
+        *out = s;
+        return CM_OK;
+    });
+}
+
+cm_status cm_set_destroy(cm_set *set) {
+    if (!set) return CM_OK;
+    return guarded([&]() -> cm_status {
+        {
+            std::lock_guard<std::mutex> lock(set->ctx->mu);
+            --set->ctx->live_sets;
+        }
+        delete set;
+        return CM_OK;
+    });
+}
+
+cm_status cm_fragment_id(cm_context *ctx, const cm_fragment *frag, cm_stream_t stream,
+                         cm_id *out_id, uint64_t *out_norm_key) {
+    return guarded([&]() -> cm_status {
+        if (!ctx) return fail(CM_ERR_INVALID_ARG, "context is NULL");
+        if (!out_id) return fail(CM_ERR_INVALID_ARG, "out_id is NULL");
+        cm_status st = validate_fragment(frag);
+        if (st != CM_OK) return st;
+        if (routing_layer_for(ctx, frag->num_layers) >= frag->num_layers)
+            return fail(CM_ERR_INVALID_ARG, "routing layer >= num_layers");
+        std::lock_guard<std::mutex> lock(ctx->mu);
+        DeviceScope scope(ctx->device);
+        if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
+        std::vector<uint64_t> Q;
+        st = fragment_digest(ctx, frag, reinterpret_cast<cudaStream_t>(stream), out_id,
+                             out_norm_key ? &Q : nullptr);
+        if (st != CM_OK) return st;
+        if (out_norm_key) std::memcpy(out_norm_key, Q.data(), Q.size() * sizeof(uint64_t));
+        return CM_OK;
+    });
+}
+
+cm_status cm_ingest(cm_set *set, const cm_fragment *frag, cm_stream_t stream, cm_id *out_id,
+                    int32_t *out_absorbed) {
+    return guarded([&]() -> cm_status {
+        if (!set) return fail(CM_ERR_INVALID_ARG, "set is NULL");
+        cm_status st = validate_fragment(frag);
+        if (st != CM_OK) return st;
+        cm_context *ctx = set->ctx;
+        if (set->has_shape && (frag->num_layers != set->L || frag->num_kv_heads != set->H ||
+                               frag->head_dim != set->d))
+            return fail(CM_ERR_SHAPE_MISMATCH,
+                        "fragment (layers, kv_heads, head_dim) differ from the set's");
+        if (routing_layer_for(ctx, frag->num_layers) >= frag->num_layers)
+            return fail(CM_ERR_INVALID_ARG, "routing layer >= num_layers");
+        std::lock_guard<std::mutex> lock(ctx->mu);
+        DeviceScope scope(ctx->device);
+        if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
+        const cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+        auto rec = std::make_shared<Record>();
+        st = fragment_digest(ctx, frag, cs, &rec->id, &rec->Q);
+        if (st != CM_OK) return st;
+        if (out_id) *out_id = rec->id;
+        const IdKey key = key_of(rec->id);
+        auto it = set->items.find(key);
+        if (it != set->items.end()) {
+            if (ctx->verify) {
+                bool equal = false;
+                st = bytes_equal(ctx, frag, *it->second, cs, &equal);
+                if (st != CM_OK) return st;
+                if (!equal)
+                    return fail(CM_ERR_COLLISION, "content address hit with different bytes");
+            }
+            if (out_absorbed) *out_absorbed = 1;
+            return CM_OK;
+        }
+        rec->L = frag->num_layers;
+        rec->H = frag->num_kv_heads;
+        rec->T = frag->seq_len;
+        rec->d = frag->head_dim;
+        rec->k = frag->k;
+        rec->v = frag->v;
+        set->items.emplace(key, std::move(rec));
+        if (!set->has_shape) {
+            set->has_shape = true;
+            set->L = frag->num_layers;
+            set->H = frag->num_kv_heads;
+            set->d = frag->head_dim;
+        }
+        if (out_absorbed) *out_absorbed = 0;
+        return CM_OK;
+    });
+}
+
+cm_status cm_union(cm_set *dst, const cm_set *src) {
+    return guarded([&]() -> cm_status {
+        if (!dst || !src) return fail(CM_ERR_INVALID_ARG, "set is NULL");
+        if (dst == src) return CM_OK;
+        if (dst->ctx != src->ctx)
+            return fail(CM_ERR_INVALID_ARG, "sets belong to different contexts");
+        if (dst->has_shape && src->has_shape &&
+            (dst->L != src->L || dst->H != src->H || dst->d != src->d))
+            return fail(CM_ERR_SHAPE_MISMATCH, "sets have different shapes");
+        for (const auto &kv : src->items) dst->items.emplace(kv.first, kv.second);
+        if (!dst->has_shape && src->has_shape) {
+            dst->has_shape = true;
+            dst->L = src->L;
+            dst->H = src->H;
+            dst->d = src->d;
+        }
+        return CM_OK;
+    });
+}
+
+cm_status cm_set_size(const cm_set *set, int64_t *out) {
+    if (!set || !out) return fail(CM_ERR_INVALID_ARG, "set or out is NULL");
+    *out = (int64_t)set->items.size();
+    return CM_OK;
+}
+
+cm_status cm_set_seq_len(const cm_set *set, int64_t *out) {
+    if (!set || !out) return fail(CM_ERR_INVALID_ARG, "set or out is NULL");
+    int64_t total = 0;
+    for (const auto &kv : set->items) total += kv.second->T;
+    *out = total;
+    return CM_OK;
+}
+
+cm_status cm_set_ids(const cm_set *set, cm_id *out, int64_t capacity) {
+    if (!set) return fail(CM_ERR_INVALID_ARG, "set is NULL");
+    if (capacity > 0 && !out) return fail(CM_ERR_INVALID_ARG, "out is NULL");
+    int64_t i = 0;
+    for (const auto &kv : set->items) {
+        if (i >= capacity) break;
+        out[i++] = kv.second->id;
+    }
+    return CM_OK;
+}
+
+cm_status cm_render(const cm_set *set, void *k_out, void *v_out, int64_t capacity_tokens,
+                    cm_stream_t stream, int64_t *out_seq_len, cm_id *out_order) {
+    return guarded([&]() -> cm_status {
+        if (!set) return fail(CM_ERR_INVALID_ARG, "set is NULL");
+        if (capacity_tokens < 0) return fail(CM_ERR_INVALID_ARG, "capacity_tokens < 0");
+        int64_t total = 0;
+        for (const auto &kv : set->items) total += kv.second->T;
+        cm_status st = validate_outputs(k_out, v_out, capacity_tokens, total);
+        if (st != CM_OK) return st;
+        const auto order = canonical_order(set);
+        if (out_seq_len) *out_seq_len = total;
+        if (out_order)
+            for (size_t i = 0; i < order.size(); ++i) out_order[i] = order[i]->id;
+        if (order.empty()) return CM_OK;
+        std::vector<Slot> slots;
+        slots.reserve(order.size());
+        int64_t s = 0;
+        for (const auto &r : order) {
+            slots.push_back({r->k, r->v, r->T, s});
+            s += r->T;
+        }
+        cm_context *ctx = set->ctx;
+        std::lock_guard<std::mutex> lock(ctx->mu);
+        DeviceScope scope(ctx->device);
+        if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
+        return launch_slots(ctx, slots, set->L, set->H, set->d, k_out, v_out, capacity_tokens,
+                            reinterpret_cast<cudaStream_t>(stream));
+    });
+}
+
+cm_status cm_bagmerge(cm_context *ctx, const cm_fragment *frags, int32_t n, void *k_out,
+                      void *v_out, int64_t capacity_tokens, cm_stream_t stream,
+                      int64_t *out_seq_len) {
+    return guarded([&]() -> cm_status {
+        if (!ctx) return fail(CM_ERR_INVALID_ARG, "context is NULL");
+        if (!frags || n < 1) return fail(CM_ERR_INVALID_ARG, "need n >= 1 fragments");
+        if (capacity_tokens < 0) return fail(CM_ERR_INVALID_ARG, "capacity_tokens < 0");
+        int64_t total = 0;
+        for (int32_t i = 0; i < n; ++i) {
+            cm_status st = validate_fragment(&frags[i]);
+            if (st != CM_OK) return st;
+            if (frags[i].num_layers != frags[0].num_layers ||
+                frags[i].num_kv_heads != frags[0].num_kv_heads ||
+                frags[i].head_dim != frags[0].head_dim)
+                return fail(CM_ERR_SHAPE_MISMATCH, "fragments have different shapes");
+            total += frags[i].seq_len;
+        }
+        cm_status st = validate_outputs(k_out, v_out, capacity_tokens, total);
+        if (st != CM_OK) return st;
+        std::vector<Slot> slots;
+        int64_t s = 0;
+        for (int32_t i = 0; i < n; ++i) {
+            slots.push_back({frags[i].k, frags[i].v, frags[i].seq_len, s});
+            s += frags[i].seq_len;
+        }
+        if (out_seq_len) *out_seq_len = total;
+        std::lock_guard<std::mutex> lock(ctx->mu);
+        DeviceScope scope(ctx->device);
+        if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
+        return launch_slots(ctx, slots, frags[0].num_layers, frags[0].num_kv_heads,
+                            frags[0].head_dim, k_out, v_out, capacity_tokens,
+                            reinterpret_cast<cudaStream_t>(stream));
+    });
+}
+
+}  // extern "C"

@@ -1,0 +1,88 @@
+// Internal interface between the host core (cm_host.cpp) and the CUDA kernels
+// (blake2s_tree.cu, render.cu). Not part of the public ABI.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+namespace cm {
+
+// ---------------------------------------------------------------- content address
+// BLAKE2s tree mode (RFC 7693 compression; tree parameters of the BLAKE2 paper):
+// 1024-byte leaves, fanout 128, 16-byte node digests.
+constexpr int kDigestBytes = 16;
+constexpr int kLeafBytes = 1024;
+constexpr int kFanout = 128;
+
+// Chaining value a node starts from: IV xor the 32-byte parameter block with the
+// node offset and node depth fields zero. Kernels xor in offset and depth.
+struct TreeParams {
+    uint32_t h_base[8];
+};
+
+struct LeafLaunch {
+    const uint8_t *k;              // fragment K, device
+    const uint8_t *v;              // fragment V, device
+    uint64_t plane_bytes;          // bytes of one layer of K (= of V): H*T*d*2
+    uint64_t stream_bytes;         // 2 * L * plane_bytes
+    uint64_t num_leaves;           // ceil(stream_bytes / 1024)
+    uint64_t norm_begin;           // stream offset of K[l*]; its length is plane_bytes
+    uint32_t row_bytes;            // d*2; a power of two <= 1024, so rows never straddle leaves
+    uint32_t seq_len;              // T
+    unsigned long long *norm_key;  // Q[T] accumulators, zeroed before the launch
+    uint8_t *digests;              // num_leaves * 16 bytes out
+    TreeParams tree;
+};
+
+// Level 0: one thread per leaf; also accumulates the routing-layer norm key.
+cudaError_t launch_leaf_hash(const LeafLaunch &a, cudaStream_t stream);
+
+// Level `depth` >= 1: node j hashes the digests of children [128 j, 128 j + 128).
+cudaError_t launch_inner_hash(const uint8_t *children, uint64_t num_children, uint8_t *out,
+                              uint64_t num_nodes, uint32_t depth, const TreeParams &tree,
+                              cudaStream_t stream);
+
+// *flag |= 1 if the `bytes` bytes at a and b differ (16-byte aligned, bytes % 16 == 0).
+cudaError_t launch_compare(const void *a, const void *b, uint64_t bytes, unsigned int *flag,
+                           cudaStream_t stream);
+
+// ---------------------------------------------------------------- render
+constexpr int kMaxSlots = 32;          // fragments per render launch
+constexpr int kMaxTablePairs = 1792;   // sum over slots of head_dim / 2
+constexpr int kChunkBytes = 32768;     // bytes of one source plane handled per work item
+
+struct RenderSlot {
+    const void *k;              // source K [L][H][T][d], device
+    const void *v;              // source V
+    int64_t seq_len;            // T
+    int64_t offset;             // s: first output position of this slot
+    uint32_t chunk_begin;       // first global work item of this slot
+    uint32_t chunks_per_plane;  // ceil(T / rows_per_chunk)
+    int32_t rotate;             // 0: K is copied as bytes (offset 0)
+    int32_t table_base;         // index of (cos, sin)[j = 0] of this slot in cs[]
+};
+
+// Passed by value (kernel parameter space, < 32 KiB), so a launch owns its table.
+struct RenderParams {
+    void *k_out;                // [L][H][capacity][d], device
+    void *v_out;
+    int64_t capacity;
+    int32_t num_layers;
+    int32_t num_heads;
+    int32_t head_dim;
+    int32_t num_slots;
+    int32_t rows_per_chunk;     // kChunkBytes / (2 d)
+    int32_t log2_pairs_per_row; // log2(d / 16)
+    uint32_t total_chunks;
+    uint32_t pad_;
+    RenderSlot slot[kMaxSlots];
+    double cs[2 * kMaxTablePairs];   // (cos a, sin a) of a = s * theta^(-2j/d), interleaved
+};
+
+cudaError_t launch_render(const RenderParams &p, int grid, cudaStream_t stream);
+int render_threads_per_block();
+cudaError_t render_blocks_per_sm(int *out);
+
+}  // namespace cm

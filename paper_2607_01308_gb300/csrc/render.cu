@@ -1,0 +1,234 @@
+// Render: BagMerge with RoPE re-encoding (Section 4.2, Eq. bagmerge-k /
+// bagmerge-v) in a given slot order; CanonicalMerge (Algorithm 1) is this with
+// the canonical order computed on the host.
+//
+// Every (slot, layer, head) plane of K and of V is a contiguous run of T rows of
+// head_dim bf16 in the source and a contiguous run at row offset s of the output
+// plane, so the render is a set of streaming copies. V and the K of the slot at
+// offset 0 are copied as bytes. Every other K row is rotated by R(s): the stored
+// key is R(t) k, and R(s) R(0)^-1 R(t) k = R(s + t) k, so a slot's whole K is
+// turned by one constant angle a_j = s * theta^(-2j/d) per frequency j (the delta
+// formula of Section 2.3), pairing element j with element j + d/2.
+//
+// Work item: 32 KiB of one source plane; a persistent grid walks the items.
+// A thread holds whole 16-byte vectors: for K it loads vector v of the row's first
+// half and vector v of its second half, i.e. 8 (x, y) pairs that share the
+// thread's 8 (cos, sin) values for the whole item.
+//
+// Rounding. The result must equal round-to-nearest-even-bf16 of
+// fl64(fl64(x c) - fl64(y s)) (and fl64(fl64(y c) + fl64(x s))), c and s the fp64
+// cosine and sine. The fast path computes z in fp32 with one fma from c and s
+// rounded to fp32 and bounds its distance to the fp64 value by
+// E = 2^-22 (|z| + |x| + |y|) + 2^-146. If z - E and z + E (rounded outward) round
+// to the same bf16, every value between them does (rounding is monotone), the fp64
+// value included, and z's rounding is the answer. Otherwise (about one element in
+// several thousand) the element is recomputed in fp64 with the same operation
+// sequence and rounded directly to bf16, so the output is bit-exact either way.
+#include "cm_kernels.h"
+
+namespace cm {
+namespace {
+
+constexpr int kThreads = 256;
+static_assert(sizeof(RenderParams) <= 32764, "render parameters exceed the kernel parameter limit");
+
+__device__ __forceinline__ uint4 ld_stream(const uint4 *p) { return __ldcs(p); }
+__device__ __forceinline__ void st_stream(uint4 *p, const uint4 &v) { __stcs(p, v); }
+
+// Two fp32 -> bf16 round-to-nearest-even, `lo` in bits 0..15, `hi` in bits 16..31.
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+// fp64 -> bf16 bits, round to nearest, ties to even, with bf16 subnormals and
+// overflow to infinity; NaN -> 0x7FC0.
+__device__ uint32_t f64_to_bf16_bits(double z) {
+    const unsigned long long u = (unsigned long long)__double_as_longlong(z);
+    const uint32_t sign = (uint32_t)(u >> 48) & 0x8000u;
+    const unsigned long long mag = u & 0x7FFFFFFFFFFFFFFFull;
+    if (mag > 0x7FF0000000000000ull) return 0x7FC0u;
+    if (mag == 0x7FF0000000000000ull) return sign | 0x7F80u;
+    const double a = __longlong_as_double((long long)mag);
+    if (a < 0x1p-126) {
+        // spacing 2^-133 below the normal range; the count 128 is the smallest normal
+        return sign | (uint32_t)rint(a * 0x1p133);
+    }
+    // keep 7 of the 52 stored significand bits: add half an ulp minus one, plus
+    // the kept lsb (ties to even); a carry moves into the exponent field
+    const unsigned long long r = (mag + 0x00000FFFFFFFFFFFull + ((mag >> 45) & 1ull)) >> 45;
+    const int e = (int)(r >> 7) - 1023 + 127;
+    if (e >= 255) return sign | 0x7F80u;
+    return sign | ((uint32_t)e << 7) | (uint32_t)(r & 0x7Fu);
+}
+
+__device__ __forceinline__ float err_bound(float z, float xy_abs) {
+    return __fmaf_ru(__fadd_ru(fabsf(z), xy_abs), 0x1p-22f, 0x1p-146f);
+}
+
+// Rotate the pairs (x0, y0), (x1, y1) held in word xw (x0 low, x1 high) and word yw.
+// Returns the rotated words and a mask whose nonzero 16-bit halves mark elements
+// whose fp32 result is not certified.
+__device__ __forceinline__ void rotate_word(uint32_t xw, uint32_t yw, float c0, float s0, float c1,
+                                            float s1, uint32_t &xo, uint32_t &yo, uint32_t &bad) {
+    const float x0 = bf16_lo(xw), x1 = bf16_hi(xw);
+    const float y0 = bf16_lo(yw), y1 = bf16_hi(yw);
+    const float zx0 = __fmaf_rn(x0, c0, -__fmul_rn(y0, s0));
+    const float zx1 = __fmaf_rn(x1, c1, -__fmul_rn(y1, s1));
+    const float zy0 = __fmaf_rn(y0, c0, __fmul_rn(x0, s0));
+    const float zy1 = __fmaf_rn(y1, c1, __fmul_rn(x1, s1));
+    const float m0 = __fadd_ru(fabsf(x0), fabsf(y0));
+    const float m1 = __fadd_ru(fabsf(x1), fabsf(y1));
+    const float ex0 = err_bound(zx0, m0), ex1 = err_bound(zx1, m1);
+    const float ey0 = err_bound(zy0, m0), ey1 = err_bound(zy1, m1);
+    const uint32_t bx = pack_bf16x2(__fsub_rd(zx0, ex0), __fsub_rd(zx1, ex1)) ^
+                        pack_bf16x2(__fadd_ru(zx0, ex0), __fadd_ru(zx1, ex1));
+    const uint32_t by = pack_bf16x2(__fsub_rd(zy0, ey0), __fsub_rd(zy1, ey1)) ^
+                        pack_bf16x2(__fadd_ru(zy0, ey0), __fadd_ru(zy1, ey1));
+    xo = pack_bf16x2(zx0, zx1);
+    yo = pack_bf16x2(zy0, zy1);
+    bad = bx | by;
+}
+
+__device__ __forceinline__ uint32_t set_half(uint32_t w, int half, uint32_t bits) {
+    return half ? (w & 0x0000FFFFu) | (bits << 16) : (w & 0xFFFF0000u) | bits;
+}
+
+// Exact recomputation of the uncertified elements of one vector pair.
+__device__ __noinline__ void fixup_pair(const RenderParams &p, int cs_index, const uint4 &a,
+                                        const uint4 &b, uint4 &ao, uint4 &bo) {
+    const uint32_t xi[4] = {a.x, a.y, a.z, a.w};
+    const uint32_t yi[4] = {b.x, b.y, b.z, b.w};
+    uint32_t xo[4] = {ao.x, ao.y, ao.z, ao.w};
+    uint32_t yo[4] = {bo.x, bo.y, bo.z, bo.w};
+    for (int e = 0; e < 8; ++e) {
+        const int w = e >> 1, half = e & 1;
+        const double x = (double)(half ? bf16_hi(xi[w]) : bf16_lo(xi[w]));
+        const double y = (double)(half ? bf16_hi(yi[w]) : bf16_lo(yi[w]));
+        const double c = p.cs[2 * (cs_index + e)];
+        const double s = p.cs[2 * (cs_index + e) + 1];
+        const double zx = __dsub_rn(__dmul_rn(x, c), __dmul_rn(y, s));
+        const double zy = __dadd_rn(__dmul_rn(y, c), __dmul_rn(x, s));
+        xo[w] = set_half(xo[w], half, f64_to_bf16_bits(zx));
+        yo[w] = set_half(yo[w], half, f64_to_bf16_bits(zy));
+    }
+    ao = make_uint4(xo[0], xo[1], xo[2], xo[3]);
+    bo = make_uint4(yo[0], yo[1], yo[2], yo[3]);
+}
+
+__device__ __forceinline__ void copy_item(const uint4 *__restrict__ src, uint4 *__restrict__ dst,
+                                          int n_vec) {
+    constexpr int kU = kChunkBytes / 16 / kThreads;   // 8 vectors per thread
+    uint4 r[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+        const int i = threadIdx.x + u * kThreads;
+        if (i < n_vec) r[u] = ld_stream(src + i);
+    }
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+        const int i = threadIdx.x + u * kThreads;
+        if (i < n_vec) st_stream(dst + i, r[u]);
+    }
+}
+
+__device__ __forceinline__ void rotate_item(const RenderParams &p, const float2 *cs32, int cs_index,
+                                            const uint4 *__restrict__ src,
+                                            uint4 *__restrict__ dst, int rows, int lane_v) {
+    constexpr int kU = kChunkBytes / 32 / kThreads;   // 4 vector pairs per thread
+    const int vecs_per_row = p.head_dim >> 3;
+    const int half_vecs = p.head_dim >> 4;
+    const int n_pairs = rows * half_vecs;
+    uint4 a[kU], b[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+        const int q = threadIdx.x + u * kThreads;
+        if (q < n_pairs) {
+            const int row = q >> p.log2_pairs_per_row;
+            const uint4 *r = src + (int64_t)row * vecs_per_row + lane_v;
+            a[u] = ld_stream(r);
+            b[u] = ld_stream(r + half_vecs);
+        }
+    }
+    float c[8], s[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        const float2 t = cs32[cs_index + e];
+        c[e] = t.x;
+        s[e] = t.y;
+    }
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+        const int q = threadIdx.x + u * kThreads;
+        if (q < n_pairs) {
+            uint4 ao, bo;
+            uint32_t b0, b1, b2, b3;
+            rotate_word(a[u].x, b[u].x, c[0], s[0], c[1], s[1], ao.x, bo.x, b0);
+            rotate_word(a[u].y, b[u].y, c[2], s[2], c[3], s[3], ao.y, bo.y, b1);
+            rotate_word(a[u].z, b[u].z, c[4], s[4], c[5], s[5], ao.z, bo.z, b2);
+            rotate_word(a[u].w, b[u].w, c[6], s[6], c[7], s[7], ao.w, bo.w, b3);
+            if ((b0 | b1 | b2 | b3) != 0u) fixup_pair(p, cs_index, a[u], b[u], ao, bo);
+            const int row = q >> p.log2_pairs_per_row;
+            uint4 *r = dst + (int64_t)row * vecs_per_row + lane_v;
+            st_stream(r, ao);
+            st_stream(r + half_vecs, bo);
+        }
+    }
+}
+
+__global__ void __launch_bounds__(kThreads)
+render_kernel(const __grid_constant__ RenderParams p) {
+    __shared__ float2 cs32[kMaxTablePairs];
+    const int half = p.head_dim >> 1;
+    const int n_table = p.num_slots * half;
+    for (int i = threadIdx.x; i < n_table; i += kThreads)
+        cs32[i] = make_float2(__double2float_rn(p.cs[2 * i]), __double2float_rn(p.cs[2 * i + 1]));
+    __syncthreads();
+
+    const int vecs_per_row = p.head_dim >> 3;
+    const int lane_v = threadIdx.x & ((p.head_dim >> 4) - 1);
+    const uint32_t lh_planes = (uint32_t)p.num_layers * (uint32_t)p.num_heads;
+
+    for (uint32_t g = blockIdx.x; g < p.total_chunks; g += gridDim.x) {
+        int si = 0;
+        while (si + 1 < p.num_slots && g >= p.slot[si + 1].chunk_begin) ++si;
+        const RenderSlot &S = p.slot[si];
+        const uint32_t local = g - S.chunk_begin;
+        const uint32_t plane = local / S.chunks_per_plane;
+        const uint32_t c = local - plane * S.chunks_per_plane;
+        const bool is_v = plane >= lh_planes;       // K planes first, then V planes
+        const int64_t lh = is_v ? plane - lh_planes : plane;
+        const int64_t row0 = (int64_t)c * p.rows_per_chunk;
+        const int64_t left = S.seq_len - row0;
+        const int rows = left < p.rows_per_chunk ? (int)left : p.rows_per_chunk;
+        const uint4 *src = static_cast<const uint4 *>(is_v ? S.v : S.k) +
+                           (lh * S.seq_len + row0) * vecs_per_row;
+        uint4 *dst = static_cast<uint4 *>(is_v ? p.v_out : p.k_out) +
+                     (lh * p.capacity + S.offset + row0) * vecs_per_row;
+        if (is_v || !S.rotate) {
+            copy_item(src, dst, rows * vecs_per_row);
+        } else {
+            rotate_item(p, cs32, S.table_base + 8 * lane_v, src, dst, rows, lane_v);
+        }
+    }
+}
+
+}  // namespace
+
+int render_threads_per_block() { return kThreads; }
+
+cudaError_t render_blocks_per_sm(int *out) {
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, render_kernel, kThreads, 0);
+}
+
+cudaError_t launch_render(const RenderParams &p, int grid, cudaStream_t stream) {
+    if (p.total_chunks == 0) return cudaSuccess;
+    render_kernel<<<grid, kThreads, 0, stream>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace cm

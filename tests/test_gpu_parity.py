@@ -1,0 +1,276 @@
+"""GPU parity: the CUDA library through its C ABI against the CPU oracle.
+
+Bar: content addresses, norm keys, set membership, canonical order and V are
+bit-exact; K is within 1 bf16 ulp per element (the non-exact count is also
+asserted to be 0: the kernel certifies its fp32 rounding and recomputes the
+rest in fp64 exactly as the oracle does). Every render is also byte-identical
+across all delivery orders of its set.
+"""
+import itertools
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synthetic
+from parity_util import THETA, assert_k_parity, empty_out, gpu_fragments, oracle_fragment
+
+pytestmark = pytest.mark.gpu
+
+cm = pytest.importorskip("paper_2607_01308_gb300")
+
+
+@pytest.fixture(scope="module")
+def ctx():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    c = cm.Context(0, THETA)
+    yield c
+    c.close()
+
+
+def _render(ctx, deliveries, cap=None, fill=None):
+    S = cm.FragmentSet(ctx)
+    absorbed = [S.ingest(K, V)[1] for K, V in deliveries]
+    K0 = deliveries[0][0]
+    L, H, _, d = K0.shape
+    total = S.seq_len()
+    k_out, v_out = empty_out(L, H, cap or max(total, 1), d, fill=fill)
+    n, order = S.render(k_out, v_out)
+    torch.cuda.synchronize()
+    S.close()
+    return k_out, v_out, n, order, absorbed
+
+
+# ---------------------------------------------------------------- content address + norm key
+
+ID_SHAPES = [(4, 2, 37, 64), (4, 2, 53, 64), (1, 1, 1, 16), (2, 3, 1, 512), (3, 1, 5, 16),
+             (2, 2, 33, 32), (5, 2, 7, 256), (28, 8, 9, 128), (1, 1, 300, 128)]
+
+
+@pytest.mark.parametrize("shape", ID_SHAPES)
+def test_fragment_id_and_norm_key_match_oracle(ctx, shape):
+    L, H, T, d = shape
+    g = torch.Generator(device="cuda:0").manual_seed(sum(shape))
+    K = (torch.randn(shape, generator=g, device="cuda:0") * 1.3).to(torch.bfloat16)
+    V = torch.randn(shape, generator=g, device="cuda:0").to(torch.bfloat16)
+    fid, Q = ctx.fragment_id(K, V)
+    ref = oracle_fragment(K, V)
+    assert fid == ref.fid
+    assert np.array_equal(np.array(Q, dtype=np.uint64), ref.Q)
+
+
+def test_norm_key_special_values(ctx):
+    L, H, T, d = 2, 2, 6, 16
+    K = torch.zeros((L, H, T, d), dtype=torch.bfloat16, device="cuda:0")
+    V = torch.zeros_like(K)
+    Kb = K.view(torch.int16)
+    Kb[1, 0, 0, :] = 0x7F7F           # largest finite: saturates
+    Kb[1, 0, 1, 3] = 0x7FC0           # NaN: saturates
+    Kb[1, 1, 2, 5] = -0x8000 + 0x0001  # negative subnormal (0x8001)
+    Kb[1, 1, 3, :] = 0x3F80           # ones: norm 4
+    fid, Q = ctx.fragment_id(K, V)
+    ref = oracle_fragment(K, V)
+    assert fid == ref.fid
+    assert np.array_equal(np.array(Q, dtype=np.uint64), ref.Q)
+
+
+# ---------------------------------------------------------------- tiny workload: every order
+
+def test_tiny_all_delivery_orders_match_oracle(ctx):
+    w, frags, sched = gpu_fragments("tiny")
+    msgs = [(frags[i][0].clone(), frags[i][1].clone()) for i in sched]
+    ref_frags = [oracle_fragment(K, V) for K, V in frags]
+    K_ref, V_ref, o_order = oracle.render(oracle.from_deliveries(ref_frags), THETA)
+    first = None
+    for perm in itertools.permutations(range(len(msgs))):
+        k_out, v_out, n, order, absorbed = _render(ctx, [msgs[i] for i in perm])
+        assert sum(absorbed) == 1 and n == K_ref.shape[2] == 37 + 53
+        assert order == [f.fid for f in o_order]
+        kb, vb = synthetic.to_bits(k_out), synthetic.to_bits(v_out)
+        assert np.array_equal(vb, V_ref)
+        assert assert_k_parity(kb, K_ref) == 0
+        if first is None:
+            first = (kb, vb)
+        assert np.array_equal(kb, first[0]) and np.array_equal(vb, first[1])
+
+
+# ---------------------------------------------------------------- Qwen3-1.7B shaped, N = 2
+
+def test_q17_n2_full_parity(ctx):
+    w, frags, sched = gpu_fragments("q17_n2")
+    ref_frags = [oracle_fragment(K, V) for K, V in frags]
+    K_ref, V_ref, o_order = oracle.render(oracle.from_deliveries(ref_frags), THETA)
+    results = []
+    for perm in itertools.permutations(range(2)):
+        k_out, v_out, n, order, absorbed = _render(ctx, [frags[i] for i in perm])
+        assert n == 1024 and order == [f.fid for f in o_order] and not any(absorbed)
+        results.append((synthetic.to_bits(k_out), synthetic.to_bits(v_out)))
+    kb, vb = results[0]
+    assert np.array_equal(vb, V_ref)
+    assert assert_k_parity(kb, K_ref) == 0
+    assert np.array_equal(results[1][0], kb) and np.array_equal(results[1][1], vb)
+
+
+# ---------------------------------------------------------------- rounding edge cases
+
+def test_rotation_of_special_values_matches_oracle(ctx):
+    L, H, T, d = 1, 2, 64, 128
+    rng = np.random.default_rng(3)
+    bits = rng.integers(0, 1 << 16, size=(L, H, T, d), dtype=np.uint64).astype(np.uint16)
+    # avoid NaN payload patterns, keep +-inf, +-0, subnormals, the largest finites
+    nan = ((bits & 0x7F80) == 0x7F80) & ((bits & 0x7F) != 0)
+    bits[nan] = 0x3F80
+    bits[0, 0, 0, :8] = [0x0000, 0x8000, 0x0001, 0x8001, 0x007F, 0x7F7F, 0xFF7F, 0x7F80]
+    bits[0, 0, 0, 64:72] = [0x8000, 0x0000, 0x0001, 0x0002, 0x807F, 0x7F7F, 0x7F7F, 0x3F80]
+    bits[0, 1, :, :] = (bits[0, 1, :, :] & 0x80FF) | 0x0000   # many subnormals
+    base = torch.from_numpy(bits.view(np.int16)).to("cuda:0").view(torch.bfloat16)
+    lead = torch.zeros((L, H, 1000, d), dtype=torch.bfloat16, device="cuda:0")
+    frags = [(lead, lead.clone()), (base.contiguous(), base.clone())]
+    k_out, v_out = empty_out(L, H, 1000 + T, d)
+    n = ctx.bagmerge(frags, k_out, v_out)
+    torch.cuda.synchronize()
+    assert n == 1000 + T
+    ref = oracle.rotate_k(bits, 1000, THETA)
+    got = synthetic.to_bits(k_out)[:, :, 1000:]
+    assert assert_k_parity(got, ref) == 0
+
+
+# ---------------------------------------------------------------- layout, capacity, canaries
+
+@pytest.mark.parametrize("d", [16, 64, 256, 512])
+def test_render_layout_with_capacity_and_canaries(ctx, d):
+    L, H = 3, 2
+    lengths = [1, 129, 70, 600]
+    g = torch.Generator(device="cuda:0").manual_seed(d)
+    frags = []
+    for i, T in enumerate(lengths):
+        K = (torch.randn((L, H, T, d), generator=g, device="cuda:0") * (0.6 + 0.3 * i)).to(torch.bfloat16)
+        V = torch.randn((L, H, T, d), generator=g, device="cuda:0").to(torch.bfloat16)
+        frags.append((K, V))
+    total = sum(lengths)
+    cap = total + 37
+    k_out, v_out, n, order, _ = _render(ctx, frags, cap=cap, fill=0x5A5A)
+    ref_frags = [oracle_fragment(K, V) for K, V in frags]
+    K_ref, V_ref, o_order = oracle.render(oracle.from_deliveries(ref_frags), THETA)
+    assert n == total and order == [f.fid for f in o_order]
+    kb, vb = synthetic.to_bits(k_out), synthetic.to_bits(v_out)
+    assert np.array_equal(vb[:, :, :total], V_ref)
+    assert assert_k_parity(kb[:, :, :total], K_ref) == 0
+    assert (kb[:, :, total:] == 0x5A5A).all() and (vb[:, :, total:] == 0x5A5A).all()
+
+
+def test_bagmerge_explicit_order_and_naive_redelivery(ctx):
+    w, frags, _ = gpu_fragments("tiny")
+    a, b = frags
+    ref = [oracle_fragment(K, V) for K, V in frags]
+    for order_idx in ([0, 1], [1, 0], [0, 1, 0, 1, 0, 1]):
+        seq = [frags[i] for i in order_idx]
+        L, H, _, d = a[0].shape
+        total = sum(f[0].shape[2] for f in seq)
+        k_out, v_out = empty_out(L, H, total, d)
+        n = ctx.bagmerge(seq, k_out, v_out)
+        torch.cuda.synchronize()
+        K_ref, V_ref = oracle.bagmerge([ref[i] for i in order_idx], THETA)
+        assert n == total
+        assert np.array_equal(synthetic.to_bits(v_out), V_ref)
+        assert assert_k_parity(synthetic.to_bits(k_out), K_ref) == 0
+
+
+def test_empty_set_renders_nothing(ctx):
+    S = cm.FragmentSet(ctx)
+    n, order = cm.cm_render(S.handle, 0, 0, 0)
+    assert n == 0 and order == []
+    S.close()
+
+
+# ---------------------------------------------------------------- ABI errors on the GPU path
+
+def test_abi_errors(ctx):
+    g = torch.Generator(device="cuda:0").manual_seed(1)
+    K = torch.randn((2, 2, 8, 64), generator=g, device="cuda:0").to(torch.bfloat16)
+    V = torch.randn((2, 2, 8, 64), generator=g, device="cuda:0").to(torch.bfloat16)
+    S = cm.FragmentSet(ctx)
+    S.ingest(K, V)
+    K2 = torch.zeros((2, 2, 8, 32), dtype=torch.bfloat16, device="cuda:0")
+    with pytest.raises(cm.CMError) as e:
+        S.ingest(K2, K2.clone())
+    assert e.value.status == cm.Status.ERR_SHAPE_MISMATCH
+    # odd head_dim / not a power of two
+    bad = cm.cm_fragment(2, 2, 8, 48, K.data_ptr(), V.data_ptr())
+    with pytest.raises(cm.CMError) as e:
+        cm.cm_ingest(S.handle, bad)
+    assert e.value.status == cm.Status.ERR_INVALID_ARG
+    # misaligned pointer
+    mis = cm.cm_fragment(2, 2, 8, 64, K.data_ptr() + 2, V.data_ptr())
+    with pytest.raises(cm.CMError) as e:
+        cm.cm_ingest(S.handle, mis)
+    assert e.value.status == cm.Status.ERR_ALIGNMENT
+    # capacity too small
+    k_out, v_out = empty_out(2, 2, 7, 64)
+    with pytest.raises(cm.CMError) as e:
+        S.render(k_out, v_out)
+    assert e.value.status == cm.Status.ERR_CAPACITY
+    # union across contexts
+    other = cm.Context(0, THETA)
+    S2 = cm.FragmentSet(other)
+    with pytest.raises(cm.CMError) as e:
+        S.union(S2)
+    assert e.value.status == cm.Status.ERR_INVALID_ARG
+    S2.close()
+    other.close()
+    # routing layer out of range
+    c3 = cm.Context(0, THETA, routing_layer=5)
+    with pytest.raises(cm.CMError) as e:
+        c3.fragment_id(K, V)
+    assert e.value.status == cm.Status.ERR_INVALID_ARG
+    c3.close()
+    S.close()
+
+
+def test_verify_bytes_on_hit_accepts_true_duplicates(ctx):
+    c = cm.Context(0, THETA, verify_bytes_on_hit=True)
+    g = torch.Generator(device="cuda:0").manual_seed(2)
+    K = torch.randn((2, 2, 9, 64), generator=g, device="cuda:0").to(torch.bfloat16)
+    V = torch.randn((2, 2, 9, 64), generator=g, device="cuda:0").to(torch.bfloat16)
+    S = cm.FragmentSet(c)
+    assert S.ingest(K, V)[1] is False
+    assert S.ingest(K.clone(), V.clone())[1] is True
+    assert len(S) == 1
+    S.close()
+    c.close()
+
+
+# ---------------------------------------------------------------- union on the GPU-built sets
+
+def test_union_algebra_and_render_invariance(ctx):
+    w, frags, _ = gpu_fragments("q17_arity")
+    frags = [(K[:, :, :64].contiguous(), V[:, :, :64].contiguous()) for K, V in frags]
+    singles = []
+    for K, V in frags:
+        S = cm.FragmentSet(ctx)
+        S.ingest(K, V)
+        singles.append(S)
+    L, H, _, d = frags[0][0].shape
+    k0, v0 = empty_out(L, H, 64 * 5, d)
+    ref_bits = None
+    for perm in itertools.permutations(range(5)):
+        U = cm.FragmentSet(ctx)
+        for i in perm:
+            U.union(singles[i])
+        U.union(singles[perm[0]])          # idempotent / absorbing
+        assert len(U) == 5
+        n, order = U.render(k0, v0)
+        torch.cuda.synchronize()
+        kb = (synthetic.to_bits(k0), synthetic.to_bits(v0))
+        if ref_bits is None:
+            ref_bits = kb
+        assert np.array_equal(kb[0], ref_bits[0]) and np.array_equal(kb[1], ref_bits[1])
+        U.close()
+    ref_frags = [oracle_fragment(K, V) for K, V in frags]
+    K_ref, V_ref, _ = oracle.render(oracle.from_deliveries(ref_frags), THETA)
+    assert np.array_equal(ref_bits[1], V_ref)
+    assert assert_k_parity(ref_bits[0], K_ref) == 0
+    for S in singles:
+        S.close()
