@@ -1,0 +1,381 @@
+"""Benchmark of the CanonicalMerge / LatentFragmentSet hot path on GB300.
+
+One step = one whole merge of the Qwen3-4B-shaped workload (36 layers, 8 KV
+heads, head_dim 128, RoPE theta 1e6, 4 fragments x 4096 tokens, bf16):
+  replica A ingests fragments 0 and 1, replica B ingests fragments 2 and 3
+  (content address + routing-layer norm key on the GPU, membership on the host),
+  A := A u B (set union), then A is rendered (canonical order on the host, one
+  fused copy-and-rotate kernel) into a preallocated [36, 8, 16384, 128] K/V cache.
+
+Prints one JSON line: value = merges per second over the timed steps (inputs
+resident in HBM), the render kernel's achieved HBM bandwidth against the measured
+copy peak, the end-to-end rate through the C ABI with host buffers (inputs copied
+in and the merged cache copied out every step), and the CPU oracle timed on a
+bounded sample. `--impl reference` times the CPU oracle alone.
+
+Multi-GPU (torchrun): every rank runs its own merges on its own GPU (independent
+requests; no data-path collective), value = all ranks' merges / max rank time.
+"""
+from __future__ import annotations
+
+import argparse
+import csv
+import hashlib
+import io
+import json
+import os
+import re
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "cm_render merged-cache GB/s and % of HBM peak; merges/sec (ingest+union+render)"
+UNIT = "merges/s"
+WORKLOAD = "q4b"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+CLOCK_FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--e2e-steps", type=int, default=None)
+    return p.parse_args()
+
+
+def workload_config(w):
+    import synthetic
+    specs = synthetic.fragment_specs(w)
+    return {
+        "workload": "Qwen3-4B-shaped merge: 36 layers, 8 KV heads, head_dim 128, RoPE theta 1e6, "
+                    "N=4 fragments x 4096 tokens (16384 merged tokens), bf16",
+        "name": w.name, "num_layers": w.num_layers, "num_kv_heads": w.num_kv_heads,
+        "head_dim": w.head_dim, "fragments": len(specs), "seq_lens": [s.seq_len for s in specs],
+        "merged_tokens": sum(s.seq_len for s in specs), "routing_layer": w.num_layers // 2,
+        "replicas_per_merge": 2,
+        "l2": "no flush: every step streams 2.4 GB of fragments and 2.4 GB of output (> 129 MB L2)",
+    }
+
+
+# ---------------------------------------------------------------- measured peaks, clocks, profiles
+
+def hbm_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            v = float(json.load(f)["hbm_gbs"])
+        return v, "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples every 200 ms while the timed region runs."""
+
+    def __init__(self, device_index):
+        self.device_index = device_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.device_index), "--query-gpu=" + CLOCK_FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+                self.out = ""
+
+    def summary(self):
+        rows = [r for r in csv.reader(io.StringIO(getattr(self, "out", ""))) if len(r) >= 9]
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        sm = sorted(float(r[1]) for r in rows if r[1].strip().replace(".", "").isdigit())
+        mx = [float(r[2]) for r in rows if r[2].strip().replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if "Active" == r[5 + i].strip()})
+        return {"sm_mhz": sm[len(sm) // 2] if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def render_profile_traffic():
+    """DRAM bytes per render launch from the committed ncu summary, if it was taken on the
+    current render kernel source (its sha256 is recorded in the summary)."""
+    src = os.path.join(ROOT, "paper_2607_01308_gb300", "csrc", "render.cu")
+    summ = os.path.join(ROOT, "profiles", "render_kernel_q4b.md")
+    try:
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()
+        text = open(summ).read()
+        m_sha = re.search(r"render\.cu sha256:\s*([0-9a-f]{64})", text)
+        m_tr = re.search(r"dram_bytes_per_full_launch:\s*([0-9.eE+]+)", text)
+        if m_sha and m_tr and m_sha.group(1) == sha:
+            return float(m_tr.group(1))
+    except OSError:
+        pass
+    return None
+
+
+# ---------------------------------------------------------------- CPU oracle (baseline leg)
+
+def oracle_sample_seconds(layers=1, w=None):
+    """The oracle as it stands on a bounded sample of the workload: the first `layers`
+    layers of each of the 4 fragments (T = 4096), full ingest (id + norm key), union
+    and render; returns (seconds, bytes of that sample's fragments)."""
+    import numpy as np
+    import oracle
+    import synthetic
+    w = w or synthetic.WORKLOADS[WORKLOAD]
+    specs = synthetic.fragment_specs(w)
+    frags = [synthetic.make_fragment_bits(s, layers, w.num_kv_heads, w.head_dim) for s in specs]
+    t0 = time.perf_counter()
+    A = oracle.FragmentSet()
+    B = oracle.FragmentSet()
+    for i, (K, V) in enumerate(frags):
+        f = oracle.make_fragment(K, V, routing_layer=layers // 2)
+        if i < 2:
+            A = oracle.ingest(A, f)
+        else:
+            B = oracle.ingest(B, f)
+    S = oracle.union(A, B)
+    K_out, V_out, _ = oracle.render(S, synthetic.ROPE_THETA)
+    dt = time.perf_counter() - t0
+    nbytes = sum(K.nbytes + V.nbytes for K, V in frags)
+    assert K_out.shape[2] == sum(s.seq_len for s in specs)
+    return dt, nbytes
+
+
+def cpu_baseline_entry(layers=2):
+    import synthetic
+    w = synthetic.WORKLOADS[WORKLOAD]
+    dt, _ = oracle_sample_seconds(layers, w)
+    per_merge = dt * w.num_layers / layers
+    return {"value": 1.0 / per_merge, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"one merge restricted to the first {layers} of {w.num_layers} layers "
+                      f"(4 fragments x 4096 tokens; ingest + union + render), timed once "
+                      f"({dt:.2f} s) and scaled by {w.num_layers}/{layers} to a full merge; "
+                      f"single thread (numpy fp64 + hashlib)",
+            "seconds_per_merge": per_merge}
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    os.environ.setdefault("OMP_NUM_THREADS", "1")
+    import synthetic
+    w = synthetic.WORKLOADS[WORKLOAD]
+    layers = 1
+    for _ in range(args.warmup):
+        oracle_sample_seconds(layers, w)
+    total = 0.0
+    for _ in range(args.steps):
+        dt, _ = oracle_sample_seconds(layers, w)
+        total += dt * w.num_layers / layers
+    value = args.steps / total
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1000.0 * total / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u16 bits / f64", "data": "synthetic",
+        "config": workload_config(w),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": f"each step: one merge restricted to the first {layers} of "
+                                   f"{w.num_layers} layers, scaled by {w.num_layers} to a full "
+                                   f"merge; single thread"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ---------------------------------------------------------------- GPU arm
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+    import torch.distributed as dist
+
+    import paper_2607_01308_gb300 as cm
+    import synthetic
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+
+    w = synthetic.WORKLOADS[WORKLOAD]
+    L, H, d = w.num_layers, w.num_kv_heads, w.head_dim
+    specs = synthetic.fragment_specs(w)
+    frags = [synthetic.make_fragment_torch(s, L, H, d, dev) for s in specs]
+    total_T = sum(s.seq_len for s in specs)
+    k_out = torch.empty((L, H, total_T, d), dtype=torch.bfloat16, device=dev)
+    v_out = torch.empty_like(k_out)
+    ctx = cm.Context(local_rank, synthetic.ROPE_THETA)
+    stream = torch.cuda.current_stream(dev)
+    fdesc = [cm.fragment_from_tensors(K, V) for K, V in frags]
+    render_bytes = 2 * total_T * w.bytes_per_token          # read + write of all K and V
+    hash_bytes = sum(s.seq_len for s in specs) * w.bytes_per_token
+
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+
+    def one_merge(timers=None, inputs=None):
+        a = cm.cm_set_create(ctx.handle)
+        b = cm.cm_set_create(ctx.handle)
+        fd = inputs or fdesc
+        if timers is not None:
+            timers["ingest"][0].record(stream)
+        for i, f in enumerate(fd):
+            cm.cm_ingest(a if i < 2 else b, f, stream)
+        if timers is not None:
+            timers["ingest"][1].record(stream)
+        cm.cm_union(a, b)
+        if timers is not None:
+            timers["render"][0].record(stream)
+        n, _ = cm.cm_render(a, k_out.data_ptr(), v_out.data_ptr(), total_T, stream)
+        if timers is not None:
+            timers["render"][1].record(stream)
+        cm.cm_set_destroy(b)
+        cm.cm_set_destroy(a)
+        return n
+
+    for _ in range(args.warmup):
+        one_merge()
+    torch.cuda.synchronize(dev)
+
+    step_timers = [{"ingest": (ev(), ev()), "render": (ev(), ev())} for _ in range(args.steps)]
+    start, end = ev(), ev()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    with ClockSampler(local_rank) as clocks:
+        start.record(stream)
+        for i in range(args.steps):
+            one_merge(step_timers[i])
+        end.record(stream)
+        torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    elapsed_ms = start.elapsed_time(end)
+    render_ms = sum(t["render"][0].elapsed_time(t["render"][1]) for t in step_timers) / args.steps
+    ingest_ms = sum(t["ingest"][0].elapsed_time(t["ingest"][1]) for t in step_timers) / args.steps
+    if world > 1:
+        tt = torch.tensor([elapsed_ms], device=dev, dtype=torch.float64)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(tt.item())
+
+    # end to end through the C ABI with host buffers: pinned inputs copied in and the
+    # merged cache copied out inside the timed region, every step
+    e2e_steps = args.e2e_steps or min(args.steps, 10)
+    host_in = [(K.cpu().pin_memory(), V.cpu().pin_memory()) for K, V in frags]
+    dev_in = [(torch.empty_like(K), torch.empty_like(V)) for K, V in frags]
+    dev_desc = [cm.fragment_from_tensors(K, V) for K, V in dev_in]
+    host_out = (torch.empty(k_out.shape, dtype=k_out.dtype, pin_memory=True),
+                torch.empty(v_out.shape, dtype=v_out.dtype, pin_memory=True))
+    h2d = sum(K.numel() * 2 + V.numel() * 2 for K, V in host_in)
+    d2h = 2 * k_out.numel() * 2
+
+    def e2e_step():
+        for (hk, hv), (dk, dv) in zip(host_in, dev_in):
+            dk.copy_(hk, non_blocking=True)
+            dv.copy_(hv, non_blocking=True)
+        one_merge(inputs=dev_desc)
+        host_out[0].copy_(k_out, non_blocking=True)
+        host_out[1].copy_(v_out, non_blocking=True)
+
+    e2e_step()
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    e0, e1 = ev(), ev()
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_ms = e0.elapsed_time(e1)
+    if world > 1:
+        tt = torch.tensor([e2e_ms], device=dev, dtype=torch.float64)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_ms = float(tt.item())
+        dist.barrier()
+
+    if rank == 0:
+        peak, peak_src = hbm_peak()
+        render_gbs = render_bytes / (render_ms * 1e-3) / 1e9
+        ms_per_step = elapsed_ms / args.steps
+        levels = 1
+        n_leaves = -(-(w.bytes_per_token * specs[0].seq_len) // 1024)
+        while n_leaves > 1 or levels == 1:
+            n_leaves = -(-n_leaves // 128)
+            levels += 1
+        launches_per_step = len(specs) * levels + 1
+        line = {
+            "metric": METRIC,
+            "value": world * args.steps / (elapsed_ms * 1e-3),
+            "unit": UNIT,
+            "n_gpus": world,
+            "steps": args.steps,
+            "warmup": args.warmup,
+            "ms_per_step": ms_per_step,
+            "higher_is_better": True,
+            "scaling": "weak",
+            "vs_baseline": None,
+            "dtype": "bf16",
+            "data": "synthetic",
+            "config": workload_config(w),
+            "render_gbs": render_gbs,
+            "render_frac_of_measured_hbm": render_gbs / peak,
+            "render_frac_of_8tbs": render_gbs / NOMINAL_HBM_GBS,
+            "render_ms": render_ms,
+            "ingest_ms_per_merge": ingest_ms,
+            "ingest_gbs": hash_bytes / (ingest_ms * 1e-3) / 1e9,
+            "roofline": {
+                "kernel": "render_kernel", "bound": "hbm", "achieved": render_gbs, "peak": peak,
+                "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
+                else "fallback 6.8 TB/s",
+                "unit": "GB/s", "frac": render_gbs / peak, "traffic": render_profile_traffic(),
+                "algorithmic_bytes_per_launch": render_bytes,
+            },
+            "e2e": {"value": world * e2e_steps / (e2e_ms * 1e-3), "unit": UNIT,
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "gpu_launches": launches_per_step * args.steps,
+            "clocks": clocks.summary(),
+        }
+        if world == 1 and not args.no_cpu_baseline:
+            line["cpu_baseline"] = cpu_baseline_entry()
+        print(json.dumps(line), flush=True)
+    ctx.close()
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())
