@@ -51,15 +51,26 @@ def parse_args():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--e2e-steps", type=int, default=None)
+    p.add_argument("--workload", default=WORKLOAD, choices=["q4b", "q17_n2", "tiny"],
+                   help="single-request workload (q4b is the benchmark; the others are small "
+                        "cases for profiling)")
     return p.parse_args()
+
+
+WORKLOAD_TEXT = {
+    "q4b": "Qwen3-4B-shaped merge: 36 layers, 8 KV heads, head_dim 128, RoPE theta 1e6, "
+           "N=4 fragments x 4096 tokens (16384 merged tokens), bf16",
+    "q17_n2": "Qwen3-1.7B-shaped merge: 28 layers, 8 KV heads, head_dim 128, RoPE theta 1e6, "
+              "N=2 fragments x 512 tokens, bf16",
+    "tiny": "tiny merge: 4 layers, 2 KV heads, head_dim 64, fragments of 37 and 53 tokens, bf16",
+}
 
 
 def workload_config(w):
     import synthetic
     specs = synthetic.fragment_specs(w)
     return {
-        "workload": "Qwen3-4B-shaped merge: 36 layers, 8 KV heads, head_dim 128, RoPE theta 1e6, "
-                    "N=4 fragments x 4096 tokens (16384 merged tokens), bf16",
+        "workload": WORKLOAD_TEXT[w.name],
         "name": w.name, "num_layers": w.num_layers, "num_kv_heads": w.num_kv_heads,
         "head_dim": w.head_dim, "fragments": len(specs), "seq_lens": [s.seq_len for s in specs],
         "merged_tokens": sum(s.seq_len for s in specs), "routing_layer": w.num_layers // 2,
@@ -230,7 +241,7 @@ def main():
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
 
-    w = synthetic.WORKLOADS[WORKLOAD]
+    w = synthetic.WORKLOADS[args.workload]
     L, H, d = w.num_layers, w.num_kv_heads, w.head_dim
     specs = synthetic.fragment_specs(w)
     frags = [synthetic.make_fragment_torch(s, L, H, d, dev) for s in specs]
@@ -252,10 +263,10 @@ def main():
         if timers is not None:
             timers["ingest"][0].record(stream)
         for i, f in enumerate(fd):
-            cm.cm_ingest(a if i < 2 else b, f, stream)
+            cm.cm_ingest(a if i < (len(fd) + 1) // 2 else b, f, stream)
         if timers is not None:
             timers["ingest"][1].record(stream)
-        cm.cm_union(a, b)
+        cm.cm_union(a, b)   # replica exchange: A := A u B
         if timers is not None:
             timers["render"][0].record(stream)
         n, _ = cm.cm_render(a, k_out.data_ptr(), v_out.data_ptr(), total_T, stream)
@@ -368,7 +379,7 @@ def main():
             "gpu_launches": launches_per_step * args.steps,
             "clocks": clocks.summary(),
         }
-        if world == 1 and not args.no_cpu_baseline:
+        if world == 1 and not args.no_cpu_baseline and args.workload == WORKLOAD:
             line["cpu_baseline"] = cpu_baseline_entry()
         print(json.dumps(line), flush=True)
     ctx.close()
