@@ -58,7 +58,7 @@ typedef enum cm_status {
     CM_ERR_COLLISION = 5,       /* verify_bytes_on_hit: equal id, different bytes */
     CM_ERR_CUDA = 6,            /* a CUDA runtime call failed (message has the CUDA error text) */
     CM_ERR_OOM = 7,             /* host or device allocation failed */
-    CM_ERR_TIMEOUT = 8,         /* reserved: a bounded device-side wait ran out (no such wait exists yet) */
+    CM_ERR_TIMEOUT = 8,         /* a bounded device-side wait ran out (reported by cm_context_check) */
     CM_ERR_UNSUPPORTED = 9      /* too many fragments for one render launch group, or shape beyond limits */
 } cm_status;
 
@@ -169,6 +169,13 @@ cm_status cm_render(const cm_set *set, void *k_out, void *v_out, int64_t capacit
 cm_status cm_bagmerge(cm_context *ctx, const cm_fragment *frags, int32_t n, void *k_out,
                       void *v_out, int64_t capacity_tokens, cm_stream_t stream,
                       int64_t *out_seq_len);
+
+/* Synchronise `stream` and report whether any render launched from ctx since the
+ * last check had a device-side wait run out (render kernels bound every wait on
+ * their own TMA copies to about one second, then record the failure and return
+ * instead of hanging). Returns CM_ERR_TIMEOUT once per such event and clears it;
+ * the output of the affected render is incomplete. CM_OK otherwise. */
+cm_status cm_context_check(cm_context *ctx, cm_stream_t stream);
 
 /* Static name of a status code. */
 const char *cm_status_string(cm_status status);

@@ -70,6 +70,7 @@ _SIGS = {
     "cm_ingest": (_c.c_int, [_P, _c.POINTER(cm_fragment), _P, _c.POINTER(cm_id),
                              _c.POINTER(_c.c_int32)]),
     "cm_union": (_c.c_int, [_P, _P]),
+    "cm_context_check": (_c.c_int, [_P, _P]),
     "cm_set_size": (_c.c_int, [_P, _c.POINTER(_c.c_int64)]),
     "cm_set_seq_len": (_c.c_int, [_P, _c.POINTER(_c.c_int64)]),
     "cm_set_ids": (_c.c_int, [_P, _c.POINTER(cm_id), _c.c_int64]),
@@ -128,6 +129,10 @@ def cm_context_create(device: int = 0, rope_theta: float = 1.0e6, routing_layer:
 
 def cm_context_destroy(ctx: Optional[int]) -> None:
     _check(lib.cm_context_destroy(ctx))
+
+
+def cm_context_check(ctx: int, stream=None) -> None:
+    _check(lib.cm_context_check(ctx, _stream_handle(stream)))
 
 
 def cm_set_create(ctx: int) -> int:
@@ -232,6 +237,9 @@ class Context:
             self.close()
         except Exception:
             pass
+
+    def check(self, stream=None) -> None:
+        cm_context_check(self.handle, stream)
 
     def fragment_id(self, K, V, stream=None):
         return cm_fragment_id(self.handle, fragment_from_tensors(K, V), stream)

@@ -110,7 +110,7 @@ struct cm_context {
     int32_t routing_layer = -1;
     bool verify = false;
     int num_sms = 0;
-    int render_blocks_per_sm = 1;
+    unsigned int *d_error = nullptr;   // set by a kernel whose bounded wait timed out
     std::mutex mu;
     // hashing scratch (device): leaf digests, inner levels, Q[t], compare flag
     uint8_t *d_scratch = nullptr;
@@ -258,6 +258,23 @@ cm_status fragment_digest(cm_context *ctx, const cm_fragment *f, cudaStream_t st
     return CM_OK;
 }
 
+// Reads and clears the context's error word on `stream` (synchronising it).
+cm_status take_device_error(cm_context *ctx, cudaStream_t stream) {
+    cm_status st = ensure_scratch(ctx, 0, 16);
+    if (st != CM_OK) return st;
+    CM_CUDA_TRY(cudaMemcpyAsync(ctx->h_pinned, ctx->d_error, sizeof(unsigned int),
+                                cudaMemcpyDeviceToHost, stream),
+                "error word copy");
+    CM_CUDA_TRY(cudaStreamSynchronize(stream), "error word synchronisation");
+    unsigned int e;
+    std::memcpy(&e, ctx->h_pinned, sizeof e);
+    if (e == 0) return CM_OK;
+    CM_CUDA_TRY(cudaMemsetAsync(ctx->d_error, 0, sizeof(unsigned int), stream), "error word reset");
+    CM_CUDA_TRY(cudaStreamSynchronize(stream), "error word synchronisation");
+    return fail(CM_ERR_TIMEOUT, "a bounded wait inside a render kernel timed out; that render's "
+                                "output is incomplete");
+}
+
 // Byte comparison of a new fragment against a stored record with the same id.
 cm_status bytes_equal(cm_context *ctx, const cm_fragment *f, const Record &r, cudaStream_t stream,
                       bool *equal) {
@@ -338,8 +355,8 @@ cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t 
         if (chunk > 0xFFFFFFFFull)
             return fail(CM_ERR_UNSUPPORTED, "render launch group exceeds 2^32 work items");
         p->total_chunks = (uint32_t)chunk;
-        const uint64_t resident = (uint64_t)ctx->num_sms * ctx->render_blocks_per_sm;
-        const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(chunk, resident));
+        p->error = ctx->d_error;
+        const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(chunk, ctx->num_sms));
         CM_CUDA_TRY(cm::launch_render(*p, grid, stream), "render launch");
     }
     return CM_OK;
@@ -444,8 +461,9 @@ cm_status cm_context_create(int32_t device, double rope_theta, int32_t routing_l
         ctx->verify = verify_bytes_on_hit != 0;
         CM_CUDA_TRY(cudaDeviceGetAttribute(&ctx->num_sms, cudaDevAttrMultiProcessorCount, device),
                     "multiprocessor count");
-        CM_CUDA_TRY(cm::render_blocks_per_sm(&ctx->render_blocks_per_sm), "render occupancy");
-        if (ctx->render_blocks_per_sm < 1) ctx->render_blocks_per_sm = 1;
+        CM_CUDA_TRY(cm::render_prepare(), "render kernel attributes");
+        CM_CUDA_TRY(cudaMalloc(&ctx->d_error, sizeof(unsigned int)), "error word allocation");
+        CM_CUDA_TRY(cudaMemset(ctx->d_error, 0, sizeof(unsigned int)), "error word reset");
         *out = ctx.release();
         return CM_OK;
     });
@@ -459,6 +477,7 @@ cm_status cm_context_destroy(cm_context *ctx) {
         DeviceScope scope(ctx->device);
         if (ctx->d_scratch) cudaFree(ctx->d_scratch);
         if (ctx->h_pinned) cudaFreeHost(ctx->h_pinned);
+        if (ctx->d_error) cudaFree(ctx->d_error);
         delete ctx;
         return CM_OK;
     });
@@ -635,6 +654,16 @@ cm_status cm_render(const cm_set *set, void *k_out, void *v_out, int64_t capacit
         if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
         return launch_slots(ctx, slots, set->L, set->H, set->d, k_out, v_out, capacity_tokens,
                             reinterpret_cast<cudaStream_t>(stream));
+    });
+}
+
+cm_status cm_context_check(cm_context *ctx, cm_stream_t stream) {
+    return guarded([&]() -> cm_status {
+        if (!ctx) return fail(CM_ERR_INVALID_ARG, "context is NULL");
+        std::lock_guard<std::mutex> lock(ctx->mu);
+        DeviceScope scope(ctx->device);
+        if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
+        return take_device_error(ctx, reinterpret_cast<cudaStream_t>(stream));
     });
 }
 

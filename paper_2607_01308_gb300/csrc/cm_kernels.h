@@ -77,12 +77,14 @@ struct RenderParams {
     int32_t log2_pairs_per_row; // log2(d / 16)
     uint32_t total_chunks;
     uint32_t pad_;
+    unsigned int *error;        // device word: bit 0 set when a bounded wait timed out
     RenderSlot slot[kMaxSlots];
     double cs[2 * kMaxTablePairs];   // (cos a, sin a) of a = s * theta^(-2j/d), interleaved
 };
 
+// One CTA per SM; render_prepare() once per device before the first launch.
 cudaError_t launch_render(const RenderParams &p, int grid, cudaStream_t stream);
 int render_threads_per_block();
-cudaError_t render_blocks_per_sm(int *out);
+cudaError_t render_prepare();
 
 }  // namespace cm

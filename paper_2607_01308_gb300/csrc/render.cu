@@ -10,10 +10,11 @@
 // turned by one constant angle a_j = s * theta^(-2j/d) per frequency j (the delta
 // formula of Section 2.3), pairing element j with element j + d/2.
 //
-// Work item: 32 KiB of one source plane; a persistent grid walks the items.
-// A thread holds whole 16-byte vectors: for K it loads vector v of the row's first
-// half and vector v of its second half, i.e. 8 (x, y) pairs that share the
-// thread's 8 (cos, sin) values for the whole item.
+// Work item: up to 32 KiB of one source plane. A persistent grid of one CTA per SM
+// walks the items; 1-D TMA bulk copies stage them through shared memory (see
+// render_kernel). For a rotated K item a thread takes vector v of a row's first
+// half and vector v of its second half: 8 (x, y) pairs that share the thread's
+// 8 (cos, sin) values for the whole item.
 //
 // Rounding. The result must equal round-to-nearest-even-bf16 of
 // fl64(fl64(x c) - fl64(y s)) (and fl64(fl64(y c) + fl64(x s))), c and s the fp64
@@ -29,10 +30,9 @@
 namespace cm {
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 512;
 static_assert(sizeof(RenderParams) <= 32764, "render parameters exceed the kernel parameter limit");
 
-__device__ __forceinline__ uint4 ld_stream(const uint4 *p) { return __ldcs(p); }
 __device__ __forceinline__ void st_stream(uint4 *p, const uint4 &v) { __stcs(p, v); }
 
 // Two fp32 -> bf16 round-to-nearest-even, `lo` in bits 0..15, `hi` in bits 16..31.
@@ -120,40 +120,134 @@ __device__ __noinline__ void fixup_pair(const RenderParams &p, int cs_index, con
     bo = make_uint4(yo[0], yo[1], yo[2], yo[3]);
 }
 
-__device__ __forceinline__ void copy_item(const uint4 *__restrict__ src, uint4 *__restrict__ dst,
-                                          int n_vec) {
-    constexpr int kU = kChunkBytes / 16 / kThreads;   // 8 vectors per thread
-    uint4 r[kU];
-#pragma unroll
-    for (int u = 0; u < kU; ++u) {
-        const int i = threadIdx.x + u * kThreads;
-        if (i < n_vec) r[u] = ld_stream(src + i);
-    }
-#pragma unroll
-    for (int u = 0; u < kU; ++u) {
-        const int i = threadIdx.x + u * kThreads;
-        if (i < n_vec) st_stream(dst + i, r[u]);
-    }
+// ---------------------------------------------------------------- TMA bulk pipeline
+
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
 }
 
-__device__ __forceinline__ void rotate_item(const RenderParams &p, const float2 *cs32, int cs_index,
-                                            const uint4 *__restrict__ src,
-                                            uint4 *__restrict__ dst, int rows, int lane_v) {
-    constexpr int kU = kChunkBytes / 32 / kThreads;   // 4 vector pairs per thread
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count)
+                 : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
+                 "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
+    uint32_t done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(smem_addr(bar)), "r"(parity)
+        : "memory");
+    return done != 0;
+}
+
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Waits for phase `parity` of an mbarrier for at most kWaitLimitNs; false on timeout.
+constexpr uint64_t kWaitLimitNs = 1000000000ull;
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_ns();
+    while (!mbar_try_wait(bar, parity)) {
+        if (global_ns() - t0 > kWaitLimitNs) return false;
+    }
+    return true;
+}
+
+// 1-D bulk copy global -> shared, completion counted in bytes on `bar`.
+__device__ __forceinline__ void bulk_load(void *dst_smem, const void *src, uint32_t bytes,
+                                          uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+        ::"r"(smem_addr(dst_smem)), "l"(src), "r"(bytes), "r"(smem_addr(bar))
+        : "memory");
+}
+
+// 1-D bulk copy shared -> global, tracked by bulk async-groups.
+__device__ __forceinline__ void bulk_store(void *dst, const void *src_smem, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst),
+                 "r"(smem_addr(src_smem)), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void bulk_commit() {
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+
+__device__ __forceinline__ void bulk_wait_read_1() {
+    asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
+
+__device__ __forceinline__ void bulk_wait_all() {
+    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+constexpr int kStages = 6;
+constexpr size_t kTableBytes = sizeof(float2) * kMaxTablePairs;
+constexpr size_t kDynSmem = (size_t)kStages * kChunkBytes + kTableBytes;
+
+// One work item: up to kChunkBytes of one source plane and where it goes.
+struct Item {
+    const uint8_t *src;
+    uint8_t *dst;
+    uint32_t bytes;
+    int32_t rows;
+    int32_t rotate;      // 1: K of a slot at a nonzero offset
+    int32_t cs_index;    // first (cos, sin) of this slot
+};
+
+__device__ __forceinline__ Item item_of(const RenderParams &p, uint32_t g) {
+    int si = 0;
+    while (si + 1 < p.num_slots && g >= p.slot[si + 1].chunk_begin) ++si;
+    const RenderSlot &S = p.slot[si];
+    const uint32_t local = g - S.chunk_begin;
+    const uint32_t plane = local / S.chunks_per_plane;
+    const uint32_t c = local - plane * S.chunks_per_plane;
+    const uint32_t lh_planes = (uint32_t)p.num_layers * (uint32_t)p.num_heads;
+    const bool is_v = plane >= lh_planes;            // K planes first, then V planes
+    const int64_t lh = is_v ? plane - lh_planes : plane;
+    const int64_t row0 = (int64_t)c * p.rows_per_chunk;
+    const int64_t left = S.seq_len - row0;
+    const int rows = left < p.rows_per_chunk ? (int)left : p.rows_per_chunk;
+    const int64_t row_bytes = (int64_t)p.head_dim * 2;
+    Item it;
+    it.src = static_cast<const uint8_t *>(is_v ? S.v : S.k) + (lh * S.seq_len + row0) * row_bytes;
+    it.dst = static_cast<uint8_t *>(is_v ? p.v_out : p.k_out) +
+             (lh * p.capacity + S.offset + row0) * row_bytes;
+    it.bytes = (uint32_t)(rows * row_bytes);
+    it.rows = rows;
+    it.rotate = (!is_v && S.rotate) ? 1 : 0;
+    it.cs_index = S.table_base;
+    return it;
+}
+
+// K rows of one item, staged in shared memory: rotate and store to global.
+__device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const float2 *cs32,
+                                                 const Item &it, const uint8_t *buf, int lane_v) {
     const int vecs_per_row = p.head_dim >> 3;
     const int half_vecs = p.head_dim >> 4;
-    const int n_pairs = rows * half_vecs;
-    uint4 a[kU], b[kU];
-#pragma unroll
-    for (int u = 0; u < kU; ++u) {
-        const int q = threadIdx.x + u * kThreads;
-        if (q < n_pairs) {
-            const int row = q >> p.log2_pairs_per_row;
-            const uint4 *r = src + (int64_t)row * vecs_per_row + lane_v;
-            a[u] = ld_stream(r);
-            b[u] = ld_stream(r + half_vecs);
-        }
-    }
+    const int n_pairs = it.rows * half_vecs;
+    const int cs_index = it.cs_index + 8 * lane_v;
     float c[8], s[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
@@ -161,58 +255,96 @@ __device__ __forceinline__ void rotate_item(const RenderParams &p, const float2 
         c[e] = t.x;
         s[e] = t.y;
     }
-#pragma unroll
-    for (int u = 0; u < kU; ++u) {
-        const int q = threadIdx.x + u * kThreads;
-        if (q < n_pairs) {
-            uint4 ao, bo;
-            uint32_t b0, b1, b2, b3;
-            rotate_word(a[u].x, b[u].x, c[0], s[0], c[1], s[1], ao.x, bo.x, b0);
-            rotate_word(a[u].y, b[u].y, c[2], s[2], c[3], s[3], ao.y, bo.y, b1);
-            rotate_word(a[u].z, b[u].z, c[4], s[4], c[5], s[5], ao.z, bo.z, b2);
-            rotate_word(a[u].w, b[u].w, c[6], s[6], c[7], s[7], ao.w, bo.w, b3);
-            if ((b0 | b1 | b2 | b3) != 0u) fixup_pair(p, cs_index, a[u], b[u], ao, bo);
-            const int row = q >> p.log2_pairs_per_row;
-            uint4 *r = dst + (int64_t)row * vecs_per_row + lane_v;
-            st_stream(r, ao);
-            st_stream(r + half_vecs, bo);
-        }
+    const uint4 *src = reinterpret_cast<const uint4 *>(buf);
+    uint4 *dst = reinterpret_cast<uint4 *>(it.dst);
+#pragma unroll 2
+    for (int q = threadIdx.x; q < n_pairs; q += kThreads) {
+        const int row = q >> p.log2_pairs_per_row;
+        const int off = row * vecs_per_row + lane_v;
+        const uint4 a = src[off];
+        const uint4 b = src[off + half_vecs];
+        uint4 ao, bo;
+        uint32_t b0, b1, b2, b3;
+        rotate_word(a.x, b.x, c[0], s[0], c[1], s[1], ao.x, bo.x, b0);
+        rotate_word(a.y, b.y, c[2], s[2], c[3], s[3], ao.y, bo.y, b1);
+        rotate_word(a.z, b.z, c[4], s[4], c[5], s[5], ao.z, bo.z, b2);
+        rotate_word(a.w, b.w, c[6], s[6], c[7], s[7], ao.w, bo.w, b3);
+        if ((b0 | b1 | b2 | b3) != 0u) fixup_pair(p, cs_index, a, b, ao, bo);
+        st_stream(dst + off, ao);
+        st_stream(dst + off + half_vecs, bo);
     }
 }
 
-__global__ void __launch_bounds__(kThreads)
+// Persistent kernel, one CTA per SM. Thread 0 keeps kStages - 1 work items in
+// flight as 1-D TMA bulk loads into shared memory (completion on one mbarrier per
+// stage). A copy item (V, or K at offset 0) leaves shared memory by a TMA bulk
+// store; a rotate item is read by all threads, rotated and stored with 16-byte
+// streaming stores. A stage is refilled one iteration after its use, once its bulk
+// store (if any) has finished reading it. Every wait is bounded: on timeout the
+// CTA records an error, waits (bounded) for its own copies and returns.
+__global__ void __launch_bounds__(kThreads, 1)
 render_kernel(const __grid_constant__ RenderParams p) {
-    __shared__ float2 cs32[kMaxTablePairs];
+    extern __shared__ __align__(128) uint8_t smem[];
+    __shared__ __align__(8) uint64_t full[kStages];
+    __shared__ Item items[kStages];
+    float2 *cs32 = reinterpret_cast<float2 *>(smem + (size_t)kStages * kChunkBytes);
+
     const int half = p.head_dim >> 1;
     const int n_table = p.num_slots * half;
     for (int i = threadIdx.x; i < n_table; i += kThreads)
         cs32[i] = make_float2(__double2float_rn(p.cs[2 * i]), __double2float_rn(p.cs[2 * i + 1]));
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) mbar_init(&full[s], 1);
+        fence_mbar_init();
+    }
     __syncthreads();
 
-    const int vecs_per_row = p.head_dim >> 3;
+    const uint32_t first = blockIdx.x, stride = gridDim.x;
+    const uint32_t n = p.total_chunks > first ? (p.total_chunks - first + stride - 1) / stride : 0;
     const int lane_v = threadIdx.x & ((p.head_dim >> 4) - 1);
-    const uint32_t lh_planes = (uint32_t)p.num_layers * (uint32_t)p.num_heads;
+    uint32_t produced = 0;
 
-    for (uint32_t g = blockIdx.x; g < p.total_chunks; g += gridDim.x) {
-        int si = 0;
-        while (si + 1 < p.num_slots && g >= p.slot[si + 1].chunk_begin) ++si;
-        const RenderSlot &S = p.slot[si];
-        const uint32_t local = g - S.chunk_begin;
-        const uint32_t plane = local / S.chunks_per_plane;
-        const uint32_t c = local - plane * S.chunks_per_plane;
-        const bool is_v = plane >= lh_planes;       // K planes first, then V planes
-        const int64_t lh = is_v ? plane - lh_planes : plane;
-        const int64_t row0 = (int64_t)c * p.rows_per_chunk;
-        const int64_t left = S.seq_len - row0;
-        const int rows = left < p.rows_per_chunk ? (int)left : p.rows_per_chunk;
-        const uint4 *src = static_cast<const uint4 *>(is_v ? S.v : S.k) +
-                           (lh * S.seq_len + row0) * vecs_per_row;
-        uint4 *dst = static_cast<uint4 *>(is_v ? p.v_out : p.k_out) +
-                     (lh * p.capacity + S.offset + row0) * vecs_per_row;
-        if (is_v || !S.rotate) {
-            copy_item(src, dst, rows * vecs_per_row);
-        } else {
-            rotate_item(p, cs32, S.table_base + 8 * lane_v, src, dst, rows, lane_v);
+    auto produce = [&](uint32_t j) {
+        const uint32_t s = j % kStages;
+        const Item it = item_of(p, first + j * stride);
+        items[s] = it;
+        mbar_arrive_expect_tx(&full[s], it.bytes);
+        bulk_load(smem + (size_t)s * kChunkBytes, it.src, it.bytes, &full[s]);
+    };
+
+    if (threadIdx.x == 0) {
+        for (; produced < n && produced < (uint32_t)kStages; ++produced) produce(produced);
+    }
+
+    uint32_t i = 0;
+    bool aborted = false;
+    for (; i < n; ++i) {
+        const uint32_t s = i % kStages;
+        const bool ok = mbar_wait(&full[s], (i / kStages) & 1u);
+        if (__syncthreads_or(!ok)) {
+            aborted = true;
+            break;
+        }
+        const Item it = items[s];
+        const uint8_t *buf = smem + (size_t)s * kChunkBytes;
+        if (it.rotate) {
+            rotate_from_smem(p, cs32, it, buf, lane_v);
+        } else if (threadIdx.x == 0) {
+            bulk_store(it.dst, buf, it.bytes);
+        }
+        if (threadIdx.x == 0) bulk_commit();   // one group per item, possibly empty
+        __syncthreads();                       // every thread is done reading stage s
+        if (threadIdx.x == 0 && i >= 1 && produced < n) {
+            bulk_wait_read_1();                // the store of item i - 1 has left its stage
+            fence_proxy_async_smem();
+            produce(produced++);               // item i - 1 + kStages into stage (i - 1) % kStages
+        }
+    }
+    if (threadIdx.x == 0) {
+        bulk_wait_all();
+        if (aborted) {
+            atomicOr(p.error, 1u);
+            for (uint32_t j = i; j < produced; ++j) mbar_wait(&full[j % kStages], (j / kStages) & 1u);
         }
     }
 }
@@ -221,13 +353,14 @@ render_kernel(const __grid_constant__ RenderParams p) {
 
 int render_threads_per_block() { return kThreads; }
 
-cudaError_t render_blocks_per_sm(int *out) {
-    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, render_kernel, kThreads, 0);
+cudaError_t render_prepare() {
+    return cudaFuncSetAttribute(render_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)kDynSmem);
 }
 
 cudaError_t launch_render(const RenderParams &p, int grid, cudaStream_t stream) {
     if (p.total_chunks == 0) return cudaSuccess;
-    render_kernel<<<grid, kThreads, 0, stream>>>(p);
+    render_kernel<<<grid, kThreads, kDynSmem, stream>>>(p);
     return cudaGetLastError();
 }
 
