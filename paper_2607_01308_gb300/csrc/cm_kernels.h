@@ -51,7 +51,7 @@ cudaError_t launch_compare(const void *a, const void *b, uint64_t bytes, unsigne
 // ---------------------------------------------------------------- render
 constexpr int kMaxSlots = 32;          // fragments per render launch
 constexpr int kMaxTablePairs = 1792;   // sum over slots of head_dim / 2
-constexpr int kChunkBytes = 32768;     // bytes of one source plane handled per work item
+constexpr int kChunkBytes = 4096;      // bytes of one source plane handled per work item
 
 struct RenderSlot {
     const void *k;              // source K [L][H][T][d], device

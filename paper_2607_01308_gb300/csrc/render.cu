@@ -179,34 +179,18 @@ __device__ __forceinline__ void bulk_load(void *dst_smem, const void *src, uint3
         : "memory");
 }
 
-// 1-D bulk copy shared -> global, tracked by bulk async-groups.
-__device__ __forceinline__ void bulk_store(void *dst, const void *src_smem, uint32_t bytes) {
-    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst),
-                 "r"(smem_addr(src_smem)), "r"(bytes)
-                 : "memory");
-}
-
-__device__ __forceinline__ void bulk_commit() {
-    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-}
-
-__device__ __forceinline__ void bulk_wait_read_1() {
-    asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
-}
-
-__device__ __forceinline__ void bulk_wait_all() {
-    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
-}
-
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-constexpr int kStages = 6;
+constexpr int kWarps = kThreads / 32;
+constexpr int kStages = 3;                          // per warp
+constexpr uint32_t kItemBytes = 4096;               // one work item = one stage
 constexpr size_t kTableBytes = sizeof(float2) * kMaxTablePairs;
-constexpr size_t kDynSmem = (size_t)kStages * kChunkBytes + kTableBytes;
+constexpr size_t kDynSmem = (size_t)kWarps * kStages * kItemBytes + kTableBytes;
+static_assert(kChunkBytes == (int)kItemBytes, "host and kernel disagree on the work item size");
 
-// One work item: up to kChunkBytes of one source plane and where it goes.
+// One work item: up to kItemBytes of one source plane and where it goes.
 struct Item {
     const uint8_t *src;
     uint8_t *dst;
@@ -241,9 +225,27 @@ __device__ __forceinline__ Item item_of(const RenderParams &p, uint32_t g) {
     return it;
 }
 
-// K rows of one item, staged in shared memory: rotate and store to global.
+// Byte copy of one staged item: shared memory -> registers -> 16-byte streaming stores.
+__device__ __forceinline__ void copy_from_smem(const Item &it, const uint8_t *buf, int lane) {
+    constexpr int kU = kItemBytes / 16 / 32;          // 8 vectors per lane
+    const int n_vec = (int)(it.bytes >> 4);
+    const uint4 *src = reinterpret_cast<const uint4 *>(buf);
+    uint4 *dst = reinterpret_cast<uint4 *>(it.dst);
+    uint4 r[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u)
+        if (lane + 32 * u < n_vec) r[u] = src[lane + 32 * u];
+#pragma unroll
+    for (int u = 0; u < kU; ++u)
+        if (lane + 32 * u < n_vec) st_stream(dst + lane + 32 * u, r[u]);
+}
+
+// K rows of one staged item: rotate and store. Lane `lane` takes vector pairs
+// q = lane, lane + 32, ...; its vector index within the row half is lane % (d/16),
+// the same for every q, so its 8 (cos, sin) values are loaded once per item.
 __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const float2 *cs32,
-                                                 const Item &it, const uint8_t *buf, int lane_v) {
+                                                 const Item &it, const uint8_t *buf, int lane,
+                                                 int lane_v) {
     const int vecs_per_row = p.head_dim >> 3;
     const int half_vecs = p.head_dim >> 4;
     const int n_pairs = it.rows * half_vecs;
@@ -258,7 +260,7 @@ __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const fl
     const uint4 *src = reinterpret_cast<const uint4 *>(buf);
     uint4 *dst = reinterpret_cast<uint4 *>(it.dst);
 #pragma unroll 2
-    for (int q = threadIdx.x; q < n_pairs; q += kThreads) {
+    for (int q = lane; q < n_pairs; q += 32) {
         const int row = q >> p.log2_pairs_per_row;
         const int off = row * vecs_per_row + lane_v;
         const uint4 a = src[off];
@@ -275,77 +277,75 @@ __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const fl
     }
 }
 
-// Persistent kernel, one CTA per SM. Thread 0 keeps kStages - 1 work items in
-// flight as 1-D TMA bulk loads into shared memory (completion on one mbarrier per
-// stage). A copy item (V, or K at offset 0) leaves shared memory by a TMA bulk
-// store; a rotate item is read by all threads, rotated and stored with 16-byte
-// streaming stores. A stage is refilled one iteration after its use, once its bulk
-// store (if any) has finished reading it. Every wait is bounded: on timeout the
-// CTA records an error, waits (bounded) for its own copies and returns.
+// Persistent kernel, one CTA of kWarps warps per SM; every warp runs its own
+// pipeline over its own items (global item g = warp id + j * total warps), with no
+// block-wide barrier after set-up. Lane 0 keeps up to kStages items in flight as
+// 1-D TMA bulk loads into the warp's stages (completion on one mbarrier per
+// stage); all lanes wait for an item, move it from shared memory to its place in
+// the output (rotating K rows of slots at a nonzero offset), and lane 0 refills the
+// stage with the warp's next item. Every wait is bounded: on timeout the warp
+// records an error, waits (bounded) for its own copies in flight and returns.
 __global__ void __launch_bounds__(kThreads, 1)
 render_kernel(const __grid_constant__ RenderParams p) {
     extern __shared__ __align__(128) uint8_t smem[];
-    __shared__ __align__(8) uint64_t full[kStages];
-    __shared__ Item items[kStages];
-    float2 *cs32 = reinterpret_cast<float2 *>(smem + (size_t)kStages * kChunkBytes);
+    __shared__ __align__(8) uint64_t full[kWarps][kStages];
+    __shared__ Item items[kWarps][kStages];
+    float2 *cs32 = reinterpret_cast<float2 *>(smem + (size_t)kWarps * kStages * kItemBytes);
 
     const int half = p.head_dim >> 1;
     const int n_table = p.num_slots * half;
     for (int i = threadIdx.x; i < n_table; i += kThreads)
         cs32[i] = make_float2(__double2float_rn(p.cs[2 * i]), __double2float_rn(p.cs[2 * i + 1]));
-    if (threadIdx.x == 0) {
-        for (int s = 0; s < kStages; ++s) mbar_init(&full[s], 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) {
+        for (int s = 0; s < kStages; ++s) mbar_init(&full[warp][s], 1);
         fence_mbar_init();
     }
     __syncthreads();
 
-    const uint32_t first = blockIdx.x, stride = gridDim.x;
+    const uint32_t first = blockIdx.x * kWarps + warp;
+    const uint32_t stride = gridDim.x * kWarps;
     const uint32_t n = p.total_chunks > first ? (p.total_chunks - first + stride - 1) / stride : 0;
-    const int lane_v = threadIdx.x & ((p.head_dim >> 4) - 1);
-    uint32_t produced = 0;
+    const int lane_v = lane & ((p.head_dim >> 4) - 1);
+    uint8_t *wbuf = smem + (size_t)warp * kStages * kItemBytes;
 
     auto produce = [&](uint32_t j) {
         const uint32_t s = j % kStages;
         const Item it = item_of(p, first + j * stride);
-        items[s] = it;
-        mbar_arrive_expect_tx(&full[s], it.bytes);
-        bulk_load(smem + (size_t)s * kChunkBytes, it.src, it.bytes, &full[s]);
+        items[warp][s] = it;
+        mbar_arrive_expect_tx(&full[warp][s], it.bytes);
+        bulk_load(wbuf + (size_t)s * kItemBytes, it.src, it.bytes, &full[warp][s]);
     };
 
-    if (threadIdx.x == 0) {
+    uint32_t produced = 0;
+    if (lane == 0)
         for (; produced < n && produced < (uint32_t)kStages; ++produced) produce(produced);
-    }
 
     uint32_t i = 0;
     bool aborted = false;
     for (; i < n; ++i) {
         const uint32_t s = i % kStages;
-        const bool ok = mbar_wait(&full[s], (i / kStages) & 1u);
-        if (__syncthreads_or(!ok)) {
+        const bool ok = mbar_wait(&full[warp][s], (i / kStages) & 1u);
+        if (__any_sync(0xFFFFFFFFu, !ok)) {
             aborted = true;
             break;
         }
-        const Item it = items[s];
-        const uint8_t *buf = smem + (size_t)s * kChunkBytes;
-        if (it.rotate) {
-            rotate_from_smem(p, cs32, it, buf, lane_v);
-        } else if (threadIdx.x == 0) {
-            bulk_store(it.dst, buf, it.bytes);
-        }
-        if (threadIdx.x == 0) bulk_commit();   // one group per item, possibly empty
-        __syncthreads();                       // every thread is done reading stage s
-        if (threadIdx.x == 0 && i >= 1 && produced < n) {
-            bulk_wait_read_1();                // the store of item i - 1 has left its stage
+        const Item it = items[warp][s];
+        const uint8_t *buf = wbuf + (size_t)s * kItemBytes;
+        if (it.rotate)
+            rotate_from_smem(p, cs32, it, buf, lane, lane_v);
+        else
+            copy_from_smem(it, buf, lane);
+        __syncwarp();                          // every lane is done reading stage s
+        if (lane == 0 && produced < n) {
             fence_proxy_async_smem();
-            produce(produced++);               // item i - 1 + kStages into stage (i - 1) % kStages
+            produce(produced++);               // item i + kStages into stage s
         }
     }
-    if (threadIdx.x == 0) {
-        bulk_wait_all();
-        if (aborted) {
-            atomicOr(p.error, 1u);
-            for (uint32_t j = i; j < produced; ++j) mbar_wait(&full[j % kStages], (j / kStages) & 1u);
-        }
+    if (aborted && lane == 0) {
+        atomicOr(p.error, 1u);
+        for (uint32_t j = i; j < produced; ++j)
+            mbar_wait(&full[warp][j % kStages], (j / kStages) & 1u);
     }
 }
 
