@@ -23,8 +23,10 @@
 // E = 2^-22 (|z| + |x| + |y|) + 2^-146. If z - E and z + E (rounded outward) round
 // to the same bf16, every value between them does (rounding is monotone), the fp64
 // value included, and z's rounding is the answer. Otherwise (about one element in
-// several thousand) the element is recomputed in fp64 with the same operation
-// sequence and rounded directly to bf16, so the output is bit-exact either way.
+// a thousand) a second fp32 level with error-free products and a ~2^-36 bound
+// decides, and the few it cannot certify are recomputed in fp64 with the operation
+// sequence of the definition and rounded directly to bf16 (fp64 throughput is very
+// low on this part, so it must stay rare). The output is bit-exact either way.
 #include "cm_kernels.h"
 
 namespace cm {
@@ -94,30 +96,65 @@ __device__ __forceinline__ void rotate_word(uint32_t xw, uint32_t yw, float c0, 
     bad = bx | by;
 }
 
-__device__ __forceinline__ uint32_t set_half(uint32_t w, int half, uint32_t bits) {
-    return half ? (w & 0x0000FFFFu) | (bits << 16) : (w & 0xFFFF0000u) | bits;
+// Second level for one element pair (x, y) whose first-level result was not
+// certified. The table holds c = c1 + c2 with c1 carrying 16 significant bits
+// (so x c1 and y s1 are exact fp32 products of bf16 inputs) and c2 = fp32(c - c1):
+//   D = fl(x c1 - y s1),  r = fl(x c2 - fl(y s2)),  z = fl(D + r),
+// within E = 2^-22 |z| + 2^-36 (|x| + |y|) + 2^-146 of the fp64 value. Certified
+// as in the first level, else (rarely) recomputed in fp64 with the operation
+// sequence of the definition. Returns x' in bits 0..15 and y' in bits 16..31.
+__device__ __noinline__ uint32_t fix_element(float x, float y, float4 t, double c, double s) {
+    const float dx = __fmaf_rn(x, t.x, -__fmul_rn(y, t.z));
+    const float rx = __fmaf_rn(x, t.y, -__fmul_rn(y, t.w));
+    const float zx = __fadd_rn(dx, rx);
+    const float dy = __fmaf_rn(y, t.x, __fmul_rn(x, t.z));
+    const float ry = __fmaf_rn(y, t.y, __fmul_rn(x, t.w));
+    const float zy = __fadd_rn(dy, ry);
+    const float m = __fmul_ru(__fadd_ru(fabsf(x), fabsf(y)), 0x1p-36f);
+    const float ex = __fmaf_ru(fabsf(zx), 0x1p-22f, __fadd_ru(m, 0x1p-146f));
+    const float ey = __fmaf_ru(fabsf(zy), 0x1p-22f, __fadd_ru(m, 0x1p-146f));
+    const uint32_t lo = pack_bf16x2(__fsub_rd(zx, ex), __fsub_rd(zy, ey));
+    const uint32_t hi = pack_bf16x2(__fadd_ru(zx, ex), __fadd_ru(zy, ey));
+    uint32_t out = pack_bf16x2(zx, zy);
+    if ((lo ^ hi) != 0u) {
+        const double xd = (double)x, yd = (double)y;
+        const uint32_t bx = f64_to_bf16_bits(__dsub_rn(__dmul_rn(xd, c), __dmul_rn(yd, s)));
+        const uint32_t by = f64_to_bf16_bits(__dadd_rn(__dmul_rn(yd, c), __dmul_rn(xd, s)));
+        out = bx | (by << 16);
+    }
+    return out;
 }
 
-// Exact recomputation of the uncertified elements of one vector pair.
-__device__ __noinline__ void fixup_pair(const RenderParams &p, int cs_index, const uint4 &a,
-                                        const uint4 &b, uint4 &ao, uint4 &bo) {
-    const uint32_t xi[4] = {a.x, a.y, a.z, a.w};
-    const uint32_t yi[4] = {b.x, b.y, b.z, b.w};
-    uint32_t xo[4] = {ao.x, ao.y, ao.z, ao.w};
-    uint32_t yo[4] = {bo.x, bo.y, bo.z, bo.w};
+__device__ __forceinline__ uint32_t pick_word(const uint4 &v, int w) {
+    return w == 0 ? v.x : w == 1 ? v.y : w == 2 ? v.z : v.w;
+}
+
+__device__ __forceinline__ void put_half(uint4 &v, int e, uint32_t bits) {
+    const int w = e >> 1;
+    const uint32_t keep = (e & 1) ? 0x0000FFFFu : 0xFFFF0000u;
+    const uint32_t val = (e & 1) ? (bits << 16) : bits;
+    if (w == 0) v.x = (v.x & keep) | val;
+    else if (w == 1) v.y = (v.y & keep) | val;
+    else if (w == 2) v.z = (v.z & keep) | val;
+    else v.w = (v.w & keep) | val;
+}
+
+// Re-evaluates the elements of one vector pair whose masks b0..b3 flag them.
+__device__ __noinline__ void fixup_pair(const RenderParams &p, const float4 *tab, int cs_index,
+                                        const uint4 &a, const uint4 &b, uint32_t b0, uint32_t b1,
+                                        uint32_t b2, uint32_t b3, uint4 &ao, uint4 &bo) {
+    const uint32_t bw[4] = {b0, b1, b2, b3};
     for (int e = 0; e < 8; ++e) {
-        const int w = e >> 1, half = e & 1;
-        const double x = (double)(half ? bf16_hi(xi[w]) : bf16_lo(xi[w]));
-        const double y = (double)(half ? bf16_hi(yi[w]) : bf16_lo(yi[w]));
-        const double c = p.cs[2 * (cs_index + e)];
-        const double s = p.cs[2 * (cs_index + e) + 1];
-        const double zx = __dsub_rn(__dmul_rn(x, c), __dmul_rn(y, s));
-        const double zy = __dadd_rn(__dmul_rn(y, c), __dmul_rn(x, s));
-        xo[w] = set_half(xo[w], half, f64_to_bf16_bits(zx));
-        yo[w] = set_half(yo[w], half, f64_to_bf16_bits(zy));
+        const uint32_t m = bw[e >> 1] >> ((e & 1) * 16);
+        if ((m & 0xFFFFu) == 0u) continue;
+        const uint32_t xw = pick_word(a, e >> 1), yw = pick_word(b, e >> 1);
+        const float x = (e & 1) ? bf16_hi(xw) : bf16_lo(xw);
+        const float y = (e & 1) ? bf16_hi(yw) : bf16_lo(yw);
+        const uint32_t r = fix_element(x, y, tab[cs_index + e], p.cs[2 * (cs_index + e)],
+                                       p.cs[2 * (cs_index + e) + 1]);
+        put_half(ao, e, r & 0xFFFFu);
+        put_half(bo, e, r >> 16);
     }
-    ao = make_uint4(xo[0], xo[1], xo[2], xo[3]);
-    bo = make_uint4(yo[0], yo[1], yo[2], yo[3]);
 }
 
 // ---------------------------------------------------------------- TMA bulk pipeline
@@ -186,7 +223,7 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 constexpr int kWarps = kThreads / 32;
 constexpr int kStages = 3;                          // per warp
 constexpr uint32_t kItemBytes = 4096;               // one work item = one stage
-constexpr size_t kTableBytes = sizeof(float2) * kMaxTablePairs;
+constexpr size_t kTableBytes = sizeof(float4) * kMaxTablePairs;
 constexpr size_t kDynSmem = (size_t)kWarps * kStages * kItemBytes + kTableBytes;
 static_assert(kChunkBytes == (int)kItemBytes, "host and kernel disagree on the work item size");
 
@@ -243,7 +280,7 @@ __device__ __forceinline__ void copy_from_smem(const Item &it, const uint8_t *bu
 // K rows of one staged item: rotate and store. Lane `lane` takes vector pairs
 // q = lane, lane + 32, ...; its vector index within the row half is lane % (d/16),
 // the same for every q, so its 8 (cos, sin) values are loaded once per item.
-__device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const float2 *cs32,
+__device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const float4 *tab,
                                                  const Item &it, const uint8_t *buf, int lane,
                                                  int lane_v) {
     const int vecs_per_row = p.head_dim >> 3;
@@ -253,9 +290,9 @@ __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const fl
     float c[8], s[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
-        const float2 t = cs32[cs_index + e];
-        c[e] = t.x;
-        s[e] = t.y;
+        const float4 t = tab[cs_index + e];
+        c[e] = __fadd_rn(t.x, t.y);   // fp32 cos (within one ulp of the fp64 value)
+        s[e] = __fadd_rn(t.z, t.w);
     }
     const uint4 *src = reinterpret_cast<const uint4 *>(buf);
     uint4 *dst = reinterpret_cast<uint4 *>(it.dst);
@@ -271,10 +308,17 @@ __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const fl
         rotate_word(a.y, b.y, c[2], s[2], c[3], s[3], ao.y, bo.y, b1);
         rotate_word(a.z, b.z, c[4], s[4], c[5], s[5], ao.z, bo.z, b2);
         rotate_word(a.w, b.w, c[6], s[6], c[7], s[7], ao.w, bo.w, b3);
-        if ((b0 | b1 | b2 | b3) != 0u) fixup_pair(p, cs_index, a, b, ao, bo);
+        if ((b0 | b1 | b2 | b3) != 0u) fixup_pair(p, tab, cs_index, a, b, b0, b1, b2, b3, ao, bo);
         st_stream(dst + off, ao);
         st_stream(dst + off + half_vecs, bo);
     }
+}
+
+// (c1, c2) split of an fp64 cosine or sine: c1 = fp32(c) with its low 8 significand
+// bits cleared (16 significant bits), c2 = fp32(c - c1).
+__device__ __forceinline__ float2 split16(double c) {
+    const float c1 = __uint_as_float(__float_as_uint(__double2float_rn(c)) & 0xFFFFFF00u);
+    return make_float2(c1, __double2float_rn(c - (double)c1));
 }
 
 // Persistent kernel, one CTA of kWarps warps per SM; every warp runs its own
@@ -290,12 +334,14 @@ render_kernel(const __grid_constant__ RenderParams p) {
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ __align__(8) uint64_t full[kWarps][kStages];
     __shared__ Item items[kWarps][kStages];
-    float2 *cs32 = reinterpret_cast<float2 *>(smem + (size_t)kWarps * kStages * kItemBytes);
+    float4 *tab = reinterpret_cast<float4 *>(smem + (size_t)kWarps * kStages * kItemBytes);
 
     const int half = p.head_dim >> 1;
     const int n_table = p.num_slots * half;
-    for (int i = threadIdx.x; i < n_table; i += kThreads)
-        cs32[i] = make_float2(__double2float_rn(p.cs[2 * i]), __double2float_rn(p.cs[2 * i + 1]));
+    for (int i = threadIdx.x; i < n_table; i += kThreads) {
+        const float2 cc = split16(p.cs[2 * i]), ss = split16(p.cs[2 * i + 1]);
+        tab[i] = make_float4(cc.x, cc.y, ss.x, ss.y);
+    }
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (lane == 0) {
         for (int s = 0; s < kStages; ++s) mbar_init(&full[warp][s], 1);
@@ -333,7 +379,7 @@ render_kernel(const __grid_constant__ RenderParams p) {
         const Item it = items[warp][s];
         const uint8_t *buf = wbuf + (size_t)s * kItemBytes;
         if (it.rotate)
-            rotate_from_smem(p, cs32, it, buf, lane, lane_v);
+            rotate_from_smem(p, tab, it, buf, lane, lane_v);
         else
             copy_from_smem(it, buf, lane);
         __syncwarp();                          // every lane is done reading stage s
