@@ -116,6 +116,30 @@ cm_status cm_set_destroy(cm_set *set);
 cm_status cm_fragment_id(cm_context *ctx, const cm_fragment *frag, cm_stream_t stream,
                          cm_id *out_id, uint64_t *out_norm_key);
 
+/* Allocation-free variant of cm_fragment_id (the paper has no counterpart; this is
+ * for callers that cannot allocate device memory: a serving engine that has
+ * handed nearly all of the GPU's memory to its own paged KV-cache pool, where a
+ * surprise cudaMalloc would fail or fragment that pool, or code that routes every
+ * device allocation through its own allocator and forbids the CUDA one).
+ * It computes the same id and norm key as cm_fragment_id on the calling thread's
+ * current device, asynchronously on `stream`, and calls no cudaMalloc, cudaFree or
+ * other allocating routine: the tree levels below the root live in a static device
+ * array of 16.25 MiB that every GPU that loads libcm.so holds until the process
+ * exits.
+ *   routing_layer  l* (0-indexed); < 0 selects floor(num_layers / 2)
+ *   id_out         DEVICE, 16-byte aligned, 16 bytes: receives the id
+ *   norm_key_out   DEVICE, 8-byte aligned, seq_len uint64: receives Q[t] (it is zeroed
+ *                  on `stream` first, then accumulated)
+ * Limit: the fragment's K and V bytes (2 * L * H * T * d * 2) must not exceed 1 GiB;
+ * larger fragments return CM_ERR_UNSUPPORTED (use cm_fragment_id).
+ * The first call on a device looks up the array's device address (cudaGetSymbolAddress)
+ * and caches it; make that first call before any stream capture on that device.
+ * Every call shares the one array: calls whose GPU work overlaps (on different
+ * streams, or from several threads) race and corrupt each other's results; order
+ * them on one stream or synchronise between them. Returns after enqueueing. */
+cm_status cm_fragment_id_static(const cm_fragment *frag, int32_t routing_layer,
+                                cm_stream_t stream, void *id_out, uint64_t *norm_key_out);
+
 /* Ingest(S, C) of Algorithm 2: content-address the fragment (one pass over its
  * bytes on `stream`, which is synchronised before return, because membership is
  * decided on the host) and insert it keyed by its id. A fragment whose id is

@@ -69,6 +69,8 @@ _SIGS = {
                                   _c.POINTER(_c.c_uint64)]),
     "cm_ingest": (_c.c_int, [_P, _c.POINTER(cm_fragment), _P, _c.POINTER(cm_id),
                              _c.POINTER(_c.c_int32)]),
+    "cm_fragment_id_static": (_c.c_int, [_c.POINTER(cm_fragment), _c.c_int32, _P, _P,
+                                         _c.POINTER(_c.c_uint64)]),
     "cm_union": (_c.c_int, [_P, _P]),
     "cm_context_check": (_c.c_int, [_P, _P]),
     "cm_set_size": (_c.c_int, [_P, _c.POINTER(_c.c_int64)]),
@@ -152,6 +154,13 @@ def cm_fragment_id(ctx: int, frag: cm_fragment, stream=None,
     _check(lib.cm_fragment_id(ctx, ctypes.byref(frag), _stream_handle(stream), ctypes.byref(out),
                               q))
     return out.to_bytes(), (list(q) if q is not None else None)
+
+
+def cm_fragment_id_static(frag: cm_fragment, id_out: int, norm_key_out: int,
+                          routing_layer: int = -1, stream=None) -> None:
+    """Allocation-free id + norm key into caller-owned device buffers (asynchronous)."""
+    _check(lib.cm_fragment_id_static(ctypes.byref(frag), routing_layer, _stream_handle(stream),
+                                     id_out, ctypes.cast(norm_key_out, ctypes.POINTER(ctypes.c_uint64))))
 
 
 def cm_ingest(s: int, frag: cm_fragment, stream=None) -> Tuple[bytes, bool]:

@@ -16,6 +16,8 @@
 // power of two with rows of at most 1024 bytes.
 #include "cm_kernels.h"
 
+#include <vector>
+
 namespace cm {
 namespace {
 
@@ -298,3 +300,114 @@ cudaError_t launch_compare(const void *a, const void *b, uint64_t bytes, unsigne
 }
 
 }  // namespace cm
+
+// ---------------------------------------------------------------- allocation-free Id(C)
+//
+// cm_fragment_id_static computes what cm_fragment_id computes, for callers that
+// cannot allocate device memory: its scratch (the digests of every tree level
+// below the root) lives in the file-scope array below, which every GPU that loads
+// this library holds for the life of the process. Host code never uses the
+// array's name as an address: the first call on a device looks its device address
+// up with cudaGetSymbolAddress (with that device current) and caches it.
+
+#include <mutex>
+
+namespace cm {
+namespace {
+
+constexpr uint64_t kStaticMaxLeaves = 1ull << 20;                // byte stream of at most 1 GiB
+constexpr size_t kStaticScratchBytes = (16u << 20) + (256u << 10);   // 16.25 MiB
+constexpr int kStaticMaxDevices = 128;
+
+std::mutex g_static_mu;
+void *g_static_addr[kStaticMaxDevices] = {};
+
+}  // namespace
+
+static __device__ __align__(256) uint8_t g_static_scratch[kStaticScratchBytes];
+
+}  // namespace cm
+
+extern "C" cm_status cm_fragment_id_static(const cm_fragment *frag, int32_t routing_layer,
+                                           cm_stream_t stream, void *id_out,
+                                           uint64_t *norm_key_out) {
+    using namespace cm;
+    try {
+        cm_status st = check_fragment(frag);
+        if (st != CM_OK) return st;
+        if (!id_out || !norm_key_out)
+            return report_error(CM_ERR_INVALID_ARG, "id_out and norm_key_out must be device pointers");
+        if ((reinterpret_cast<uintptr_t>(id_out) & 15u) != 0 ||
+            (reinterpret_cast<uintptr_t>(norm_key_out) & 7u) != 0)
+            return report_error(CM_ERR_ALIGNMENT,
+                                "id_out must be 16-byte and norm_key_out 8-byte aligned");
+        const int32_t L = frag->num_layers, H = frag->num_kv_heads, T = frag->seq_len,
+                      d = frag->head_dim;
+        const int32_t rl = routing_layer < 0 ? L / 2 : routing_layer;
+        if (rl >= L) return report_error(CM_ERR_INVALID_ARG, "routing layer >= num_layers");
+        const uint64_t plane = (uint64_t)H * T * d * 2;
+        const uint64_t stream_bytes = 2ull * L * plane;
+        std::vector<uint64_t> sizes{(stream_bytes + kLeafBytes - 1) / kLeafBytes};
+        if (sizes[0] > kStaticMaxLeaves)
+            return report_error(CM_ERR_UNSUPPORTED,
+                                "cm_fragment_id_static: the fragment's K and V bytes exceed the "
+                                "1 GiB that its static scratch covers; use cm_fragment_id");
+        while (sizes.size() == 1 || sizes.back() > 1)
+            sizes.push_back((sizes.back() + kFanout - 1) / kFanout);
+        // levels below the root in the static array, each 256-byte aligned; the root
+        // (the last level, one node) is written straight to id_out
+        std::vector<size_t> off;
+        size_t used = 0;
+        for (size_t k = 0; k + 1 < sizes.size(); ++k) {
+            off.push_back(used);
+            used += ((size_t)sizes[k] * kDigestBytes + 255) & ~(size_t)255;
+        }
+        if (used > kStaticScratchBytes)
+            return report_error(CM_ERR_UNSUPPORTED, "static scratch layout overflow");
+        int dev = 0;
+        cudaError_t e = cudaGetDevice(&dev);
+        if (e != cudaSuccess) return report_error(CM_ERR_CUDA, cudaGetErrorString(e));
+        if (dev < 0 || dev >= kStaticMaxDevices)
+            return report_error(CM_ERR_UNSUPPORTED, "device ordinal beyond 127");
+        uint8_t *scratch = nullptr;
+        {
+            std::lock_guard<std::mutex> lock(g_static_mu);
+            if (!g_static_addr[dev]) {
+                void *p = nullptr;
+                e = cudaGetSymbolAddress(&p, g_static_scratch);
+                if (e != cudaSuccess) {
+                    cudaGetLastError();
+                    return report_error(CM_ERR_CUDA, cudaGetErrorString(e));
+                }
+                g_static_addr[dev] = p;
+            }
+            scratch = static_cast<uint8_t *>(g_static_addr[dev]);
+        }
+        const cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+        e = cudaMemsetAsync(norm_key_out, 0, (size_t)T * sizeof(uint64_t), cs);
+        if (e != cudaSuccess) return report_error(CM_ERR_CUDA, cudaGetErrorString(e));
+        LeafLaunch a;
+        a.k = static_cast<const uint8_t *>(frag->k);
+        a.v = static_cast<const uint8_t *>(frag->v);
+        a.plane_bytes = plane;
+        a.stream_bytes = stream_bytes;
+        a.num_leaves = sizes[0];
+        a.norm_begin = 2ull * (uint64_t)rl * plane;
+        a.row_bytes = (uint32_t)d * 2;
+        a.seq_len = (uint32_t)T;
+        a.norm_key = reinterpret_cast<unsigned long long *>(norm_key_out);
+        a.digests = scratch + off[0];
+        a.tree = make_tree_params(L, H, d, T);
+        e = launch_leaf_hash(a, cs);
+        if (e != cudaSuccess) return report_error(CM_ERR_CUDA, cudaGetErrorString(e));
+        for (size_t k = 1; k < sizes.size(); ++k) {
+            uint8_t *out = (k + 1 == sizes.size()) ? static_cast<uint8_t *>(id_out) : scratch + off[k];
+            e = launch_inner_hash(scratch + off[k - 1], sizes[k - 1], out, sizes[k], (uint32_t)k,
+                                  a.tree, cs);
+            if (e != cudaSuccess) return report_error(CM_ERR_CUDA, cudaGetErrorString(e));
+        }
+        return CM_OK;
+    } catch (...) {
+        return report_error(CM_ERR_OOM, "host allocation failed");
+    }
+}

@@ -703,3 +703,16 @@ cm_status cm_bagmerge(cm_context *ctx, const cm_fragment *frags, int32_t n, void
 }
 
 }  // extern "C"
+
+// Helpers for the allocation-free content-address entry point (blake2s_tree.cu).
+namespace cm {
+
+TreeParams make_tree_params(int32_t L, int32_t H, int32_t d, int32_t T) {
+    return tree_params(L, H, d, T);
+}
+
+cm_status check_fragment(const cm_fragment *f) { return validate_fragment(f); }
+
+cm_status report_error(cm_status st, const char *msg) { return fail(st, msg); }
+
+}  // namespace cm

@@ -7,6 +7,8 @@
 
 #include <cuda_runtime.h>
 
+#include "cm.h"
+
 namespace cm {
 
 // ---------------------------------------------------------------- content address
@@ -47,6 +49,11 @@ cudaError_t launch_inner_hash(const uint8_t *children, uint64_t num_children, ui
 // *flag |= 1 if the `bytes` bytes at a and b differ (16-byte aligned, bytes % 16 == 0).
 cudaError_t launch_compare(const void *a, const void *b, uint64_t bytes, unsigned int *flag,
                            cudaStream_t stream);
+
+// Host-core helpers used by the allocation-free entry point in blake2s_tree.cu.
+TreeParams make_tree_params(int32_t L, int32_t H, int32_t d, int32_t T);
+cm_status check_fragment(const cm_fragment *f);
+cm_status report_error(cm_status st, const char *msg);
 
 // ---------------------------------------------------------------- render
 constexpr int kMaxSlots = 32;          // fragments per render launch
