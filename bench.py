@@ -222,6 +222,24 @@ def run_reference(args):
     return 0
 
 
+# ---------------------------------------------------------------- multi-rank aggregation
+
+def max_over_ranks(x: float, device) -> float:
+    """The largest value of x over all ranks (identity without a process group)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([float(x)], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(world: int, steps_per_rank: int, max_elapsed_ms: float) -> float:
+    """Merges per second of the whole job: every rank's merges over the slowest rank's time."""
+    return world * steps_per_rank / (max_elapsed_ms * 1e-3)
+
+
 # ---------------------------------------------------------------- GPU arm
 
 def main():
@@ -298,10 +316,7 @@ def main():
     elapsed_ms = start.elapsed_time(end)
     render_ms = sum(t["render"][0].elapsed_time(t["render"][1]) for t in step_timers) / args.steps
     ingest_ms = sum(t["ingest"][0].elapsed_time(t["ingest"][1]) for t in step_timers) / args.steps
-    if world > 1:
-        tt = torch.tensor([elapsed_ms], device=dev, dtype=torch.float64)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(tt.item())
+    elapsed_ms = max_over_ranks(elapsed_ms, dev)
 
     # end to end through the C ABI with host buffers: pinned inputs copied in and the
     # merged cache copied out inside the timed region, every step
@@ -333,10 +348,8 @@ def main():
     e1.record(stream)
     torch.cuda.synchronize(dev)
     e2e_ms = e0.elapsed_time(e1)
+    e2e_ms = max_over_ranks(e2e_ms, dev)
     if world > 1:
-        tt = torch.tensor([e2e_ms], device=dev, dtype=torch.float64)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
         dist.barrier()
 
     if rank == 0:
@@ -351,7 +364,7 @@ def main():
         launches_per_step = len(specs) * levels + 1
         line = {
             "metric": METRIC,
-            "value": world * args.steps / (elapsed_ms * 1e-3),
+            "value": whole_job_rate(world, args.steps, elapsed_ms),
             "unit": UNIT,
             "n_gpus": world,
             "steps": args.steps,
@@ -376,7 +389,7 @@ def main():
                 "unit": "GB/s", "frac": render_gbs / peak, "traffic": render_profile_traffic(),
                 "algorithmic_bytes_per_launch": render_bytes,
             },
-            "e2e": {"value": world * e2e_steps / (e2e_ms * 1e-3), "unit": UNIT,
+            "e2e": {"value": whole_job_rate(world, e2e_steps, e2e_ms), "unit": UNIT,
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": launches_per_step * args.steps,
             "clocks": clocks.summary(),
