@@ -152,6 +152,19 @@ cm_status cm_fragment_id_static(const cm_fragment *frag, int32_t routing_layer,
 cm_status cm_ingest(cm_set *set, const cm_fragment *frag, cm_stream_t stream, cm_id *out_id,
                     int32_t *out_absorbed);
 
+/* Ingest of n deliveries in order (Algorithm 2, Ingest, applied n times): the same
+ * result as n calls of cm_ingest, with one pass of GPU work for all of them (the
+ * leaf-hash launch of every fragment, then one launch per tree level covering all
+ * fragments) and a single synchronisation of `stream`. A delivery whose id is
+ * already in the set, or equal to an earlier delivery of the same batch, is
+ * absorbed. All fragments must have the set's shape (or one common shape if the
+ * set is empty). Nothing is inserted if validation fails.
+ *   frags         HOST array of n descriptors (n >= 0)
+ *   out_ids       nullable HOST array of n ids
+ *   out_absorbed  nullable HOST array of n flags */
+cm_status cm_ingest_batch(cm_set *set, const cm_fragment *frags, int32_t n, cm_stream_t stream,
+                          cm_id *out_ids, int32_t *out_absorbed);
+
 /* Merge of Algorithm 2 (Eq. setunion): dst := dst u src. Host only, no GPU work.
  * Both sets must come from the same context (CM_ERR_INVALID_ARG otherwise) and have
  * the same shape unless one is empty (CM_ERR_SHAPE_MISMATCH). On equal ids dst keeps
@@ -200,6 +213,24 @@ cm_status cm_bagmerge(cm_context *ctx, const cm_fragment *frags, int32_t n, void
  * instead of hanging). Returns CM_ERR_TIMEOUT once per such event and clears it;
  * the output of the affected render is incomplete. CM_OK otherwise. */
 cm_status cm_context_check(cm_context *ctx, cm_stream_t stream);
+
+/* Device time per kernel, accumulated while timing is on (a profiling aid). */
+typedef struct cm_kernel_times {
+    double leaf_hash_ms;          /* content address, level 0 (one launch per fragment) */
+    int64_t leaf_hash_launches;
+    double inner_hash_ms;         /* content address, tree levels above the leaves */
+    int64_t inner_hash_launches;
+    double render_ms;             /* render / BagMerge */
+    int64_t render_launches;
+} cm_kernel_times;
+
+/* Turn kernel timing on or off for ctx. While on, every launch the context makes
+ * is bracketed by two CUDA events on its stream. */
+cm_status cm_context_set_timing(cm_context *ctx, int32_t enable);
+
+/* Wait for the events of every timed launch so far, add their device times to the
+ * context's totals and report the totals; reset != 0 zeroes them afterwards. */
+cm_status cm_context_kernel_times(cm_context *ctx, cm_kernel_times *out, int32_t reset);
 
 /* Static name of a status code. */
 const char *cm_status_string(cm_status status);

@@ -54,6 +54,15 @@ class cm_fragment(ctypes.Structure):
                 ("k", ctypes.c_void_p), ("v", ctypes.c_void_p)]
 
 
+class cm_kernel_times(ctypes.Structure):
+    _fields_ = [("leaf_hash_ms", ctypes.c_double), ("leaf_hash_launches", ctypes.c_int64),
+                ("inner_hash_ms", ctypes.c_double), ("inner_hash_launches", ctypes.c_int64),
+                ("render_ms", ctypes.c_double), ("render_launches", ctypes.c_int64)]
+
+    def as_dict(self) -> dict:
+        return {name: getattr(self, name) for name, _ in self._fields_}
+
+
 _c = ctypes
 _P = ctypes.c_void_p
 _SIGS = {
@@ -71,6 +80,10 @@ _SIGS = {
                              _c.POINTER(_c.c_int32)]),
     "cm_fragment_id_static": (_c.c_int, [_c.POINTER(cm_fragment), _c.c_int32, _P, _P,
                                          _c.POINTER(_c.c_uint64)]),
+    "cm_ingest_batch": (_c.c_int, [_P, _c.POINTER(cm_fragment), _c.c_int32, _P,
+                                   _c.POINTER(cm_id), _c.POINTER(_c.c_int32)]),
+    "cm_context_set_timing": (_c.c_int, [_P, _c.c_int32]),
+    "cm_context_kernel_times": (_c.c_int, [_P, _c.POINTER(cm_kernel_times), _c.c_int32]),
     "cm_union": (_c.c_int, [_P, _P]),
     "cm_context_check": (_c.c_int, [_P, _P]),
     "cm_set_size": (_c.c_int, [_P, _c.POINTER(_c.c_int64)]),
@@ -169,6 +182,25 @@ def cm_ingest(s: int, frag: cm_fragment, stream=None) -> Tuple[bytes, bool]:
     _check(lib.cm_ingest(s, ctypes.byref(frag), _stream_handle(stream), ctypes.byref(out),
                          ctypes.byref(absorbed)))
     return out.to_bytes(), bool(absorbed.value)
+
+
+def cm_ingest_batch(s: int, frags: Sequence[cm_fragment], stream=None) -> List[Tuple[bytes, bool]]:
+    n = len(frags)
+    arr = (cm_fragment * max(n, 1))(*frags)
+    ids = (cm_id * max(n, 1))()
+    absorbed = (ctypes.c_int32 * max(n, 1))()
+    _check(lib.cm_ingest_batch(s, arr, n, _stream_handle(stream), ids, absorbed))
+    return [(ids[i].to_bytes(), bool(absorbed[i])) for i in range(n)]
+
+
+def cm_context_set_timing(ctx: int, enable: bool) -> None:
+    _check(lib.cm_context_set_timing(ctx, int(enable)))
+
+
+def cm_context_kernel_times(ctx: int, reset: bool = False) -> dict:
+    out = cm_kernel_times()
+    _check(lib.cm_context_kernel_times(ctx, ctypes.byref(out), int(reset)))
+    return out.as_dict()
 
 
 def cm_union(dst: int, src: int) -> None:
@@ -280,6 +312,14 @@ class FragmentSet:
             self.close()
         except Exception:
             pass
+
+    def ingest_batch(self, pairs, stream=None) -> List[Tuple[bytes, bool]]:
+        """Ingest [(K, V), ...] in order with one synchronisation."""
+        res = cm_ingest_batch(self.handle, [fragment_from_tensors(K, V) for K, V in pairs], stream)
+        for (fid, absorbed), kv in zip(res, pairs):
+            if not absorbed:
+                self._keep.setdefault(fid, kv)
+        return res
 
     def ingest(self, K, V, stream=None) -> Tuple[bytes, bool]:
         fid, absorbed = cm_ingest(self.handle, fragment_from_tensors(K, V), stream)

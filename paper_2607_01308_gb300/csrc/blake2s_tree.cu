@@ -257,6 +257,53 @@ inner_hash_kernel(const uint8_t *__restrict__ children, uint64_t num_children,
     store_digest(out + j * kDigestBytes, h);
 }
 
+// Node j of a tree level over children digests at `children` (n_children of them):
+// the node's 16 * min(128, n_children - 128 j) bytes are consumed one 64-byte block
+// at a time, the next block's loads issued before the current block is compressed.
+__device__ __forceinline__ void hash_inner_node(const uint8_t *children, uint64_t num_children,
+                                                uint8_t *out, uint64_t j, uint64_t num_nodes,
+                                                uint32_t depth, const TreeParams &tp) {
+    const uint64_t first = j * kFanout;
+    const uint64_t nc64 = num_children - first;
+    const uint32_t nc = nc64 < (uint64_t)kFanout ? (uint32_t)nc64 : (uint32_t)kFanout;
+    const uint32_t len = nc * kDigestBytes;
+    const uint32_t nblocks = (len + 63) / 64;
+    const bool last_node = j + 1 == num_nodes;
+    const uint8_t *src = children + first * kDigestBytes;
+    uint32_t h[8];
+    node_init(h, tp, j, depth);
+    uint4 nxt[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+        nxt[q] = (uint32_t)(q * 16) < len ? load_nc(src + q * 16) : make_uint4(0, 0, 0, 0);
+    for (uint32_t b = 0; b < nblocks; ++b) {
+        const uint4 w0 = nxt[0], w1 = nxt[1], w2 = nxt[2], w3 = nxt[3];
+        if (b + 1 < nblocks) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const uint32_t off = (b + 1) * 64 + q * 16;
+                nxt[q] = off < len ? load_nc(src + off) : make_uint4(0, 0, 0, 0);
+            }
+        }
+        const uint32_t m[16] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w,
+                                w2.x, w2.y, w2.z, w2.w, w3.x, w3.y, w3.z, w3.w};
+        const uint32_t end = (b + 1) * 64 < len ? (b + 1) * 64 : len;
+        compress(h, m, end, b + 1 == nblocks, last_node);
+    }
+    store_digest(out + j * kDigestBytes, h);
+}
+
+__global__ void __launch_bounds__(kInnerThreads)
+inner_group_kernel(const __grid_constant__ InnerGroup g) {
+    const uint64_t t = (uint64_t)blockIdx.x * kInnerThreads + threadIdx.x;
+    if (t >= g.node_begin[g.count]) return;
+    uint32_t f = 0;
+    while (f + 1 < g.count && t >= g.node_begin[f + 1]) ++f;
+    const uint64_t j = t - g.node_begin[f];
+    const uint64_t n_nodes = g.node_begin[f + 1] - g.node_begin[f];
+    hash_inner_node(g.children[f], g.num_children[f], g.out[f], j, n_nodes, g.depth, g.tree[f]);
+}
+
 __global__ void compare_kernel(const uint4 *__restrict__ a, const uint4 *__restrict__ b,
                                uint64_t n, unsigned int *flag) {
     uint32_t diff = 0;
@@ -285,6 +332,14 @@ cudaError_t launch_inner_hash(const uint8_t *children, uint64_t num_children, ui
     const uint64_t blocks = (num_nodes + kInnerThreads - 1) / kInnerThreads;
     inner_hash_kernel<<<(unsigned)blocks, kInnerThreads, 0, stream>>>(children, num_children, out,
                                                                     num_nodes, depth, tree);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_inner_group(const InnerGroup &g, cudaStream_t stream) {
+    const uint64_t total = g.node_begin[g.count];
+    if (total == 0) return cudaSuccess;
+    const uint64_t blocks = (total + kInnerThreads - 1) / kInnerThreads;
+    inner_group_kernel<<<(unsigned)blocks, kInnerThreads, 0, stream>>>(g);
     return cudaGetLastError();
 }
 

@@ -119,6 +119,16 @@ struct cm_context {
     uint8_t *h_pinned = nullptr;
     size_t pinned_bytes = 0;
     int live_sets = 0;
+    // kernel timing (cm_context_set_timing): events bracketing each launch
+    bool timing = false;
+    struct Pending {
+        int kind;
+        cudaEvent_t start, end;
+    };
+    std::vector<Pending> pending;
+    std::vector<cudaEvent_t> event_pool;
+    double time_ms[3] = {0, 0, 0};
+    int64_t launches[3] = {0, 0, 0};
 };
 
 struct cm_set {
@@ -199,61 +209,136 @@ cm::TreeParams tree_params(int32_t L, int32_t H, int32_t d, int32_t T) {
 
 uint64_t ceil_div(uint64_t a, uint64_t b) { return (a + b - 1) / b; }
 
-// Id(C) and Q[t] of one fragment; caller holds ctx->mu and the device scope.
-cm_status fragment_digest(cm_context *ctx, const cm_fragment *f, cudaStream_t stream, cm_id *id,
-                          std::vector<uint64_t> *Q) {
-    const int32_t L = f->num_layers, H = f->num_kv_heads, T = f->seq_len, d = f->head_dim;
-    const int32_t rl = routing_layer_for(ctx, L);
-    if (rl >= L) return fail(CM_ERR_INVALID_ARG, "routing layer >= num_layers");
-    const uint64_t plane = (uint64_t)H * T * d * 2;
-    const uint64_t stream_bytes = 2ull * L * plane;
-    std::vector<uint64_t> sizes{ceil_div(stream_bytes, cm::kLeafBytes)};
-    while (sizes.size() == 1 || sizes.back() > 1) sizes.push_back(ceil_div(sizes.back(), cm::kFanout));
-    // device layout: [Q: T x 8][level 0][level 1]... (each level 16-byte aligned)
-    const size_t q_bytes = ((size_t)T * 8 + 255) & ~(size_t)255;
-    std::vector<size_t> level_off;
-    size_t off = q_bytes;
-    for (uint64_t n : sizes) {
-        level_off.push_back(off);
-        off += ((size_t)n * cm::kDigestBytes + 255) & ~(size_t)255;
+enum { kTimeLeaf = 0, kTimeInner = 1, kTimeRender = 2 };
+
+cudaEvent_t take_event(cm_context *ctx) {
+    if (!ctx->event_pool.empty()) {
+        cudaEvent_t e = ctx->event_pool.back();
+        ctx->event_pool.pop_back();
+        return e;
     }
-    const size_t host_bytes = 16 + (size_t)T * 8;
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    return e;
+}
+
+// Runs `launch` on `stream`; when timing is on, brackets it with two events.
+template <class F>
+cudaError_t timed_launch(cm_context *ctx, int kind, cudaStream_t stream, F &&launch) {
+    if (!ctx->timing) return launch();
+    cudaEvent_t a = take_event(ctx), b = take_event(ctx);
+    if (!a || !b) return launch();
+    cudaEventRecord(a, stream);
+    const cudaError_t e = launch();
+    cudaEventRecord(b, stream);
+    ctx->pending.push_back({kind, a, b});
+    return e;
+}
+
+// Id(C) and Q[t] of n fragments in one pass: the leaf-hash launches of all
+// fragments, then one grouped launch per tree level (up to kMaxGroup fragments
+// each), then a single copy of every root digest and norm key to the host and one
+// synchronisation. Caller holds ctx->mu and the device scope.
+//   device scratch: [roots n x 16][Q of fragment 0]...[Q of fragment n-1][levels...]
+cm_status fragments_digest(cm_context *ctx, const cm_fragment *const *frags, size_t n,
+                           cudaStream_t stream, cm_id *ids, std::vector<uint64_t> *Qs) {
+    struct Layout {
+        std::vector<uint64_t> sizes;
+        std::vector<size_t> level_off;
+        size_t q_off;
+        uint64_t plane, stream_bytes;
+        int32_t rl;
+        cm::TreeParams tp;
+    };
+    std::vector<Layout> lay(n);
+    const size_t roots_bytes = n * 16;
+    size_t off = roots_bytes;
+    for (size_t i = 0; i < n; ++i) {
+        const cm_fragment *f = frags[i];
+        Layout &l = lay[i];
+        l.rl = routing_layer_for(ctx, f->num_layers);
+        if (l.rl >= f->num_layers) return fail(CM_ERR_INVALID_ARG, "routing layer >= num_layers");
+        l.plane = (uint64_t)f->num_kv_heads * f->seq_len * f->head_dim * 2;
+        l.stream_bytes = 2ull * f->num_layers * l.plane;
+        l.sizes.assign(1, ceil_div(l.stream_bytes, cm::kLeafBytes));
+        while (l.sizes.size() == 1 || l.sizes.back() > 1)
+            l.sizes.push_back(ceil_div(l.sizes.back(), cm::kFanout));
+        l.q_off = off;
+        off += (size_t)f->seq_len * 8;
+        l.tp = tree_params(f->num_layers, f->num_kv_heads, f->head_dim, f->seq_len);
+    }
+    const size_t host_bytes = off;     // roots and norm keys, copied back in one piece
+    off = (off + 255) & ~(size_t)255;
+    size_t max_levels = 0;
+    for (size_t i = 0; i < n; ++i) {
+        Layout &l = lay[i];
+        for (size_t k = 0; k + 1 < l.sizes.size(); ++k) {   // the root goes to the roots area
+            l.level_off.push_back(off);
+            off += ((size_t)l.sizes[k] * cm::kDigestBytes + 255) & ~(size_t)255;
+        }
+        max_levels = std::max(max_levels, l.sizes.size());
+    }
     cm_status st = ensure_scratch(ctx, off, host_bytes);
     if (st != CM_OK) return st;
     uint8_t *base = ctx->d_scratch;
-    auto *dq = reinterpret_cast<unsigned long long *>(base);
-    const cm::TreeParams tp = tree_params(L, H, d, T);
 
-    CM_CUDA_TRY(cudaMemsetAsync(dq, 0, (size_t)T * 8, stream), "zeroing the norm key");
-    cm::LeafLaunch a;
-    a.k = static_cast<const uint8_t *>(f->k);
-    a.v = static_cast<const uint8_t *>(f->v);
-    a.plane_bytes = plane;
-    a.stream_bytes = stream_bytes;
-    a.num_leaves = sizes[0];
-    a.norm_begin = 2ull * (uint64_t)rl * plane;
-    a.row_bytes = (uint32_t)d * 2;
-    a.seq_len = (uint32_t)T;
-    a.norm_key = dq;
-    a.digests = base + level_off[0];
-    a.tree = tp;
-    CM_CUDA_TRY(cm::launch_leaf_hash(a, stream), "leaf hash launch");
-    for (size_t k = 1; k < sizes.size(); ++k) {
-        CM_CUDA_TRY(cm::launch_inner_hash(base + level_off[k - 1], sizes[k - 1], base + level_off[k],
-                                          sizes[k], (uint32_t)k, tp, stream),
-                    "inner hash launch");
+    CM_CUDA_TRY(cudaMemsetAsync(base + roots_bytes, 0, host_bytes - roots_bytes, stream),
+                "zeroing the norm keys");
+    for (size_t i = 0; i < n; ++i) {
+        const cm_fragment *f = frags[i];
+        const Layout &l = lay[i];
+        cm::LeafLaunch a;
+        a.k = static_cast<const uint8_t *>(f->k);
+        a.v = static_cast<const uint8_t *>(f->v);
+        a.plane_bytes = l.plane;
+        a.stream_bytes = l.stream_bytes;
+        a.num_leaves = l.sizes[0];
+        a.norm_begin = 2ull * (uint64_t)l.rl * l.plane;
+        a.row_bytes = (uint32_t)f->head_dim * 2;
+        a.seq_len = (uint32_t)f->seq_len;
+        a.norm_key = reinterpret_cast<unsigned long long *>(base + l.q_off);
+        a.digests = base + l.level_off[0];
+        a.tree = l.tp;
+        CM_CUDA_TRY(timed_launch(ctx, kTimeLeaf, stream, [&] { return cm::launch_leaf_hash(a, stream); }),
+                    "leaf hash launch");
     }
-    CM_CUDA_TRY(cudaMemcpyAsync(ctx->h_pinned, base + level_off.back(), 16, cudaMemcpyDeviceToHost,
-                                stream),
+    for (size_t k = 1; k < max_levels; ++k) {
+        cm::InnerGroup g;
+        std::memset(&g, 0, sizeof g);
+        g.depth = (uint32_t)k;
+        auto flush = [&]() -> cudaError_t {
+            if (g.count == 0) return cudaSuccess;
+            const cudaError_t e =
+                timed_launch(ctx, kTimeInner, stream, [&] { return cm::launch_inner_group(g, stream); });
+            g.count = 0;
+            return e;
+        };
+        for (size_t i = 0; i < n; ++i) {
+            const Layout &l = lay[i];
+            if (k >= l.sizes.size()) continue;
+            const uint32_t c = g.count;
+            g.children[c] = base + l.level_off[k - 1];
+            g.num_children[c] = l.sizes[k - 1];
+            g.out[c] = (k + 1 == l.sizes.size()) ? base + 16 * i : base + l.level_off[k];
+            g.tree[c] = l.tp;
+            g.node_begin[c + 1] = g.node_begin[c] + l.sizes[k];
+            g.count = c + 1;
+            if (g.count == (uint32_t)cm::kMaxGroup) CM_CUDA_TRY(flush(), "inner hash launch");
+        }
+        CM_CUDA_TRY(flush(), "inner hash launch");
+    }
+    CM_CUDA_TRY(cudaMemcpyAsync(ctx->h_pinned, base, host_bytes, cudaMemcpyDeviceToHost, stream),
                 "digest copy");
-    CM_CUDA_TRY(cudaMemcpyAsync(ctx->h_pinned + 16, dq, (size_t)T * 8, cudaMemcpyDeviceToHost,
-                                stream),
-                "norm key copy");
     CM_CUDA_TRY(cudaStreamSynchronize(stream), "ingest synchronisation");
-    std::memcpy(id->b, ctx->h_pinned, 16);
-    if (Q) {
-        Q->resize((size_t)T);
-        std::memcpy(Q->data(), ctx->h_pinned + 16, (size_t)T * 8);
+    for (size_t i = 0; i < n; ++i) {
+        std::memcpy(ids[i].b, ctx->h_pinned + 16 * i, 16);
+        if (Qs) {
+            Qs[i].resize((size_t)frags[i]->seq_len);
+            std::memcpy(Qs[i].data(), ctx->h_pinned + lay[i].q_off, (size_t)frags[i]->seq_len * 8);
+        }
     }
     return CM_OK;
 }
@@ -357,7 +442,9 @@ cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t 
         p->total_chunks = (uint32_t)chunk;
         p->error = ctx->d_error;
         const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(chunk, ctx->num_sms));
-        CM_CUDA_TRY(cm::launch_render(*p, grid, stream), "render launch");
+        CM_CUDA_TRY(timed_launch(ctx, kTimeRender, stream,
+                                 [&] { return cm::launch_render(*p, grid, stream); }),
+                    "render launch");
     }
     return CM_OK;
 }
@@ -478,6 +565,11 @@ cm_status cm_context_destroy(cm_context *ctx) {
         if (ctx->d_scratch) cudaFree(ctx->d_scratch);
         if (ctx->h_pinned) cudaFreeHost(ctx->h_pinned);
         if (ctx->d_error) cudaFree(ctx->d_error);
+        for (const auto &pe : ctx->pending) {
+            cudaEventDestroy(pe.start);
+            cudaEventDestroy(pe.end);
+        }
+        for (cudaEvent_t e : ctx->event_pool) cudaEventDestroy(e);
         delete ctx;
         return CM_OK;
     });
@@ -521,63 +613,132 @@ cm_status cm_fragment_id(cm_context *ctx, const cm_fragment *frag, cm_stream_t s
         std::lock_guard<std::mutex> lock(ctx->mu);
         DeviceScope scope(ctx->device);
         if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
-        std::vector<uint64_t> Q;
-        st = fragment_digest(ctx, frag, reinterpret_cast<cudaStream_t>(stream), out_id,
-                             out_norm_key ? &Q : nullptr);
+        std::vector<uint64_t> Q[1];
+        st = fragments_digest(ctx, &frag, 1, reinterpret_cast<cudaStream_t>(stream), out_id,
+                              out_norm_key ? Q : nullptr);
         if (st != CM_OK) return st;
-        if (out_norm_key) std::memcpy(out_norm_key, Q.data(), Q.size() * sizeof(uint64_t));
+        if (out_norm_key) std::memcpy(out_norm_key, Q[0].data(), Q[0].size() * sizeof(uint64_t));
         return CM_OK;
     });
 }
 
 cm_status cm_ingest(cm_set *set, const cm_fragment *frag, cm_stream_t stream, cm_id *out_id,
                     int32_t *out_absorbed) {
+    return cm_ingest_batch(set, frag, 1, stream, out_id, out_absorbed);
+}
+
+cm_status cm_ingest_batch(cm_set *set, const cm_fragment *frags, int32_t n, cm_stream_t stream,
+                          cm_id *out_ids, int32_t *out_absorbed) {
     return guarded([&]() -> cm_status {
         if (!set) return fail(CM_ERR_INVALID_ARG, "set is NULL");
-        cm_status st = validate_fragment(frag);
-        if (st != CM_OK) return st;
+        if (n < 0 || (n > 0 && !frags)) return fail(CM_ERR_INVALID_ARG, "need n >= 0 fragments");
+        if (n == 0) return CM_OK;
         cm_context *ctx = set->ctx;
-        if (set->has_shape && (frag->num_layers != set->L || frag->num_kv_heads != set->H ||
-                               frag->head_dim != set->d))
-            return fail(CM_ERR_SHAPE_MISMATCH,
-                        "fragment (layers, kv_heads, head_dim) differ from the set's");
-        if (routing_layer_for(ctx, frag->num_layers) >= frag->num_layers)
-            return fail(CM_ERR_INVALID_ARG, "routing layer >= num_layers");
+        bool has_shape = set->has_shape;
+        int32_t L = set->L, H = set->H, d = set->d;
+        std::vector<const cm_fragment *> fp((size_t)n);
+        for (int32_t i = 0; i < n; ++i) {
+            const cm_fragment *f = &frags[i];
+            cm_status st = validate_fragment(f);
+            if (st != CM_OK) return st;
+            if (!has_shape) {
+                has_shape = true;
+                L = f->num_layers;
+                H = f->num_kv_heads;
+                d = f->head_dim;
+            } else if (f->num_layers != L || f->num_kv_heads != H || f->head_dim != d) {
+                return fail(CM_ERR_SHAPE_MISMATCH,
+                            "fragment (layers, kv_heads, head_dim) differ from the set's");
+            }
+            if (routing_layer_for(ctx, f->num_layers) >= f->num_layers)
+                return fail(CM_ERR_INVALID_ARG, "routing layer >= num_layers");
+            fp[(size_t)i] = f;
+        }
         std::lock_guard<std::mutex> lock(ctx->mu);
         DeviceScope scope(ctx->device);
         if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
         const cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
-        auto rec = std::make_shared<Record>();
-        st = fragment_digest(ctx, frag, cs, &rec->id, &rec->Q);
+        std::vector<cm_id> ids((size_t)n);
+        std::vector<std::vector<uint64_t>> Qs((size_t)n);
+        cm_status st = fragments_digest(ctx, fp.data(), (size_t)n, cs, ids.data(), Qs.data());
         if (st != CM_OK) return st;
-        if (out_id) *out_id = rec->id;
-        const IdKey key = key_of(rec->id);
-        auto it = set->items.find(key);
-        if (it != set->items.end()) {
-            if (ctx->verify) {
-                bool equal = false;
-                st = bytes_equal(ctx, frag, *it->second, cs, &equal);
-                if (st != CM_OK) return st;
-                if (!equal)
-                    return fail(CM_ERR_COLLISION, "content address hit with different bytes");
+        // Ingest in order: a later delivery with an id already present (in the set or
+        // earlier in this batch) is absorbed.
+        for (int32_t i = 0; i < n; ++i) {
+            const cm_fragment *f = fp[(size_t)i];
+            if (out_ids) out_ids[i] = ids[(size_t)i];
+            const IdKey key = key_of(ids[(size_t)i]);
+            auto it = set->items.find(key);
+            if (it != set->items.end()) {
+                if (ctx->verify) {
+                    bool equal = false;
+                    st = bytes_equal(ctx, f, *it->second, cs, &equal);
+                    if (st != CM_OK) return st;
+                    if (!equal)
+                        return fail(CM_ERR_COLLISION, "content address hit with different bytes");
+                }
+                if (out_absorbed) out_absorbed[i] = 1;
+                continue;
             }
-            if (out_absorbed) *out_absorbed = 1;
-            return CM_OK;
+            auto rec = std::make_shared<Record>();
+            rec->id = ids[(size_t)i];
+            rec->L = f->num_layers;
+            rec->H = f->num_kv_heads;
+            rec->T = f->seq_len;
+            rec->d = f->head_dim;
+            rec->k = f->k;
+            rec->v = f->v;
+            rec->Q = std::move(Qs[(size_t)i]);
+            set->items.emplace(key, std::move(rec));
+            if (!set->has_shape) {
+                set->has_shape = true;
+                set->L = f->num_layers;
+                set->H = f->num_kv_heads;
+                set->d = f->head_dim;
+            }
+            if (out_absorbed) out_absorbed[i] = 0;
         }
-        rec->L = frag->num_layers;
-        rec->H = frag->num_kv_heads;
-        rec->T = frag->seq_len;
-        rec->d = frag->head_dim;
-        rec->k = frag->k;
-        rec->v = frag->v;
-        set->items.emplace(key, std::move(rec));
-        if (!set->has_shape) {
-            set->has_shape = true;
-            set->L = frag->num_layers;
-            set->H = frag->num_kv_heads;
-            set->d = frag->head_dim;
+        return CM_OK;
+    });
+}
+
+cm_status cm_context_set_timing(cm_context *ctx, int32_t enable) {
+    if (!ctx) return fail(CM_ERR_INVALID_ARG, "context is NULL");
+    std::lock_guard<std::mutex> lock(ctx->mu);
+    ctx->timing = enable != 0;
+    return CM_OK;
+}
+
+cm_status cm_context_kernel_times(cm_context *ctx, cm_kernel_times *out, int32_t reset) {
+    return guarded([&]() -> cm_status {
+        if (!ctx) return fail(CM_ERR_INVALID_ARG, "context is NULL");
+        std::lock_guard<std::mutex> lock(ctx->mu);
+        DeviceScope scope(ctx->device);
+        if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
+        for (const auto &pe : ctx->pending) {
+            float ms = 0.f;
+            CM_CUDA_TRY(cudaEventSynchronize(pe.end), "timing event");
+            CM_CUDA_TRY(cudaEventElapsedTime(&ms, pe.start, pe.end), "timing event");
+            ctx->time_ms[pe.kind] += ms;
+            ctx->launches[pe.kind] += 1;
+            ctx->event_pool.push_back(pe.start);
+            ctx->event_pool.push_back(pe.end);
         }
-        if (out_absorbed) *out_absorbed = 0;
+        ctx->pending.clear();
+        if (out) {
+            out->leaf_hash_ms = ctx->time_ms[kTimeLeaf];
+            out->leaf_hash_launches = ctx->launches[kTimeLeaf];
+            out->inner_hash_ms = ctx->time_ms[kTimeInner];
+            out->inner_hash_launches = ctx->launches[kTimeInner];
+            out->render_ms = ctx->time_ms[kTimeRender];
+            out->render_launches = ctx->launches[kTimeRender];
+        }
+        if (reset) {
+            for (int k = 0; k < 3; ++k) {
+                ctx->time_ms[k] = 0;
+                ctx->launches[k] = 0;
+            }
+        }
         return CM_OK;
     });
 }

@@ -46,6 +46,21 @@ cudaError_t launch_inner_hash(const uint8_t *children, uint64_t num_children, ui
                               uint64_t num_nodes, uint32_t depth, const TreeParams &tree,
                               cudaStream_t stream);
 
+// All nodes of one tree level of up to kMaxGroup fragments in one launch: thread t
+// hashes node t - node_begin[f] of fragment f (node_begin is the prefix sum of the
+// fragments' node counts at this level).
+constexpr int kMaxGroup = 32;
+struct InnerGroup {
+    uint32_t count;
+    uint32_t depth;
+    uint64_t node_begin[kMaxGroup + 1];
+    const uint8_t *children[kMaxGroup];
+    uint64_t num_children[kMaxGroup];
+    uint8_t *out[kMaxGroup];
+    TreeParams tree[kMaxGroup];
+};
+cudaError_t launch_inner_group(const InnerGroup &g, cudaStream_t stream);
+
 // *flag |= 1 if the `bytes` bytes at a and b differ (16-byte aligned, bytes % 16 == 0).
 cudaError_t launch_compare(const void *a, const void *b, uint64_t bytes, unsigned int *flag,
                            cudaStream_t stream);

@@ -1,0 +1,164 @@
+"""GPU parity at the benchmark's full sizes, in the launch configuration bench.py
+times (two replicas batch-ingest half the fragments each, union, render).
+
+The oracle computes every content address and norm key in full (hashlib over all
+bytes) and the render on sampled (slot, layer, head) planes: each output plane
+depends only on its source plane and the slot's offset, so a sampled plane is
+checked exactly as a full render would check it. V planes are compared bit for
+bit, K planes within 1 bf16 ulp with the non-exact count asserted to be 0.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synthetic
+from oracle.content_address import fragment_id, id_as_int
+from oracle.norm import norm_key, tail_sum
+from parity_util import THETA, assert_k_parity, empty_out
+
+pytestmark = pytest.mark.gpu
+
+cm = pytest.importorskip("paper_2607_01308_gb300")
+
+
+@pytest.fixture(scope="module")
+def ctx():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    c = cm.Context(0, THETA)
+    yield c
+    c.close()
+
+
+def _oracle_keys(frags, routing_layer):
+    """(id, Q) of each fragment from its full bytes."""
+    out = []
+    for K, V in frags:
+        Kb, Vb = synthetic.to_bits(K), synthetic.to_bits(V)
+        out.append((fragment_id(Kb, Vb), norm_key(Kb, routing_layer)))
+    return out
+
+
+def _oracle_order(keys, lengths):
+    t_star = min(lengths)
+    S = [tail_sum(Q, t_star) for _, Q in keys]
+    return sorted(range(len(keys)), key=lambda i: (-S[i], -id_as_int(keys[i][0])))
+
+
+def _check_sampled_planes(frags, order, k_out, v_out, layers, heads):
+    s = 0
+    for i in order:
+        K, V = frags[i]
+        T = K.shape[2]
+        for l in layers:
+            for h in heads:
+                src_k = synthetic.to_bits(K[l, h])
+                got_k = synthetic.to_bits(k_out[l, h, s:s + T])
+                want_k = oracle.rotate_k(src_k, s, THETA)
+                assert assert_k_parity(got_k, want_k, f"K slot@{s} l={l} h={h}") == 0
+                assert np.array_equal(synthetic.to_bits(v_out[l, h, s:s + T]),
+                                      synthetic.to_bits(V[l, h]))
+        s += T
+
+
+def test_q4b_full_size_bench_configuration(ctx):
+    w = synthetic.WORKLOADS["q4b"]
+    specs = synthetic.fragment_specs(w)
+    frags = [synthetic.make_fragment_torch(sp, w.num_layers, w.num_kv_heads, w.head_dim, "cuda:0")
+             for sp in specs]
+    A, B = cm.FragmentSet(ctx), cm.FragmentSet(ctx)
+    ra = A.ingest_batch(frags[:2])
+    rb = B.ingest_batch(frags[2:])
+    A.union(B)
+    total = sum(sp.seq_len for sp in specs)
+    k_out, v_out = empty_out(w.num_layers, w.num_kv_heads, total, w.head_dim)
+    n, order_ids = A.render(k_out, v_out)
+    ctx.check()
+    torch.cuda.synchronize()
+    keys = _oracle_keys(frags, w.num_layers // 2)
+    assert [fid for fid, _ in ra + rb] == [k[0] for k in keys]
+    order = _oracle_order(keys, [sp.seq_len for sp in specs])
+    assert order_ids == [keys[i][0] for i in order]
+    assert n == total
+    _check_sampled_planes(frags, order, k_out, v_out, layers=[0, 18, 35], heads=[0, 7])
+    A.close()
+    B.close()
+
+
+@pytest.mark.parametrize("request_index", [0, 1])
+def test_serving_requests_with_redelivery(ctx, request_index):
+    w = synthetic.WORKLOADS["serve"]
+    specs = synthetic.fragment_specs(w, request_index)
+    frags = [synthetic.make_fragment_torch(sp, w.num_layers, w.num_kv_heads, w.head_dim, "cuda:0")
+             for sp in specs]
+    sched = synthetic.delivery_schedule(w, request_index)
+    msgs = [(frags[i][0].clone(), frags[i][1].clone()) for i in sched]
+    S = cm.FragmentSet(ctx)
+    res = S.ingest_batch(msgs)
+    seen = set()
+    for (fid, absorbed), i in zip(res, sched):
+        assert absorbed == (i in seen)
+        seen.add(i)
+    assert len(S) == len(specs)
+    total = sum(sp.seq_len for sp in specs)
+    k_out, v_out = empty_out(w.num_layers, w.num_kv_heads, total, w.head_dim)
+    n, order_ids = S.render(k_out, v_out)
+    torch.cuda.synchronize()
+    keys = _oracle_keys(frags, w.num_layers // 2)
+    order = _oracle_order(keys, [sp.seq_len for sp in specs])
+    assert order_ids == [keys[i][0] for i in order] and n == total
+    _check_sampled_planes(frags, order, k_out, v_out, layers=[1, 18], heads=[3])
+    S.close()
+
+
+def test_arity_batch_matches_sequential_ingest_and_oracle(ctx):
+    w = synthetic.WORKLOADS["q17_arity"]
+    specs = synthetic.fragment_specs(w)
+    frags = [synthetic.make_fragment_torch(sp, w.num_layers, w.num_kv_heads, w.head_dim, "cuda:0")
+             for sp in specs]
+    sched = synthetic.delivery_schedule(w)
+    assert len(sched) == 8
+    msgs = [(frags[i][0].clone(), frags[i][1].clone()) for i in sched]
+    S1 = cm.FragmentSet(ctx)
+    batch = S1.ingest_batch(msgs)
+    S2 = cm.FragmentSet(ctx)
+    seq = [S2.ingest(K, V) for K, V in msgs]
+    assert batch == seq
+    assert sum(a for _, a in batch) == 3 and len(S1) == 5
+    keys = _oracle_keys(frags, w.num_layers // 2)
+    assert sorted(S1.ids()) == sorted(k[0] for k in keys)
+    total = sum(sp.seq_len for sp in specs)
+    outs = []
+    for S in (S1, S2):
+        k_out, v_out = empty_out(w.num_layers, w.num_kv_heads, total, w.head_dim)
+        n, order_ids = S.render(k_out, v_out)
+        outs.append((k_out, v_out, order_ids))
+    torch.cuda.synchronize()
+    assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
+    order = _oracle_order(keys, [sp.seq_len for sp in specs])
+    assert outs[0][2] == [keys[i][0] for i in order]
+    _check_sampled_planes(frags, order, outs[0][0], outs[0][1], layers=[0, 14, 27], heads=[0, 5])
+    S1.close()
+    S2.close()
+
+
+def test_kernel_timing_counts_every_launch(ctx):
+    w, L, H, d = None, 4, 2, 64
+    g = torch.Generator(device="cuda:0").manual_seed(5)
+    frags = [(torch.randn((L, H, T, d), generator=g, device="cuda:0").to(torch.bfloat16),
+              torch.randn((L, H, T, d), generator=g, device="cuda:0").to(torch.bfloat16))
+             for T in (300, 40, 2100)]
+    cm.cm_context_kernel_times(ctx.handle, reset=True)
+    cm.cm_context_set_timing(ctx.handle, True)
+    S = cm.FragmentSet(ctx)
+    S.ingest_batch(frags)
+    k_out, v_out = empty_out(L, H, S.seq_len(), d)
+    S.render(k_out, v_out)
+    cm.cm_context_set_timing(ctx.handle, False)
+    t = cm.cm_context_kernel_times(ctx.handle, reset=True)
+    assert t["leaf_hash_launches"] == 3
+    assert t["inner_hash_launches"] >= 1
+    assert t["render_launches"] == 1
+    assert t["leaf_hash_ms"] > 0 and t["render_ms"] > 0
+    S.close()
