@@ -38,6 +38,13 @@ UNIT = "merges/s"
 WORKLOAD = "q4b"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
+# Integer-ALU roofline of the content-address kernel: a BLAKE2s block (64 bytes) is
+# 10 rounds x 8 G x (2 three-input adds + 4 xors + 4 rotates) + 8 xors = 808 ops that
+# must issue on the integer ALU pipe; the pipe takes 16 lanes per SMSP per clock
+# (4 SMSPs -> 64 ops/clk/SM), so the peak is 152 SMs x 64 x the maximum SM clock.
+HASH_ALU_OPS_PER_BYTE = 808.0 / 64.0
+ALU_OPS_PER_CLK_PER_SM = 64
+NUM_SMS = 152
 CLOCK_FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
                 "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
                 "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
@@ -132,21 +139,29 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
-def render_profile_traffic():
-    """DRAM bytes per render launch from the committed ncu summary, if it was taken on the
-    current render kernel source (its sha256 is recorded in the summary)."""
-    src = os.path.join(ROOT, "paper_2607_01308_gb300", "csrc", "render.cu")
-    summ = os.path.join(ROOT, "profiles", "render_kernel_q4b.md")
+def profile_traffic(source: str, summary: str):
+    """DRAM bytes per full launch from a committed ncu summary, if that summary was taken
+    on the current kernel source (the source's sha256 is recorded in it); else None."""
+    src = os.path.join(ROOT, "paper_2607_01308_gb300", "csrc", source)
+    summ = os.path.join(ROOT, "profiles", summary)
     try:
         sha = hashlib.sha256(open(src, "rb").read()).hexdigest()
         text = open(summ).read()
-        m_sha = re.search(r"render\.cu sha256:\s*([0-9a-f]{64})", text)
+        m_sha = re.search(re.escape(source) + r" sha256:\s*([0-9a-f]{64})", text)
         m_tr = re.search(r"dram_bytes_per_full_launch:\s*([0-9.eE+]+)", text)
         if m_sha and m_tr and m_sha.group(1) == sha:
             return float(m_tr.group(1))
     except OSError:
         pass
     return None
+
+
+def sm_max_mhz():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["sm_max_mhz"])
+    except Exception:
+        return 2070.0
 
 
 # ---------------------------------------------------------------- CPU oracle (baseline leg)
@@ -280,10 +295,11 @@ def main():
         a = cm.cm_set_create(ctx.handle)
         b = cm.cm_set_create(ctx.handle)
         fd = inputs or fdesc
+        half = (len(fd) + 1) // 2
         if timers is not None:
             timers["ingest"][0].record(stream)
-        for i, f in enumerate(fd):
-            cm.cm_ingest(a if i < (len(fd) + 1) // 2 else b, f, stream)
+        cm.cm_ingest_batch(a, fd[:half], stream)    # replica A
+        cm.cm_ingest_batch(b, fd[half:], stream)    # replica B
         if timers is not None:
             timers["ingest"][1].record(stream)
         cm.cm_union(a, b)   # replica exchange: A := A u B
@@ -305,12 +321,16 @@ def main():
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize(dev)
+    cm.cm_context_kernel_times(ctx.handle, reset=True)
+    cm.cm_context_set_timing(ctx.handle, True)   # events around every launch, on its stream
     with ClockSampler(local_rank) as clocks:
         start.record(stream)
         for i in range(args.steps):
             one_merge(step_timers[i])
         end.record(stream)
         torch.cuda.synchronize(dev)
+    cm.cm_context_set_timing(ctx.handle, False)
+    ktimes = cm.cm_context_kernel_times(ctx.handle, reset=True)
     if world > 1:
         dist.barrier()
     elapsed_ms = start.elapsed_time(end)
@@ -356,12 +376,35 @@ def main():
         peak, peak_src = hbm_peak()
         render_gbs = render_bytes / (render_ms * 1e-3) / 1e9
         ms_per_step = elapsed_ms / args.steps
-        levels = 1
-        n_leaves = -(-(w.bytes_per_token * specs[0].seq_len) // 1024)
-        while n_leaves > 1 or levels == 1:
-            n_leaves = -(-n_leaves // 128)
-            levels += 1
-        launches_per_step = len(specs) * levels + 1
+        launches_per_step = (ktimes["leaf_hash_launches"] + ktimes["inner_hash_launches"] +
+                             ktimes["render_launches"]) / args.steps
+        leaf_ms = ktimes["leaf_hash_ms"] / max(1, ktimes["leaf_hash_launches"])
+        frag_bytes = hash_bytes / len(specs)
+        hash_tops = HASH_ALU_OPS_PER_BYTE * frag_bytes / (leaf_ms * 1e-3) / 1e12
+        alu_peak = NUM_SMS * ALU_OPS_PER_CLK_PER_SM * sm_max_mhz() * 1e6 / 1e12
+        kernel_render_ms = ktimes["render_ms"] / max(1, ktimes["render_launches"])
+        render_roof = {
+            "kernel": "render_kernel", "bound": "hbm",
+            "achieved": render_bytes / (kernel_render_ms * 1e-3) / 1e9, "peak": peak,
+            "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
+            else "fallback 6.8 TB/s", "unit": "GB/s",
+            "frac": render_bytes / (kernel_render_ms * 1e-3) / 1e9 / peak,
+            "traffic": profile_traffic("render.cu", "render_kernel_q4b.md"),
+            "algorithmic_bytes_per_launch": render_bytes, "ms_per_launch": kernel_render_ms,
+        }
+        hash_roof = {
+            "kernel": "leaf_hash_kernel", "bound": "alu", "achieved": hash_tops, "peak": alu_peak,
+            "peak_source": "derived: 152 SMs x 64 integer-ALU lanes x max SM clock",
+            "unit": "Tops/s", "frac": hash_tops / alu_peak,
+            "traffic": profile_traffic("blake2s_tree.cu", "leaf_hash_kernel_q4b.md"),
+            "algorithmic_ops_per_launch": HASH_ALU_OPS_PER_BYTE * frag_bytes,
+            "bytes_hashed_per_launch": frag_bytes, "ms_per_launch": leaf_ms,
+            "hash_gbs": frag_bytes / (leaf_ms * 1e-3) / 1e9,
+        }
+        per_step = {"leaf_hash": ktimes["leaf_hash_ms"] / args.steps,
+                    "inner_hash": ktimes["inner_hash_ms"] / args.steps,
+                    "render": ktimes["render_ms"] / args.steps}
+        dominant = max(per_step, key=per_step.get)
         line = {
             "metric": METRIC,
             "value": whole_job_rate(world, args.steps, elapsed_ms),
@@ -382,16 +425,14 @@ def main():
             "render_ms": render_ms,
             "ingest_ms_per_merge": ingest_ms,
             "ingest_gbs": hash_bytes / (ingest_ms * 1e-3) / 1e9,
-            "roofline": {
-                "kernel": "render_kernel", "bound": "hbm", "achieved": render_gbs, "peak": peak,
-                "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
-                else "fallback 6.8 TB/s",
-                "unit": "GB/s", "frac": render_gbs / peak, "traffic": render_profile_traffic(),
-                "algorithmic_bytes_per_launch": render_bytes,
-            },
+            "roofline": hash_roof if dominant != "render" else render_roof,
+            "render_roofline": render_roof,
+            "hash_roofline": hash_roof,
+            "kernel_ms_per_step": per_step,
+            "dominant_kernel": dominant,
             "e2e": {"value": whole_job_rate(world, e2e_steps, e2e_ms), "unit": UNIT,
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-            "gpu_launches": launches_per_step * args.steps,
+            "gpu_launches": int(round(launches_per_step * args.steps)),
             "clocks": clocks.summary(),
         }
         if world == 1 and not args.no_cpu_baseline and args.workload == WORKLOAD:
