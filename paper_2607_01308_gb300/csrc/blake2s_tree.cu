@@ -260,6 +260,15 @@ inner_hash_kernel(const uint8_t *__restrict__ children, uint64_t num_children,
 // Node j of a tree level over children digests at `children` (n_children of them):
 // the node's 16 * min(128, n_children - 128 j) bytes are consumed one 64-byte block
 // at a time, the next block's loads issued before the current block is compressed.
+// kCoherent: the children were written by other threads of the same launch, so
+// they are read through L2 (ld.global.cg) instead of the non-coherent path.
+template <bool kCoherent>
+__device__ __forceinline__ uint4 load_child(const uint8_t *p) {
+    if (kCoherent) return __ldcg(reinterpret_cast<const uint4 *>(p));
+    return load_nc(p);
+}
+
+template <bool kCoherent = false>
 __device__ __forceinline__ void hash_inner_node(const uint8_t *children, uint64_t num_children,
                                                 uint8_t *out, uint64_t j, uint64_t num_nodes,
                                                 uint32_t depth, const TreeParams &tp) {
@@ -275,14 +284,14 @@ __device__ __forceinline__ void hash_inner_node(const uint8_t *children, uint64_
     uint4 nxt[4];
 #pragma unroll
     for (int q = 0; q < 4; ++q)
-        nxt[q] = (uint32_t)(q * 16) < len ? load_nc(src + q * 16) : make_uint4(0, 0, 0, 0);
+        nxt[q] = (uint32_t)(q * 16) < len ? load_child<kCoherent>(src + q * 16) : make_uint4(0, 0, 0, 0);
     for (uint32_t b = 0; b < nblocks; ++b) {
         const uint4 w0 = nxt[0], w1 = nxt[1], w2 = nxt[2], w3 = nxt[3];
         if (b + 1 < nblocks) {
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 const uint32_t off = (b + 1) * 64 + q * 16;
-                nxt[q] = off < len ? load_nc(src + off) : make_uint4(0, 0, 0, 0);
+                nxt[q] = off < len ? load_child<kCoherent>(src + off) : make_uint4(0, 0, 0, 0);
             }
         }
         const uint32_t m[16] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w,
@@ -294,14 +303,29 @@ __device__ __forceinline__ void hash_inner_node(const uint8_t *children, uint64_
 }
 
 __global__ void __launch_bounds__(kInnerThreads)
-inner_group_kernel(const __grid_constant__ InnerGroup g) {
-    const uint64_t t = (uint64_t)blockIdx.x * kInnerThreads + threadIdx.x;
-    if (t >= g.node_begin[g.count]) return;
-    uint32_t f = 0;
-    while (f + 1 < g.count && t >= g.node_begin[f + 1]) ++f;
-    const uint64_t j = t - g.node_begin[f];
-    const uint64_t n_nodes = g.node_begin[f + 1] - g.node_begin[f];
-    hash_inner_node(g.children[f], g.num_children[f], g.out[f], j, n_nodes, g.depth, g.tree[f]);
+tree_top_kernel(const __grid_constant__ TreeTop t) {
+    const uint64_t g = (uint64_t)blockIdx.x * kInnerThreads + threadIdx.x;
+    if (g >= t.node_begin[t.count]) return;
+    uint32_t fi = 0;
+    while (fi + 1 < t.count && g >= t.node_begin[fi + 1]) ++fi;
+    const TreeTopFragment &f = t.frag[fi];
+    uint64_t j = g - t.node_begin[fi];
+    hash_inner_node<false>(f.level[0], f.size[0], f.level[1], j, f.size[1], 1, f.tree);
+    for (uint32_t k = 1; k + 1 < f.levels; ++k) {
+        // this thread finished node j of level k; the one that finishes the last
+        // child of parent j / 128 hashes the parent
+        const uint64_t parent = j / kFanout;
+        const uint64_t first = parent * kFanout;
+        const uint64_t left = f.size[k] - first;
+        const uint32_t siblings = left < (uint64_t)kFanout ? (uint32_t)left : (uint32_t)kFanout;
+        __threadfence();                                  // publish this node's digest
+        const uint32_t done = atomicAdd(f.arrivals[k + 1] + parent, 1u) + 1;
+        if (done != siblings) return;
+        __threadfence();                                  // see every sibling's digest
+        hash_inner_node<true>(f.level[k], f.size[k], f.level[k + 1], parent, f.size[k + 1], k + 1,
+                              f.tree);
+        j = parent;
+    }
 }
 
 __global__ void compare_kernel(const uint4 *__restrict__ a, const uint4 *__restrict__ b,
@@ -335,11 +359,11 @@ cudaError_t launch_inner_hash(const uint8_t *children, uint64_t num_children, ui
     return cudaGetLastError();
 }
 
-cudaError_t launch_inner_group(const InnerGroup &g, cudaStream_t stream) {
-    const uint64_t total = g.node_begin[g.count];
+cudaError_t launch_tree_top(const TreeTop &t, cudaStream_t stream) {
+    const uint64_t total = t.node_begin[t.count];
     if (total == 0) return cudaSuccess;
     const uint64_t blocks = (total + kInnerThreads - 1) / kInnerThreads;
-    inner_group_kernel<<<(unsigned)blocks, kInnerThreads, 0, stream>>>(g);
+    tree_top_kernel<<<(unsigned)blocks, kInnerThreads, 0, stream>>>(t);
     return cudaGetLastError();
 }
 

@@ -272,21 +272,32 @@ cm_status fragments_digest(cm_context *ctx, const cm_fragment *const *frags, siz
     }
     const size_t host_bytes = off;     // roots and norm keys, copied back in one piece
     off = (off + 255) & ~(size_t)255;
-    size_t max_levels = 0;
     for (size_t i = 0; i < n; ++i) {
         Layout &l = lay[i];
+        if (l.sizes.size() > (size_t)cm::kMaxLevels)
+            return fail(CM_ERR_UNSUPPORTED, "fragment too large for the hash tree depth");
         for (size_t k = 0; k + 1 < l.sizes.size(); ++k) {   // the root goes to the roots area
             l.level_off.push_back(off);
             off += ((size_t)l.sizes[k] * cm::kDigestBytes + 255) & ~(size_t)255;
         }
-        max_levels = std::max(max_levels, l.sizes.size());
     }
+    // arrival counters of every node at levels >= 2, zeroed before the tree-top launch
+    const size_t arrivals_off = off;
+    std::vector<size_t> arr_off(n);
+    for (size_t i = 0; i < n; ++i) {
+        arr_off[i] = off;
+        for (size_t k = 2; k < lay[i].sizes.size(); ++k) off += (size_t)lay[i].sizes[k] * 4;
+    }
+    const size_t arrivals_bytes = off - arrivals_off;
     cm_status st = ensure_scratch(ctx, off, host_bytes);
     if (st != CM_OK) return st;
     uint8_t *base = ctx->d_scratch;
 
     CM_CUDA_TRY(cudaMemsetAsync(base + roots_bytes, 0, host_bytes - roots_bytes, stream),
                 "zeroing the norm keys");
+    if (arrivals_bytes)
+        CM_CUDA_TRY(cudaMemsetAsync(base + arrivals_off, 0, arrivals_bytes, stream),
+                    "zeroing the arrival counters");
     for (size_t i = 0; i < n; ++i) {
         const cm_fragment *f = frags[i];
         const Layout &l = lay[i];
@@ -305,31 +316,35 @@ cm_status fragments_digest(cm_context *ctx, const cm_fragment *const *frags, siz
         CM_CUDA_TRY(timed_launch(ctx, kTimeLeaf, stream, [&] { return cm::launch_leaf_hash(a, stream); }),
                     "leaf hash launch");
     }
-    for (size_t k = 1; k < max_levels; ++k) {
-        cm::InnerGroup g;
-        std::memset(&g, 0, sizeof g);
-        g.depth = (uint32_t)k;
-        auto flush = [&]() -> cudaError_t {
-            if (g.count == 0) return cudaSuccess;
-            const cudaError_t e =
-                timed_launch(ctx, kTimeInner, stream, [&] { return cm::launch_inner_group(g, stream); });
-            g.count = 0;
-            return e;
-        };
-        for (size_t i = 0; i < n; ++i) {
-            const Layout &l = lay[i];
-            if (k >= l.sizes.size()) continue;
-            const uint32_t c = g.count;
-            g.children[c] = base + l.level_off[k - 1];
-            g.num_children[c] = l.sizes[k - 1];
-            g.out[c] = (k + 1 == l.sizes.size()) ? base + 16 * i : base + l.level_off[k];
-            g.tree[c] = l.tp;
-            g.node_begin[c + 1] = g.node_begin[c] + l.sizes[k];
-            g.count = c + 1;
-            if (g.count == (uint32_t)cm::kMaxGroup) CM_CUDA_TRY(flush(), "inner hash launch");
+    std::unique_ptr<cm::TreeTop> top(new cm::TreeTop);
+    std::memset(top.get(), 0, sizeof(cm::TreeTop));
+    auto flush = [&]() -> cudaError_t {
+        if (top->count == 0) return cudaSuccess;
+        const cudaError_t e =
+            timed_launch(ctx, kTimeInner, stream, [&] { return cm::launch_tree_top(*top, stream); });
+        std::memset(top.get(), 0, sizeof(cm::TreeTop));
+        return e;
+    };
+    for (size_t i = 0; i < n; ++i) {
+        const Layout &l = lay[i];
+        const uint32_t c = top->count;
+        cm::TreeTopFragment &tf = top->frag[c];
+        tf.levels = (uint32_t)l.sizes.size();
+        size_t a_off = arr_off[i];
+        for (size_t k = 0; k < l.sizes.size(); ++k) {
+            tf.size[k] = l.sizes[k];
+            tf.level[k] = (k + 1 == l.sizes.size()) ? base + 16 * i : base + l.level_off[k];
+            if (k >= 2) {
+                tf.arrivals[k] = reinterpret_cast<uint32_t *>(base + a_off);
+                a_off += (size_t)l.sizes[k] * 4;
+            }
         }
-        CM_CUDA_TRY(flush(), "inner hash launch");
+        tf.tree = l.tp;
+        top->node_begin[c + 1] = top->node_begin[c] + l.sizes[1];
+        top->count = c + 1;
+        if (top->count == (uint32_t)cm::kMaxGroup) CM_CUDA_TRY(flush(), "tree-top launch");
     }
+    CM_CUDA_TRY(flush(), "tree-top launch");
     CM_CUDA_TRY(cudaMemcpyAsync(ctx->h_pinned, base, host_bytes, cudaMemcpyDeviceToHost, stream),
                 "digest copy");
     CM_CUDA_TRY(cudaStreamSynchronize(stream), "ingest synchronisation");

@@ -46,20 +46,26 @@ cudaError_t launch_inner_hash(const uint8_t *children, uint64_t num_children, ui
                               uint64_t num_nodes, uint32_t depth, const TreeParams &tree,
                               cudaStream_t stream);
 
-// All nodes of one tree level of up to kMaxGroup fragments in one launch: thread t
-// hashes node t - node_begin[f] of fragment f (node_begin is the prefix sum of the
-// fragments' node counts at this level).
 constexpr int kMaxGroup = 32;
-struct InnerGroup {
-    uint32_t count;
-    uint32_t depth;
-    uint64_t node_begin[kMaxGroup + 1];
-    const uint8_t *children[kMaxGroup];
-    uint64_t num_children[kMaxGroup];
-    uint8_t *out[kMaxGroup];
-    TreeParams tree[kMaxGroup];
+
+// Every tree level above the leaves, for up to kMaxGroup fragments, in one launch.
+// One thread per level-1 node hashes it; then, level by level, the thread that
+// completes a parent's last child (a per-node arrival counter, zeroed before the
+// launch) hashes that parent, up to the root. No thread ever waits for another.
+constexpr int kMaxLevels = 8;
+struct TreeTopFragment {
+    uint8_t *level[kMaxLevels];       // digests of level k; level[levels - 1] is the root
+    uint64_t size[kMaxLevels];        // nodes of level k
+    uint32_t *arrivals[kMaxLevels];   // per node of level k >= 2: children finished so far
+    uint32_t levels;                  // >= 2
+    TreeParams tree;
 };
-cudaError_t launch_inner_group(const InnerGroup &g, cudaStream_t stream);
+struct TreeTop {
+    uint32_t count;
+    uint64_t node_begin[kMaxGroup + 1];   // prefix sum of the fragments' level-1 sizes
+    TreeTopFragment frag[kMaxGroup];
+};
+cudaError_t launch_tree_top(const TreeTop &t, cudaStream_t stream);
 
 // *flag |= 1 if the `bytes` bytes at a and b differ (16-byte aligned, bytes % 16 == 0).
 cudaError_t launch_compare(const void *a, const void *b, uint64_t bytes, unsigned int *flag,

@@ -237,16 +237,19 @@ struct Item {
     int32_t cs_index;    // first (cos, sin) of this slot
 };
 
+// Item g: pair g / 2 of its slot (row chunk c of (layer, head) plane lh), K if g is
+// even, V if odd.
 __device__ __forceinline__ Item item_of(const RenderParams &p, uint32_t g) {
     int si = 0;
     while (si + 1 < p.num_slots && g >= p.slot[si + 1].chunk_begin) ++si;
     const RenderSlot &S = p.slot[si];
     const uint32_t local = g - S.chunk_begin;
-    const uint32_t plane = local / S.chunks_per_plane;
-    const uint32_t c = local - plane * S.chunks_per_plane;
     const uint32_t lh_planes = (uint32_t)p.num_layers * (uint32_t)p.num_heads;
-    const bool is_v = plane >= lh_planes;            // K planes first, then V planes
-    const int64_t lh = is_v ? plane - lh_planes : plane;
+    const bool is_v = (local & 1u) != 0;             // K and V items alternate
+    const uint32_t pair = local >> 1;
+    const uint32_t lhp = pair / S.chunks_per_plane;
+    const uint32_t c = pair - lhp * S.chunks_per_plane;
+    const int64_t lh = lhp;
     const int64_t row0 = (int64_t)c * p.rows_per_chunk;
     const int64_t left = S.seq_len - row0;
     const int rows = left < p.rows_per_chunk ? (int)left : p.rows_per_chunk;
@@ -322,8 +325,10 @@ __device__ __forceinline__ float2 split16(double c) {
 }
 
 // Persistent kernel, one CTA of kWarps warps per SM; every warp runs its own
-// pipeline over its own items (global item g = warp id + j * total warps), with no
-// block-wide barrier after set-up. Lane 0 keeps up to kStages items in flight as
+// pipeline over its own items, with no block-wide barrier after set-up. Items come
+// in (K, V) pairs of the same (slot, layer, head, row chunk); a warp takes pairs
+// warp id + m * total warps and does the K item, then the V item, so rotation work
+// and pure copies alternate within every warp. Lane 0 keeps up to kStages items in flight as
 // 1-D TMA bulk loads into the warp's stages (completion on one mbarrier per
 // stage); all lanes wait for an item, move it from shared memory to its place in
 // the output (rotating K rows of slots at a nonzero offset), and lane 0 refills the
@@ -351,13 +356,14 @@ render_kernel(const __grid_constant__ RenderParams p) {
 
     const uint32_t first = blockIdx.x * kWarps + warp;
     const uint32_t stride = gridDim.x * kWarps;
-    const uint32_t n = p.total_chunks > first ? (p.total_chunks - first + stride - 1) / stride : 0;
+    const uint32_t npairs = p.total_chunks / 2;
+    const uint32_t n = npairs > first ? 2 * ((npairs - first + stride - 1) / stride) : 0;
     const int lane_v = lane & ((p.head_dim >> 4) - 1);
     uint8_t *wbuf = smem + (size_t)warp * kStages * kItemBytes;
 
     auto produce = [&](uint32_t j) {
         const uint32_t s = j % kStages;
-        const Item it = item_of(p, first + j * stride);
+        const Item it = item_of(p, 2 * (first + (j >> 1) * stride) + (j & 1));
         items[warp][s] = it;
         mbar_arrive_expect_tx(&full[warp][s], it.bytes);
         bulk_load(wbuf + (size_t)s * kItemBytes, it.src, it.bytes, &full[warp][s]);
