@@ -18,7 +18,7 @@
  * capacity_tokens); positions >= the rendered length are left untouched.
  *
  * Conventions fixed by this library where the paper leaves a choice:
- *   - content address: BLAKE2s tree hash (RFC 7693; 1024-byte leaves, fanout 128,
+ *   - content address: BLAKE2s tree hash (RFC 7693; 1024-byte leaves, fanout 16,
  *     16-byte digests, shapes and dtype in the salt, seq_len in the personalisation)
  *     of the byte stream K[0],V[0],...,K[L-1],V[L-1];
  *   - routing layer l* 0-indexed, default floor(L/2); the K-norm score is carried
@@ -124,7 +124,7 @@ cm_status cm_fragment_id(cm_context *ctx, const cm_fragment *frag, cm_stream_t s
  * It computes the same id and norm key as cm_fragment_id on the calling thread's
  * current device, asynchronously on `stream`, and calls no cudaMalloc, cudaFree or
  * other allocating routine: the tree levels below the root live in a static device
- * array of 16.25 MiB that every GPU that loads libcm.so holds until the process
+ * array of 17.25 MiB that every GPU that loads libcm.so holds until the process
  * exits.
  *   routing_layer  l* (0-indexed); < 0 selects floor(num_layers / 2)
  *   id_out         DEVICE, 16-byte aligned, 16 bytes: receives the id

@@ -7,13 +7,13 @@ not name the hash. Reading used here: BLAKE2s (RFC 7693) in its tree mode
 (BLAKE2 paper, Section 2.10), 16-byte digests, computed with hashlib.blake2s.
 
 Byte stream:   K[0] V[0] K[1] V[1] ... K[L-1] V[L-1], each [H][T][d] bf16, little endian
-Every node:    digest_size=16, no key, fanout=128, depth=255, leaf_size=1024,
+Every node:    digest_size=16, no key, fanout=16, depth=255, leaf_size=1024,
                inner_size=16, salt = <L,H,d,1> as four little-endian uint16
                (1 = bf16), person = <T> as a little-endian uint64
 Level 0:       leaf j hashes stream bytes [1024 j, 1024 (j+1)), node_offset=j,
                node_depth=0, last_node set on the final leaf
 Level k >= 1:  node j hashes the concatenated 16-byte digests of children
-               [128 j, 128 j + 128) of level k-1, node_offset=j, node_depth=k,
+               [16 j, 16 j + 16) of level k-1, node_offset=j, node_depth=k,
                last_node set on the final node of the level
 Root:          the digest of the first level k >= 1 that has a single node.
 """
@@ -27,7 +27,7 @@ import numpy as np
 
 DIGEST_SIZE = 16
 LEAF_SIZE = 1024
-FANOUT = 128
+FANOUT = 16
 DEPTH = 255
 DTYPE_CODE_BF16 = 1
 

@@ -3,7 +3,7 @@
 //
 // Id is a BLAKE2s tree hash (RFC 7693 compression function; tree parameters of
 // the BLAKE2 paper, Section 2.10) of the byte stream K[0] V[0] ... K[L-1] V[L-1]:
-// 1024-byte leaves (depth 0), inner nodes over 128 child digests, 16-byte
+// 1024-byte leaves (depth 0), inner nodes over 16 child digests, 16-byte
 // digests, shapes and dtype in the salt, seq_len in the personalisation.
 //
 // Level 0 runs one thread per leaf: 16 compressions of 64-byte blocks, loaded as
@@ -193,33 +193,20 @@ leaf_hash_kernel(const __grid_constant__ LeafLaunch a) {
     StreamCursor cur = cursor_at(a, begin);
     NormState ns{0.0};
 
-    // Two 64-byte blocks (one 128-byte line) per step: eight 16-byte loads in flight.
-    for (uint32_t b = 0; b < nblocks; b += 2) {
-        uint4 w[8];
+    for (uint32_t b = 0; b < nblocks; ++b) {
+        uint4 w[4];
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-            const uint32_t off = b * 64 + q * 16;
-            w[q] = off < len ? load_nc(cursor_next(a, cur)) : make_uint4(0, 0, 0, 0);
-        }
+        for (int q = 0; q < 4; ++q)
+            w[q] = b * 64 + q * 16 < len ? load_nc(cursor_next(a, cur)) : make_uint4(0, 0, 0, 0);
         if (norm_leaf) {
 #pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                const uint32_t off = b * 64 + q * 16;
-                if (off < len) norm_vector(a, ns, w[q], begin + off);
-            }
+            for (int q = 0; q < 4; ++q)
+                if (b * 64 + q * 16 < len) norm_vector(a, ns, w[q], begin + b * 64 + q * 16);
         }
-        {
-            const uint32_t m[16] = {w[0].x, w[0].y, w[0].z, w[0].w, w[1].x, w[1].y, w[1].z, w[1].w,
-                                    w[2].x, w[2].y, w[2].z, w[2].w, w[3].x, w[3].y, w[3].z, w[3].w};
-            const uint32_t end = (b + 1) * 64 < len ? (b + 1) * 64 : len;
-            compress(h, m, end, b + 1 == nblocks, last_node);
-        }
-        if (b + 1 < nblocks) {
-            const uint32_t m[16] = {w[4].x, w[4].y, w[4].z, w[4].w, w[5].x, w[5].y, w[5].z, w[5].w,
-                                    w[6].x, w[6].y, w[6].z, w[6].w, w[7].x, w[7].y, w[7].z, w[7].w};
-            const uint32_t end = (b + 2) * 64 < len ? (b + 2) * 64 : len;
-            compress(h, m, end, b + 2 == nblocks, last_node);
-        }
+        const uint32_t m[16] = {w[0].x, w[0].y, w[0].z, w[0].w, w[1].x, w[1].y, w[1].z, w[1].w,
+                                w[2].x, w[2].y, w[2].z, w[2].w, w[3].x, w[3].y, w[3].z, w[3].w};
+        const uint32_t end = (b + 1) * 64 < len ? (b + 1) * 64 : len;
+        compress(h, m, end, b + 1 == nblocks, last_node);
     }
     store_digest(a.digests + leaf * kDigestBytes, h);
 }
@@ -257,21 +244,23 @@ inner_hash_kernel(const uint8_t *__restrict__ children, uint64_t num_children,
     store_digest(out + j * kDigestBytes, h);
 }
 
-// Node j of a tree level over children digests at `children` (n_children of them):
-// the node's 16 * min(128, n_children - 128 j) bytes are consumed one 64-byte block
-// at a time, the next block's loads issued before the current block is compressed.
-// kCoherent: the children were written by other threads of the same launch, so
-// they are read through L2 (ld.global.cg) instead of the non-coherent path.
+// Loads of child digests. kCoherent: the children were written by other threads of
+// the same launch, so they are read through L2 (ld.global.cg) instead of the
+// non-coherent path.
 template <bool kCoherent>
 __device__ __forceinline__ uint4 load_child(const uint8_t *p) {
     if (kCoherent) return __ldcg(reinterpret_cast<const uint4 *>(p));
     return load_nc(p);
 }
 
+// Node j of a tree level over the digests at `children` (num_children of them):
+// its 16 * min(16, num_children - 16 j) bytes, at most four 64-byte blocks.
 template <bool kCoherent = false>
 __device__ __forceinline__ void hash_inner_node(const uint8_t *children, uint64_t num_children,
                                                 uint8_t *out, uint64_t j, uint64_t num_nodes,
                                                 uint32_t depth, const TreeParams &tp) {
+    // a node's input is at most 16 digests = 256 bytes: all of it is loaded at once
+    static_assert(kFanout * kDigestBytes <= 256, "an inner node must fit four blocks");
     const uint64_t first = j * kFanout;
     const uint64_t nc64 = num_children - first;
     const uint32_t nc = nc64 < (uint64_t)kFanout ? (uint32_t)nc64 : (uint32_t)kFanout;
@@ -281,23 +270,20 @@ __device__ __forceinline__ void hash_inner_node(const uint8_t *children, uint64_
     const uint8_t *src = children + first * kDigestBytes;
     uint32_t h[8];
     node_init(h, tp, j, depth);
-    uint4 nxt[4];
+    uint4 w[16];
 #pragma unroll
-    for (int q = 0; q < 4; ++q)
-        nxt[q] = (uint32_t)(q * 16) < len ? load_child<kCoherent>(src + q * 16) : make_uint4(0, 0, 0, 0);
-    for (uint32_t b = 0; b < nblocks; ++b) {
-        const uint4 w0 = nxt[0], w1 = nxt[1], w2 = nxt[2], w3 = nxt[3];
-        if (b + 1 < nblocks) {
+    for (int q = 0; q < 16; ++q)
+        w[q] = (uint32_t)(q * 16) < len ? load_child<kCoherent>(src + q * 16) : make_uint4(0, 0, 0, 0);
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const uint32_t off = (b + 1) * 64 + q * 16;
-                nxt[q] = off < len ? load_child<kCoherent>(src + off) : make_uint4(0, 0, 0, 0);
-            }
+    for (uint32_t b = 0; b < 4; ++b) {
+        if (b < nblocks) {
+            const uint32_t m[16] = {w[4 * b].x,     w[4 * b].y,     w[4 * b].z,     w[4 * b].w,
+                                    w[4 * b + 1].x, w[4 * b + 1].y, w[4 * b + 1].z, w[4 * b + 1].w,
+                                    w[4 * b + 2].x, w[4 * b + 2].y, w[4 * b + 2].z, w[4 * b + 2].w,
+                                    w[4 * b + 3].x, w[4 * b + 3].y, w[4 * b + 3].z, w[4 * b + 3].w};
+            const uint32_t end = (b + 1) * 64 < len ? (b + 1) * 64 : len;
+            compress(h, m, end, b + 1 == nblocks, last_node);
         }
-        const uint32_t m[16] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w,
-                                w2.x, w2.y, w2.z, w2.w, w3.x, w3.y, w3.z, w3.w};
-        const uint32_t end = (b + 1) * 64 < len ? (b + 1) * 64 : len;
-        compress(h, m, end, b + 1 == nblocks, last_node);
     }
     store_digest(out + j * kDigestBytes, h);
 }
@@ -313,7 +299,7 @@ tree_top_kernel(const __grid_constant__ TreeTop t) {
     hash_inner_node<false>(f.level[0], f.size[0], f.level[1], j, f.size[1], 1, f.tree);
     for (uint32_t k = 1; k + 1 < f.levels; ++k) {
         // this thread finished node j of level k; the one that finishes the last
-        // child of parent j / 128 hashes the parent
+        // child of parent j / 16 hashes the parent
         const uint64_t parent = j / kFanout;
         const uint64_t first = parent * kFanout;
         const uint64_t left = f.size[k] - first;
@@ -395,7 +381,7 @@ namespace cm {
 namespace {
 
 constexpr uint64_t kStaticMaxLeaves = 1ull << 20;                // byte stream of at most 1 GiB
-constexpr size_t kStaticScratchBytes = (16u << 20) + (256u << 10);   // 16.25 MiB
+constexpr size_t kStaticScratchBytes = (17u << 20) + (256u << 10);   // 17.25 MiB
 constexpr int kStaticMaxDevices = 128;
 
 std::mutex g_static_mu;

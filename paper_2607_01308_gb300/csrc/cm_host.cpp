@@ -176,7 +176,7 @@ cm_status ensure_scratch(cm_context *ctx, size_t dev_bytes, size_t host_bytes) {
 }
 
 // BLAKE2s parameter block (32 bytes) of the tree, node offset and depth zero,
-// xored into the IV: digest 16, no key, fanout 128, depth 255 (unlimited),
+// xored into the IV: digest 16, no key, fanout 16, depth 255 (unlimited),
 // leaf 1024, inner 16, salt = <L, H, d, 1 (bf16)> as little-endian uint16,
 // personalisation = <T> as a little-endian uint64.
 cm::TreeParams tree_params(int32_t L, int32_t H, int32_t d, int32_t T) {

@@ -13,10 +13,10 @@ namespace cm {
 
 // ---------------------------------------------------------------- content address
 // BLAKE2s tree mode (RFC 7693 compression; tree parameters of the BLAKE2 paper):
-// 1024-byte leaves, fanout 128, 16-byte node digests.
+// 1024-byte leaves, fanout 16, 16-byte node digests.
 constexpr int kDigestBytes = 16;
 constexpr int kLeafBytes = 1024;
-constexpr int kFanout = 128;
+constexpr int kFanout = 16;
 
 // Chaining value a node starts from: IV xor the 32-byte parameter block with the
 // node offset and node depth fields zero. Kernels xor in offset and depth.
@@ -41,7 +41,7 @@ struct LeafLaunch {
 // Level 0: one thread per leaf; also accumulates the routing-layer norm key.
 cudaError_t launch_leaf_hash(const LeafLaunch &a, cudaStream_t stream);
 
-// Level `depth` >= 1: node j hashes the digests of children [128 j, 128 j + 128).
+// Level `depth` >= 1: node j hashes the digests of children [16 j, 16 j + 16).
 cudaError_t launch_inner_hash(const uint8_t *children, uint64_t num_children, uint8_t *out,
                               uint64_t num_nodes, uint32_t depth, const TreeParams &tree,
                               cudaStream_t stream);
@@ -52,7 +52,7 @@ constexpr int kMaxGroup = 32;
 // One thread per level-1 node hashes it; then, level by level, the thread that
 // completes a parent's last child (a per-node arrival counter, zeroed before the
 // launch) hashes that parent, up to the root. No thread ever waits for another.
-constexpr int kMaxLevels = 8;
+constexpr int kMaxLevels = 12;
 struct TreeTopFragment {
     uint8_t *level[kMaxLevels];       // digests of level k; level[levels - 1] is the root
     uint64_t size[kMaxLevels];        // nodes of level k

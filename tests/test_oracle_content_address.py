@@ -46,7 +46,7 @@ def test_tree_node_parameters_match_independent_blake2s(n):
 def _brute_force_root(stream: bytes, salt: bytes, person: bytes) -> bytes:
     """Level by level with the independent implementation; stop at one node, depth >= 1."""
     def node(data, off, depth, last):
-        return ref.blake2s(data, digest_size=16, last_node=last, fanout=128, depth=255,
+        return ref.blake2s(data, digest_size=16, last_node=last, fanout=ca.FANOUT, depth=255,
                            leaf_size=1024, node_offset=off, node_depth=depth, inner_size=16,
                            salt=salt, person=person)
     chunks = [stream[i:i + 1024] for i in range(0, max(len(stream), 1), 1024)] or [b""]
@@ -54,7 +54,7 @@ def _brute_force_root(stream: bytes, salt: bytes, person: bytes) -> bytes:
     depth = 0
     while True:
         depth += 1
-        groups = [level[i:i + 128] for i in range(0, len(level), 128)]
+        groups = [level[i:i + ca.FANOUT] for i in range(0, len(level), ca.FANOUT)]
         level = [node(b"".join(g), j, depth, j == len(groups) - 1) for j, g in enumerate(groups)]
         if len(level) == 1:
             return level[0]
@@ -84,14 +84,15 @@ def test_stream_order_is_k_then_v_per_layer():
 
 
 def test_level_sizes():
+    assert ca.FANOUT == 16
     assert ca.level_sizes(1) == (1, 1)
     assert ca.level_sizes(1024) == (1, 1)
     assert ca.level_sizes(1025) == (2, 1)
-    assert ca.level_sizes(128 * 1024) == (128, 1)
-    assert ca.level_sizes(128 * 1024 + 1) == (129, 2, 1)
+    assert ca.level_sizes(16 * 1024) == (16, 1)
+    assert ca.level_sizes(16 * 1024 + 1) == (17, 2, 1)
     # Qwen3-4B-shaped fragment, T = 4096: 604 MB -> 589 824 leaves
     n = 36 * 8 * 4096 * 128 * 2 * 2
-    assert ca.level_sizes(n) == (589824, 4608, 36, 1)
+    assert ca.level_sizes(n) == (589824, 36864, 2304, 144, 9, 1)
 
 
 def test_id_sensitive_to_every_byte_and_to_shape():
