@@ -93,6 +93,7 @@ _SIGS = {
                              _c.POINTER(cm_id)]),
     "cm_bagmerge": (_c.c_int, [_P, _c.POINTER(cm_fragment), _c.c_int32, _P, _P, _c.c_int64, _P,
                                _c.POINTER(_c.c_int64)]),
+    "cm_testing_render_withheld_load": (_c.c_int, [_P, _P, _P, _c.c_int64, _P]),
 }
 for _name, (_res, _args) in _SIGS.items():
     _f = getattr(lib, _name)

@@ -8,6 +8,7 @@
 //                                one fused copy-and-rotate launch (Eq. bagmerge-k/v)
 //   cm_bagmerge                  the same launch in a caller-given order (Section 4.2)
 #include "cm.h"
+#include "cm_testing.h"
 
 #include <algorithm>
 #include <array>
@@ -410,7 +411,8 @@ struct Slot {
 // Fused copy-and-rotate of slots already in order (offsets set), in launch groups
 // of at most kMaxSlots slots and kMaxTablePairs (cos, sin) pairs.
 cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t L, int32_t H,
-                       int32_t d, void *k_out, void *v_out, int64_t capacity, cudaStream_t stream) {
+                       int32_t d, void *k_out, void *v_out, int64_t capacity, cudaStream_t stream,
+                       uint32_t withhold_warp = 0) {
     const int rows_per_chunk = cm::kChunkBytes / (2 * d);
     const int half = d / 2;
     const int max_group = std::min<int>(cm::kMaxSlots, cm::kMaxTablePairs / half);
@@ -456,6 +458,7 @@ cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t 
             return fail(CM_ERR_UNSUPPORTED, "render launch group exceeds 2^32 work items");
         p->total_chunks = (uint32_t)chunk;
         p->error = ctx->d_error;
+        p->withhold_warp = g0 == 0 ? withhold_warp : 0;
         const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(chunk, ctx->num_sms));
         CM_CUDA_TRY(timed_launch(ctx, kTimeRender, stream,
                                  [&] { return cm::launch_render(*p, grid, stream); }),
@@ -803,8 +806,11 @@ cm_status cm_set_ids(const cm_set *set, cm_id *out, int64_t capacity) {
     return CM_OK;
 }
 
-cm_status cm_render(const cm_set *set, void *k_out, void *v_out, int64_t capacity_tokens,
-                    cm_stream_t stream, int64_t *out_seq_len, cm_id *out_order) {
+namespace {
+
+cm_status render_set(const cm_set *set, void *k_out, void *v_out, int64_t capacity_tokens,
+                     cm_stream_t stream, int64_t *out_seq_len, cm_id *out_order,
+                     uint32_t withhold_warp) {
     return guarded([&]() -> cm_status {
         if (!set) return fail(CM_ERR_INVALID_ARG, "set is NULL");
         if (capacity_tokens < 0) return fail(CM_ERR_INVALID_ARG, "capacity_tokens < 0");
@@ -829,8 +835,20 @@ cm_status cm_render(const cm_set *set, void *k_out, void *v_out, int64_t capacit
         DeviceScope scope(ctx->device);
         if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
         return launch_slots(ctx, slots, set->L, set->H, set->d, k_out, v_out, capacity_tokens,
-                            reinterpret_cast<cudaStream_t>(stream));
+                            reinterpret_cast<cudaStream_t>(stream), withhold_warp);
     });
+}
+
+}  // namespace
+
+cm_status cm_render(const cm_set *set, void *k_out, void *v_out, int64_t capacity_tokens,
+                    cm_stream_t stream, int64_t *out_seq_len, cm_id *out_order) {
+    return render_set(set, k_out, v_out, capacity_tokens, stream, out_seq_len, out_order, 0);
+}
+
+cm_status cm_testing_render_withheld_load(const cm_set *set, void *k_out, void *v_out,
+                                          int64_t capacity_tokens, cm_stream_t stream) {
+    return render_set(set, k_out, v_out, capacity_tokens, stream, nullptr, nullptr, 1);
 }
 
 cm_status cm_context_check(cm_context *ctx, cm_stream_t stream) {

@@ -106,6 +106,9 @@ struct RenderParams {
     uint32_t total_chunks;
     uint32_t pad_;
     unsigned int *error;        // device word: bit 0 set when a bounded wait timed out
+    uint32_t withhold_warp;     // failure-injection hook: global warp index + 1 whose first
+                                // TMA load is never issued (its wait runs out); 0 = none
+    uint32_t pad2_;
     RenderSlot slot[kMaxSlots];
     double cs[2 * kMaxTablePairs];   // (cos a, sin a) of a = s * theta^(-2j/d), interleaved
 };

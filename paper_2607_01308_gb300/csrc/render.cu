@@ -366,6 +366,7 @@ render_kernel(const __grid_constant__ RenderParams p) {
         const Item it = item_of(p, 2 * (first + (j >> 1) * stride) + (j & 1));
         items[warp][s] = it;
         mbar_arrive_expect_tx(&full[warp][s], it.bytes);
+        if (j == 0 && p.withhold_warp == first + 1) return;   // injected: the wait runs out
         bulk_load(wbuf + (size_t)s * kItemBytes, it.src, it.bytes, &full[warp][s]);
     };
 

@@ -1,0 +1,45 @@
+"""Failure detection on the GPU without a fault: every wait of the render kernel
+on its own TMA copies is bounded (about one second); when one runs out, the warp
+records the failure in the context and returns. A test-only hook withholds one
+copy so that the wait runs out; the host must read CM_ERR_TIMEOUT and the context
+must stay usable. Re-delivery (the paper's fault model, Section 5.9) is covered by
+the absorption tests."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synthetic
+from parity_util import THETA, assert_k_parity, empty_out, gpu_fragments, oracle_fragment
+
+pytestmark = pytest.mark.gpu
+
+cm = pytest.importorskip("paper_2607_01308_gb300")
+
+
+def test_withheld_copy_times_out_and_the_context_recovers():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    ctx = cm.Context(0, THETA)
+    w, frags, _ = gpu_fragments("tiny")
+    S = cm.FragmentSet(ctx)
+    S.ingest_batch(frags)
+    k_out, v_out = empty_out(w.num_layers, w.num_kv_heads, S.seq_len(), w.head_dim)
+    stream = torch.cuda.current_stream()
+    st = cm.lib.cm_testing_render_withheld_load(S.handle, k_out.data_ptr(), v_out.data_ptr(),
+                                                S.seq_len(), stream.cuda_stream or None)
+    assert st == cm.Status.OK
+    with pytest.raises(cm.CMError) as e:
+        ctx.check()
+    assert e.value.status == cm.Status.ERR_TIMEOUT
+    ctx.check()   # reported once, then cleared
+    # the context still works: a normal render matches the oracle
+    n, order = S.render(k_out, v_out)
+    ctx.check()
+    ref = oracle.from_deliveries([oracle_fragment(K, V) for K, V in frags])
+    K_ref, V_ref, o_order = oracle.render(ref, THETA)
+    assert order == [f.fid for f in o_order]
+    assert np.array_equal(synthetic.to_bits(v_out), V_ref)
+    assert assert_k_parity(synthetic.to_bits(k_out), K_ref) == 0
+    S.close()
+    ctx.close()

@@ -274,3 +274,80 @@ def test_union_algebra_and_render_invariance(ctx):
     assert assert_k_parity(ref_bits[0], K_ref) == 0
     for S in singles:
         S.close()
+
+
+# ---------------------------------------------------------------- launch-group boundaries
+
+def test_forty_fragments_span_two_render_and_two_tree_launches(ctx):
+    # more fragments than one render launch (32 slots) or one tree-top launch (32) holds
+    L, H, d = 2, 1, 64
+    g = torch.Generator(device="cuda:0").manual_seed(40)
+    frags = []
+    for i in range(40):
+        T = 1 + (i * 37) % 50
+        K = (torch.randn((L, H, T, d), generator=g, device="cuda:0") * (0.5 + 0.02 * i)).to(torch.bfloat16)
+        V = torch.randn((L, H, T, d), generator=g, device="cuda:0").to(torch.bfloat16)
+        frags.append((K, V))
+    cm.cm_context_kernel_times(ctx.handle, reset=True)
+    cm.cm_context_set_timing(ctx.handle, True)
+    S = cm.FragmentSet(ctx)
+    res = S.ingest_batch(frags)
+    total = S.seq_len()
+    k_out, v_out = empty_out(L, H, total, d)
+    n, order = S.render(k_out, v_out)
+    cm.cm_context_set_timing(ctx.handle, False)
+    t = cm.cm_context_kernel_times(ctx.handle, reset=True)
+    assert t["render_launches"] == 2 and t["inner_hash_launches"] == 2
+    ref_frags = [oracle_fragment(K, V) for K, V in frags]
+    assert [r[0] for r in res] == [f.fid for f in ref_frags]
+    K_ref, V_ref, o_order = oracle.render(oracle.from_deliveries(ref_frags), THETA)
+    assert order == [f.fid for f in o_order]
+    assert np.array_equal(synthetic.to_bits(v_out), V_ref)
+    assert assert_k_parity(synthetic.to_bits(k_out), K_ref) == 0
+    S.close()
+
+
+def test_head_dim_512_spans_table_limited_render_groups(ctx):
+    # 1792 (cos, sin) pairs per launch = 7 slots at d = 512: nine fragments need two launches
+    L, H, d = 2, 1, 512
+    g = torch.Generator(device="cuda:0").manual_seed(512)
+    frags = []
+    for i in range(9):
+        T = 3 + 5 * i
+        K = (torch.randn((L, H, T, d), generator=g, device="cuda:0") * (0.5 + 0.1 * i)).to(torch.bfloat16)
+        V = torch.randn((L, H, T, d), generator=g, device="cuda:0").to(torch.bfloat16)
+        frags.append((K, V))
+    S = cm.FragmentSet(ctx)
+    S.ingest_batch(frags)
+    k_out, v_out = empty_out(L, H, S.seq_len(), d)
+    n, order = S.render(k_out, v_out)
+    torch.cuda.synchronize()
+    ref_frags = [oracle_fragment(K, V) for K, V in frags]
+    K_ref, V_ref, o_order = oracle.render(oracle.from_deliveries(ref_frags), THETA)
+    assert order == [f.fid for f in o_order]
+    assert np.array_equal(synthetic.to_bits(v_out), V_ref)
+    assert assert_k_parity(synthetic.to_bits(k_out), K_ref) == 0
+    S.close()
+
+
+def test_long_fragment_and_large_offsets(ctx):
+    # T = 40000 tokens in slot 0 pushes the other slots' offsets past 40000 (angles of
+    # thousands of radians at the highest frequency)
+    L, H, d = 1, 2, 128
+    g = torch.Generator(device="cuda:0").manual_seed(9)
+    big = ((torch.randn((L, H, 40000, d), generator=g, device="cuda:0") * 3).to(torch.bfloat16),
+           torch.randn((L, H, 40000, d), generator=g, device="cuda:0").to(torch.bfloat16))
+    small = [((torch.randn((L, H, T, d), generator=g, device="cuda:0") * 0.3).to(torch.bfloat16),
+              torch.randn((L, H, T, d), generator=g, device="cuda:0").to(torch.bfloat16)) for T in (333, 4096)]
+    frags = [big] + small
+    S = cm.FragmentSet(ctx)
+    S.ingest_batch(frags)
+    k_out, v_out = empty_out(L, H, S.seq_len(), d)
+    n, order = S.render(k_out, v_out)
+    torch.cuda.synchronize()
+    ref_frags = [oracle_fragment(K, V) for K, V in frags]
+    K_ref, V_ref, o_order = oracle.render(oracle.from_deliveries(ref_frags), THETA)
+    assert order == [f.fid for f in o_order] and order[0] == ref_frags[0].fid
+    assert np.array_equal(synthetic.to_bits(v_out), V_ref)
+    assert assert_k_parity(synthetic.to_bits(k_out), K_ref) == 0
+    S.close()
