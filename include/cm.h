@@ -197,6 +197,51 @@ cm_status cm_set_ids(const cm_set *set, cm_id *out, int64_t capacity);
 cm_status cm_render(const cm_set *set, void *k_out, void *v_out, int64_t capacity_tokens,
                     cm_stream_t stream, int64_t *out_seq_len, cm_id *out_order);
 
+/* Incremental Render(S) (addresses the lazy O(m) re-render of Section 7): k_out and
+ * v_out already hold the render of an earlier state whose canonical order was
+ * prev_order[0..prev_n) (as returned by cm_render / this call). Slots of the longest
+ * common prefix of that order and the set's new canonical order keep their offsets,
+ * so their bytes are left in place; every later slot is rendered again from its
+ * unshifted fragment (a shifted slot cannot be re-rotated from its previous render
+ * without a second rounding). The result is byte-identical to cm_render into a fresh
+ * buffer. The caller guarantees that the buffer holds what prev_order says (the
+ * library cannot check it); prev_n = 0 is a full render.
+ *   out_reused_tokens  nullable; receives the number of tokens left in place
+ * Other arguments and the asynchrony are as for cm_render. */
+cm_status cm_render_incremental(const cm_set *set, void *k_out, void *v_out,
+                                int64_t capacity_tokens, const cm_id *prev_order, int64_t prev_n,
+                                cm_stream_t stream, int64_t *out_seq_len, cm_id *out_order,
+                                int64_t *out_reused_tokens);
+
+/* A paged KV cache (PagedAttention-style block pools) as a render destination.
+ * Token position pos of (layer l, kv head h) lives at element
+ *   block_table[pos / block_size] * stride_block + l * stride_layer + h * stride_head
+ *   + (pos % block_size) * stride_token
+ * of k_pool (K) and v_pool (V); head_dim elements are contiguous from there. Strides
+ * are in bf16 elements and must be multiples of 8 (16 bytes); pools 16-byte aligned.
+ * This covers the usual layouts, e.g. per-layer pools [L][num_blocks][block_size][H][d]
+ * or block-major [num_blocks][L][H][block_size][d]. */
+typedef struct cm_paged_cache {
+    void *k_pool;                 /* DEVICE */
+    void *v_pool;                 /* DEVICE */
+    const int32_t *block_table;   /* DEVICE: logical block -> physical block index */
+    int64_t table_entries;        /* capacity = table_entries * block_size tokens */
+    int64_t block_size;           /* tokens per block, >= 1 */
+    int64_t stride_block;
+    int64_t stride_layer;
+    int64_t stride_head;
+    int64_t stride_token;
+} cm_paged_cache;
+
+/* Render(S) (Algorithm 2; Algorithm 1) into a paged cache: the same bytes as cm_render,
+ * each merged position written to its block (Section 4.5: the merge is compatible with
+ * PagedAttention-style block-addressable caches). The physical blocks named by the first
+ * ceil(rendered length / block_size) table entries must be distinct and inside the pools
+ * (the table is on the device and is not checked); positions beyond the rendered length
+ * are left untouched. CM_ERR_CAPACITY if the table is too short. Asynchronous on `stream`. */
+cm_status cm_render_paged(const cm_set *set, const cm_paged_cache *out, cm_stream_t stream,
+                          int64_t *out_seq_len, cm_id *out_order);
+
 /* BagMerge (Section 4.2, Eq. bagmerge-k / bagmerge-v) in the caller's order:
  * frags[0] at offset 0 (byte copy), frags[i] at the sum of the previous seq_len,
  * K rotated by R(offset), V copied. No content address, no dedup: passing the same

@@ -63,6 +63,14 @@ class cm_kernel_times(ctypes.Structure):
         return {name: getattr(self, name) for name, _ in self._fields_}
 
 
+class cm_paged_cache(ctypes.Structure):
+    _fields_ = [("k_pool", ctypes.c_void_p), ("v_pool", ctypes.c_void_p),
+                ("block_table", ctypes.c_void_p), ("table_entries", ctypes.c_int64),
+                ("block_size", ctypes.c_int64), ("stride_block", ctypes.c_int64),
+                ("stride_layer", ctypes.c_int64), ("stride_head", ctypes.c_int64),
+                ("stride_token", ctypes.c_int64)]
+
+
 _c = ctypes
 _P = ctypes.c_void_p
 _SIGS = {
@@ -94,6 +102,11 @@ _SIGS = {
     "cm_bagmerge": (_c.c_int, [_P, _c.POINTER(cm_fragment), _c.c_int32, _P, _P, _c.c_int64, _P,
                                _c.POINTER(_c.c_int64)]),
     "cm_testing_render_withheld_load": (_c.c_int, [_P, _P, _P, _c.c_int64, _P]),
+    "cm_render_paged": (_c.c_int, [_P, _c.POINTER(cm_paged_cache), _P, _c.POINTER(_c.c_int64),
+                                   _c.POINTER(cm_id)]),
+    "cm_render_incremental": (_c.c_int, [_P, _P, _P, _c.c_int64, _c.POINTER(cm_id), _c.c_int64, _P,
+                                         _c.POINTER(_c.c_int64), _c.POINTER(cm_id),
+                                         _c.POINTER(_c.c_int64)]),
 }
 for _name, (_res, _args) in _SIGS.items():
     _f = getattr(lib, _name)
@@ -237,6 +250,30 @@ def cm_render(s: int, k_out: int, v_out: int, capacity_tokens: int,
     return seq.value, [order[i].to_bytes() for i in range(n)]
 
 
+def cm_render_incremental(s: int, k_out: int, v_out: int, capacity_tokens: int,
+                          prev_order: Sequence[bytes], stream=None) -> Tuple[int, List[bytes], int]:
+    n = cm_set_size(s)
+    order = (cm_id * max(n, 1))()
+    prev = (cm_id * max(len(prev_order), 1))()
+    for i, fid in enumerate(prev_order):
+        prev[i].b[:] = list(fid)
+    seq = ctypes.c_int64()
+    reused = ctypes.c_int64()
+    _check(lib.cm_render_incremental(s, k_out, v_out, capacity_tokens, prev, len(prev_order),
+                                     _stream_handle(stream), ctypes.byref(seq), order,
+                                     ctypes.byref(reused)))
+    return seq.value, [order[i].to_bytes() for i in range(n)], reused.value
+
+
+def cm_render_paged(s: int, cache: cm_paged_cache, stream=None) -> Tuple[int, List[bytes]]:
+    n = cm_set_size(s)
+    order = (cm_id * max(n, 1))()
+    seq = ctypes.c_int64()
+    _check(lib.cm_render_paged(s, ctypes.byref(cache), _stream_handle(stream), ctypes.byref(seq),
+                               order))
+    return seq.value, [order[i].to_bytes() for i in range(n)]
+
+
 def cm_bagmerge(ctx: int, frags: Sequence[cm_fragment], k_out: int, v_out: int,
                 capacity_tokens: int, stream=None) -> int:
     arr = (cm_fragment * max(len(frags), 1))(*frags)
@@ -341,6 +378,11 @@ class FragmentSet:
 
     def seq_len(self) -> int:
         return cm_set_seq_len(self.handle)
+
+    def render_incremental(self, k_out, v_out, prev_order, stream=None):
+        """(seq_len, order, reused_tokens): re-render only what changed since prev_order."""
+        return cm_render_incremental(self.handle, k_out.data_ptr(), v_out.data_ptr(),
+                                     k_out.shape[2], prev_order, stream)
 
     def render(self, k_out, v_out, stream=None) -> Tuple[int, List[bytes]]:
         return cm_render(self.handle, k_out.data_ptr() if k_out is not None else 0,

@@ -412,7 +412,7 @@ struct Slot {
 // of at most kMaxSlots slots and kMaxTablePairs (cos, sin) pairs.
 cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t L, int32_t H,
                        int32_t d, void *k_out, void *v_out, int64_t capacity, cudaStream_t stream,
-                       uint32_t withhold_warp = 0) {
+                       uint32_t withhold_warp = 0, const cm_paged_cache *paged = nullptr) {
     const int rows_per_chunk = cm::kChunkBytes / (2 * d);
     const int half = d / 2;
     const int max_group = std::min<int>(cm::kMaxSlots, cm::kMaxTablePairs / half);
@@ -459,6 +459,15 @@ cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t 
         p->total_chunks = (uint32_t)chunk;
         p->error = ctx->d_error;
         p->withhold_warp = g0 == 0 ? withhold_warp : 0;
+        if (paged) {
+            p->paged = 1;
+            p->block_table = paged->block_table;
+            p->block_size = paged->block_size;
+            p->stride_block = paged->stride_block;
+            p->stride_layer = paged->stride_layer;
+            p->stride_head = paged->stride_head;
+            p->stride_token = paged->stride_token;
+        }
         const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(chunk, ctx->num_sms));
         CM_CUDA_TRY(timed_launch(ctx, kTimeRender, stream,
                                  [&] { return cm::launch_render(*p, grid, stream); }),
@@ -810,32 +819,56 @@ namespace {
 
 cm_status render_set(const cm_set *set, void *k_out, void *v_out, int64_t capacity_tokens,
                      cm_stream_t stream, int64_t *out_seq_len, cm_id *out_order,
-                     uint32_t withhold_warp) {
+                     uint32_t withhold_warp, const cm_id *prev_order = nullptr,
+                     int64_t prev_n = 0, int64_t *out_reused_tokens = nullptr,
+                     const cm_paged_cache *paged = nullptr) {
     return guarded([&]() -> cm_status {
         if (!set) return fail(CM_ERR_INVALID_ARG, "set is NULL");
         if (capacity_tokens < 0) return fail(CM_ERR_INVALID_ARG, "capacity_tokens < 0");
+        if (prev_n < 0 || (prev_n > 0 && !prev_order))
+            return fail(CM_ERR_INVALID_ARG, "prev_order is NULL or prev_n < 0");
         int64_t total = 0;
         for (const auto &kv : set->items) total += kv.second->T;
         cm_status st = validate_outputs(k_out, v_out, capacity_tokens, total);
         if (st != CM_OK) return st;
+        if (paged && total > 0) {
+            if (!paged->block_table) return fail(CM_ERR_INVALID_ARG, "block_table is NULL");
+            if (paged->block_size < 1) return fail(CM_ERR_INVALID_ARG, "block_size < 1");
+            if (paged->stride_block % 8 || paged->stride_layer % 8 || paged->stride_head % 8 ||
+                paged->stride_token % 8 || paged->stride_block < 0 || paged->stride_layer < 0 ||
+                paged->stride_head < 0 || paged->stride_token < 0)
+                return fail(CM_ERR_ALIGNMENT, "paged strides must be non-negative multiples of 8 elements");
+            if (paged->stride_token < set->d)
+                return fail(CM_ERR_INVALID_ARG, "stride_token is smaller than head_dim");
+        }
         const auto order = canonical_order(set);
         if (out_seq_len) *out_seq_len = total;
         if (out_order)
             for (size_t i = 0; i < order.size(); ++i) out_order[i] = order[i]->id;
-        if (order.empty()) return CM_OK;
+        // slots of the common prefix of the previous and the new canonical order keep
+        // their offsets, so their bytes in the buffer are already the render's
+        size_t keep = 0;
+        while (keep < order.size() && (int64_t)keep < prev_n &&
+               std::memcmp(order[keep]->id.b, prev_order[keep].b, 16) == 0)
+            ++keep;
         std::vector<Slot> slots;
         slots.reserve(order.size());
-        int64_t s = 0;
-        for (const auto &r : order) {
-            slots.push_back({r->k, r->v, r->T, s});
-            s += r->T;
+        int64_t s = 0, reused = 0;
+        for (size_t i = 0; i < order.size(); ++i) {
+            if (i < keep)
+                reused += order[i]->T;
+            else
+                slots.push_back({order[i]->k, order[i]->v, order[i]->T, s});
+            s += order[i]->T;
         }
+        if (out_reused_tokens) *out_reused_tokens = reused;
+        if (slots.empty()) return CM_OK;
         cm_context *ctx = set->ctx;
         std::lock_guard<std::mutex> lock(ctx->mu);
         DeviceScope scope(ctx->device);
         if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
         return launch_slots(ctx, slots, set->L, set->H, set->d, k_out, v_out, capacity_tokens,
-                            reinterpret_cast<cudaStream_t>(stream), withhold_warp);
+                            reinterpret_cast<cudaStream_t>(stream), withhold_warp, paged);
     });
 }
 
@@ -844,6 +877,25 @@ cm_status render_set(const cm_set *set, void *k_out, void *v_out, int64_t capaci
 cm_status cm_render(const cm_set *set, void *k_out, void *v_out, int64_t capacity_tokens,
                     cm_stream_t stream, int64_t *out_seq_len, cm_id *out_order) {
     return render_set(set, k_out, v_out, capacity_tokens, stream, out_seq_len, out_order, 0);
+}
+
+cm_status cm_render_incremental(const cm_set *set, void *k_out, void *v_out,
+                                int64_t capacity_tokens, const cm_id *prev_order, int64_t prev_n,
+                                cm_stream_t stream, int64_t *out_seq_len, cm_id *out_order,
+                                int64_t *out_reused_tokens) {
+    return render_set(set, k_out, v_out, capacity_tokens, stream, out_seq_len, out_order, 0,
+                      prev_order, prev_n, out_reused_tokens);
+}
+
+cm_status cm_render_paged(const cm_set *set, const cm_paged_cache *out, cm_stream_t stream,
+                          int64_t *out_seq_len, cm_id *out_order) {
+    if (!out) return fail(CM_ERR_INVALID_ARG, "paged cache descriptor is NULL");
+    if (out->table_entries < 0 || out->block_size < 1)
+        return fail(CM_ERR_INVALID_ARG, "table_entries < 0 or block_size < 1");
+    if (out->table_entries > INT64_MAX / out->block_size)
+        return fail(CM_ERR_INVALID_ARG, "table capacity overflows");
+    return render_set(set, out->k_pool, out->v_pool, out->table_entries * out->block_size, stream,
+                      out_seq_len, out_order, 0, nullptr, 0, nullptr, out);
 }
 
 cm_status cm_testing_render_withheld_load(const cm_set *set, void *k_out, void *v_out,

@@ -108,7 +108,13 @@ struct RenderParams {
     unsigned int *error;        // device word: bit 0 set when a bounded wait timed out
     uint32_t withhold_warp;     // failure-injection hook: global warp index + 1 whose first
                                 // TMA load is never issued (its wait runs out); 0 = none
-    uint32_t pad2_;
+    int32_t paged;              // 1: outputs are block pools addressed through block_table
+    // paged output: token pos of (layer l, head h) lives at pool + block_table[pos / block_size]
+    // * stride_block + l * stride_layer + h * stride_head + (pos % block_size) * stride_token
+    // (element strides, head_dim contiguous); k_out / v_out are the pools
+    const int32_t *block_table; // device
+    int64_t block_size;
+    int64_t stride_block, stride_layer, stride_head, stride_token;
     RenderSlot slot[kMaxSlots];
     double cs[2 * kMaxTablePairs];   // (cos a, sin a) of a = s * theta^(-2j/d), interleaved
 };

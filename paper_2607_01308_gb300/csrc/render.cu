@@ -230,7 +230,8 @@ static_assert(kChunkBytes == (int)kItemBytes, "host and kernel disagree on the w
 // One work item: up to kItemBytes of one source plane and where it goes.
 struct Item {
     const uint8_t *src;
-    uint8_t *dst;
+    uint8_t *dst;        // contiguous: first output row; paged: pool + (layer, head) offset
+    int64_t pos0;        // output position of the first row (paged outputs)
     uint32_t bytes;
     int32_t rows;
     int32_t rotate;      // 1: K of a slot at a nonzero offset
@@ -256,8 +257,15 @@ __device__ __forceinline__ Item item_of(const RenderParams &p, uint32_t g) {
     const int64_t row_bytes = (int64_t)p.head_dim * 2;
     Item it;
     it.src = static_cast<const uint8_t *>(is_v ? S.v : S.k) + (lh * S.seq_len + row0) * row_bytes;
-    it.dst = static_cast<uint8_t *>(is_v ? p.v_out : p.k_out) +
-             (lh * p.capacity + S.offset + row0) * row_bytes;
+    if (p.paged) {
+        const int64_t l = lh / p.num_heads, h = lh - l * p.num_heads;
+        it.dst = static_cast<uint8_t *>(is_v ? p.v_out : p.k_out) +
+                 (l * p.stride_layer + h * p.stride_head) * 2;
+    } else {
+        it.dst = static_cast<uint8_t *>(is_v ? p.v_out : p.k_out) +
+                 (lh * p.capacity + S.offset + row0) * row_bytes;
+    }
+    it.pos0 = S.offset + row0;
     it.bytes = (uint32_t)(rows * row_bytes);
     it.rows = rows;
     it.rotate = (!is_v && S.rotate) ? 1 : 0;
@@ -265,24 +273,47 @@ __device__ __forceinline__ Item item_of(const RenderParams &p, uint32_t g) {
     return it;
 }
 
+// Start of output row r of an item: contiguous rows, or the row's slot in its block.
+template <bool kPaged>
+__device__ __forceinline__ uint4 *row_dst(const RenderParams &p, const Item &it, int r) {
+    if (!kPaged) return reinterpret_cast<uint4 *>(it.dst) + (int64_t)r * (p.head_dim >> 3);
+    const int64_t pos = it.pos0 + r;
+    const int64_t blk = __ldg(p.block_table + pos / p.block_size);
+    return reinterpret_cast<uint4 *>(it.dst +
+                                     (blk * p.stride_block + (pos % p.block_size) * p.stride_token) * 2);
+}
+
 // Byte copy of one staged item: shared memory -> registers -> 16-byte streaming stores.
-__device__ __forceinline__ void copy_from_smem(const Item &it, const uint8_t *buf, int lane) {
+template <bool kPaged>
+__device__ __forceinline__ void copy_from_smem(const RenderParams &p, const Item &it,
+                                               const uint8_t *buf, int lane) {
     constexpr int kU = kItemBytes / 16 / 32;          // 8 vectors per lane
     const int n_vec = (int)(it.bytes >> 4);
     const uint4 *src = reinterpret_cast<const uint4 *>(buf);
-    uint4 *dst = reinterpret_cast<uint4 *>(it.dst);
     uint4 r[kU];
 #pragma unroll
     for (int u = 0; u < kU; ++u)
         if (lane + 32 * u < n_vec) r[u] = src[lane + 32 * u];
+    if (!kPaged) {
+        uint4 *dst = reinterpret_cast<uint4 *>(it.dst);
 #pragma unroll
-    for (int u = 0; u < kU; ++u)
-        if (lane + 32 * u < n_vec) st_stream(dst + lane + 32 * u, r[u]);
+        for (int u = 0; u < kU; ++u)
+            if (lane + 32 * u < n_vec) st_stream(dst + lane + 32 * u, r[u]);
+    } else {
+        const int log2_vpr = p.log2_pairs_per_row + 1;     // vectors per row = d / 8
+        const int col_mask = (1 << log2_vpr) - 1;
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+            const int v = lane + 32 * u;
+            if (v < n_vec) st_stream(row_dst<true>(p, it, v >> log2_vpr) + (v & col_mask), r[u]);
+        }
+    }
 }
 
 // K rows of one staged item: rotate and store. Lane `lane` takes vector pairs
 // q = lane, lane + 32, ...; its vector index within the row half is lane % (d/16),
 // the same for every q, so its 8 (cos, sin) values are loaded once per item.
+template <bool kPaged>
 __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const float4 *tab,
                                                  const Item &it, const uint8_t *buf, int lane,
                                                  int lane_v) {
@@ -298,7 +329,6 @@ __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const fl
         s[e] = __fadd_rn(t.z, t.w);
     }
     const uint4 *src = reinterpret_cast<const uint4 *>(buf);
-    uint4 *dst = reinterpret_cast<uint4 *>(it.dst);
 #pragma unroll 2
     for (int q = lane; q < n_pairs; q += 32) {
         const int row = q >> p.log2_pairs_per_row;
@@ -312,8 +342,9 @@ __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const fl
         rotate_word(a.z, b.z, c[4], s[4], c[5], s[5], ao.z, bo.z, b2);
         rotate_word(a.w, b.w, c[6], s[6], c[7], s[7], ao.w, bo.w, b3);
         if ((b0 | b1 | b2 | b3) != 0u) fixup_pair(p, tab, cs_index, a, b, b0, b1, b2, b3, ao, bo);
-        st_stream(dst + off, ao);
-        st_stream(dst + off + half_vecs, bo);
+        uint4 *d = row_dst<kPaged>(p, it, row) + lane_v;
+        st_stream(d, ao);
+        st_stream(d + half_vecs, bo);
     }
 }
 
@@ -334,6 +365,7 @@ __device__ __forceinline__ float2 split16(double c) {
 // the output (rotating K rows of slots at a nonzero offset), and lane 0 refills the
 // stage with the warp's next item. Every wait is bounded: on timeout the warp
 // records an error, waits (bounded) for its own copies in flight and returns.
+template <bool kPaged>
 __global__ void __launch_bounds__(kThreads, 1)
 render_kernel(const __grid_constant__ RenderParams p) {
     extern __shared__ __align__(128) uint8_t smem[];
@@ -386,9 +418,9 @@ render_kernel(const __grid_constant__ RenderParams p) {
         const Item it = items[warp][s];
         const uint8_t *buf = wbuf + (size_t)s * kItemBytes;
         if (it.rotate)
-            rotate_from_smem(p, tab, it, buf, lane, lane_v);
+            rotate_from_smem<kPaged>(p, tab, it, buf, lane, lane_v);
         else
-            copy_from_smem(it, buf, lane);
+            copy_from_smem<kPaged>(p, it, buf, lane);
         __syncwarp();                          // every lane is done reading stage s
         if (lane == 0 && produced < n) {
             fence_proxy_async_smem();
@@ -407,13 +439,19 @@ render_kernel(const __grid_constant__ RenderParams p) {
 int render_threads_per_block() { return kThreads; }
 
 cudaError_t render_prepare() {
-    return cudaFuncSetAttribute(render_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(render_kernel<false>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kDynSmem);
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(render_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)kDynSmem);
 }
 
 cudaError_t launch_render(const RenderParams &p, int grid, cudaStream_t stream) {
     if (p.total_chunks == 0) return cudaSuccess;
-    render_kernel<<<grid, kThreads, kDynSmem, stream>>>(p);
+    if (p.paged)
+        render_kernel<true><<<grid, kThreads, kDynSmem, stream>>>(p);
+    else
+        render_kernel<false><<<grid, kThreads, kDynSmem, stream>>>(p);
     return cudaGetLastError();
 }
 

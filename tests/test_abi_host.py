@@ -30,7 +30,8 @@ def test_header_declares_the_documented_calls():
             "cm_set_destroy", "cm_fragment_id", "cm_ingest", "cm_union", "cm_set_size",
             "cm_set_seq_len", "cm_set_ids", "cm_render", "cm_bagmerge", "cm_status_string",
             "cm_last_error_message", "cm_context_check", "cm_ingest_batch",
-            "cm_context_set_timing", "cm_context_kernel_times", "cm_fragment_id_static"}
+            "cm_context_set_timing", "cm_context_kernel_times", "cm_fragment_id_static",
+            "cm_render_incremental", "cm_render_paged"}
     assert want <= set(_declared_functions())
 
 
@@ -72,6 +73,9 @@ def test_null_and_range_arguments_rejected_without_cuda(cm):
     assert lib.cm_ingest_batch(None, None, 0, None, None, None) == cm.Status.ERR_INVALID_ARG
     assert lib.cm_context_set_timing(None, 1) == cm.Status.ERR_INVALID_ARG
     assert lib.cm_context_kernel_times(None, None, 0) == cm.Status.ERR_INVALID_ARG
+    assert lib.cm_render_paged(None, None, None, None, None) == cm.Status.ERR_INVALID_ARG
+    assert lib.cm_render_incremental(None, None, None, 0, None, 0, None, None, None,
+                                     None) == cm.Status.ERR_INVALID_ARG
     # destroying NULL handles is a no-op
     assert lib.cm_set_destroy(None) == cm.Status.OK
     assert lib.cm_context_destroy(None) == cm.Status.OK
