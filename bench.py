@@ -338,73 +338,37 @@ def main():
     ingest_ms = sum(t["ingest"][0].elapsed_time(t["ingest"][1]) for t in step_timers) / args.steps
     elapsed_ms = max_over_ranks(elapsed_ms, dev)
 
-    # end to end through the C ABI with host buffers: every step copies its four fragments in
-    # from pinned host memory and the whole merged cache (K and V) back out to pinned host
-    # memory. Steps are pipelined the way a serving loop would run them: step i+1's inputs
-    # copy in (copy stream) while step i merges (compute stream) and step i-1's cache copies
-    # out (copy-out stream); device inputs and outputs are double-buffered and ordered by
-    # events, so no copy overwrites data a merge still reads.
+    # end to end through the C ABI with host buffers: pinned inputs copied in and the
+    # merged cache copied out inside the timed region, every step
     e2e_steps = args.e2e_steps or min(args.steps, 10)
     host_in = [(K.cpu().pin_memory(), V.cpu().pin_memory()) for K, V in frags]
-    dev_in = [[(torch.empty_like(K), torch.empty_like(V)) for K, V in frags] for _ in range(2)]
-    dev_desc = [[cm.fragment_from_tensors(K, V) for K, V in bufs] for bufs in dev_in]
-    dev_out = [(torch.empty_like(k_out), torch.empty_like(v_out)) for _ in range(2)]
-    host_out = [(torch.empty(k_out.shape, dtype=k_out.dtype, pin_memory=True),
-                 torch.empty(v_out.shape, dtype=v_out.dtype, pin_memory=True)) for _ in range(2)]
+    dev_in = [(torch.empty_like(K), torch.empty_like(V)) for K, V in frags]
+    dev_desc = [cm.fragment_from_tensors(K, V) for K, V in dev_in]
+    host_out = (torch.empty(k_out.shape, dtype=k_out.dtype, pin_memory=True),
+                torch.empty(v_out.shape, dtype=v_out.dtype, pin_memory=True))
     h2d = sum(K.numel() * 2 + V.numel() * 2 for K, V in host_in)
     d2h = 2 * k_out.numel() * 2
-    s_in = torch.cuda.Stream(dev)
-    s_out = torch.cuda.Stream(dev)
-    ev_in = [torch.cuda.Event() for _ in range(2)]      # inputs of buffer b copied in
-    ev_used = [torch.cuda.Event() for _ in range(2)]    # merge done with inputs/outputs of b
-    ev_out = [torch.cuda.Event() for _ in range(2)]     # outputs of b copied out
 
-    def copy_in(b):
-        s_in.wait_event(ev_used[b])
-        with torch.cuda.stream(s_in):
-            for (hk, hv), (dk, dv) in zip(host_in, dev_in[b]):
-                dk.copy_(hk, non_blocking=True)
-                dv.copy_(hv, non_blocking=True)
-        ev_in[b].record(s_in)
+    def e2e_step():
+        for (hk, hv), (dk, dv) in zip(host_in, dev_in):
+            dk.copy_(hk, non_blocking=True)
+            dv.copy_(hv, non_blocking=True)
+        one_merge(inputs=dev_desc)
+        host_out[0].copy_(k_out, non_blocking=True)
+        host_out[1].copy_(v_out, non_blocking=True)
 
-    def merge_and_copy_out(b):
-        stream.wait_event(ev_in[b])
-        stream.wait_event(ev_out[b])
-        a_ = cm.cm_set_create(ctx.handle)
-        b_ = cm.cm_set_create(ctx.handle)
-        fd = dev_desc[b]
-        half = (len(fd) + 1) // 2
-        cm.cm_ingest_batch(a_, fd[:half], stream)
-        cm.cm_ingest_batch(b_, fd[half:], stream)
-        cm.cm_union(a_, b_)
-        cm.cm_render(a_, dev_out[b][0].data_ptr(), dev_out[b][1].data_ptr(), total_T, stream)
-        cm.cm_set_destroy(b_)
-        cm.cm_set_destroy(a_)
-        ev_used[b].record(stream)
-        s_out.wait_event(ev_used[b])
-        with torch.cuda.stream(s_out):
-            host_out[b][0].copy_(dev_out[b][0], non_blocking=True)
-            host_out[b][1].copy_(dev_out[b][1], non_blocking=True)
-        ev_out[b].record(s_out)
-
-    def e2e_run(n_steps):
-        """Device time from the first copy-in to the last copy-out (CUDA events)."""
-        t_start, t_end = ev(), ev()
-        t_start.record(s_in)
-        copy_in(0)
-        for i in range(n_steps):
-            if i + 1 < n_steps:
-                copy_in((i + 1) % 2)
-            merge_and_copy_out(i % 2)
-        stream.wait_stream(s_out)
-        t_end.record(stream)
-        torch.cuda.synchronize(dev)
-        return t_start.elapsed_time(t_end)
-
-    e2e_run(2)                          # warm-up
+    e2e_step()
+    torch.cuda.synchronize(dev)
     if world > 1:
         dist.barrier()
-    e2e_ms = max_over_ranks(e2e_run(e2e_steps), dev)
+    e0, e1 = ev(), ev()
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_ms = e0.elapsed_time(e1)
+    e2e_ms = max_over_ranks(e2e_ms, dev)
     if world > 1:
         dist.barrier()
 
@@ -468,7 +432,7 @@ def main():
             "dominant_kernel": dominant,
             "e2e": {"value": whole_job_rate(world, e2e_steps, e2e_ms), "unit": UNIT,
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                    "timing": "CUDA events from the first copy-in to the last copy-out; steps pipelined"},
+                    "timing": "CUDA events around the steps; copies and merge in order on one stream"},
             "gpu_launches": int(round(launches_per_step * args.steps)),
             "clocks": clocks.summary(),
         }
