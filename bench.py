@@ -58,6 +58,9 @@ def parse_args():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--e2e-steps", type=int, default=None)
+    p.add_argument("--serve", action="store_true",
+                   help="run the serving sweep (64 requests of 3 Qwen3-4B-shaped fragments with "
+                        "re-deliveries) instead of the single-merge benchmark")
     p.add_argument("--workload", default=WORKLOAD, choices=["q4b", "q4b_t512", "q17_n2", "tiny"],
                    help="single-request workload (q4b is the benchmark; the others are small "
                         "cases for profiling)")
@@ -255,12 +258,91 @@ def whole_job_rate(world: int, steps_per_rank: int, max_elapsed_ms: float) -> fl
     return world * steps_per_rank / (max_elapsed_ms * 1e-3)
 
 
+# ---------------------------------------------------------------- serving sweep
+
+def run_serve(args):
+    """64 independent merge requests on the Qwen3-4B shape: each delivers its 3 fragments
+    (lengths U{512..4096}, each re-sent with probability 0.1, in shuffled order) into a fresh
+    set with one batched ingest, then renders. Every delivery is its own device buffer."""
+    import torch
+    import paper_2607_01308_gb300 as cm
+    import synthetic
+    w = synthetic.WORKLOADS["serve"]
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    reqs = []
+    for r in range(w.num_requests):
+        specs = synthetic.fragment_specs(w, r)
+        frags = [synthetic.make_fragment_torch(sp, w.num_layers, w.num_kv_heads, w.head_dim, dev)
+                 for sp in specs]
+        sched = synthetic.delivery_schedule(w, r)
+        seen, msgs = set(), []
+        for i in sched:
+            K, V = frags[i]
+            msgs.append((K, V) if i not in seen else (K.clone(), V.clone()))
+            seen.add(i)
+        reqs.append(([cm.fragment_from_tensors(K, V) for K, V in msgs], msgs,
+                     sum(sp.seq_len for sp in specs)))
+    cap = max(t for _, _, t in reqs)
+    k_out = torch.empty((w.num_layers, w.num_kv_heads, cap, w.head_dim), dtype=torch.bfloat16,
+                        device=dev)
+    v_out = torch.empty_like(k_out)
+    ctx = cm.Context(0, synthetic.ROPE_THETA)
+    stream = torch.cuda.current_stream(dev)
+
+    def one(req):
+        fd, _, total = req
+        s = cm.cm_set_create(ctx.handle)
+        cm.cm_ingest_batch(s, fd, stream)
+        cm.cm_render(s, k_out.data_ptr(), v_out.data_ptr(), cap, stream)
+        cm.cm_set_destroy(s)
+
+    for req in reqs[:3]:
+        one(req)
+    torch.cuda.synchronize(dev)
+    cm.cm_context_kernel_times(ctx.handle, reset=True)
+    cm.cm_context_set_timing(ctx.handle, True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(0) as clocks:
+        e0.record(stream)
+        for req in reqs:
+            one(req)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+    cm.cm_context_set_timing(ctx.handle, False)
+    kt = cm.cm_context_kernel_times(ctx.handle, reset=True)
+    ms = e0.elapsed_time(e1)
+    render_bytes = sum(2 * t * w.bytes_per_token for _, _, t in reqs)
+    peak, peak_src = hbm_peak()
+    render_gbs = render_bytes / (kt["render_ms"] * 1e-3) / 1e9
+    line = {
+        "mode": "serving sweep", "metric": METRIC, "value": len(reqs) / (ms * 1e-3), "unit": UNIT,
+        "n_gpus": 1, "requests": len(reqs), "higher_is_better": True, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": "serving sweep on the Qwen3-4B shape: 64 requests x 3 fragments, "
+                               "T ~ U{512..4096}, each delivery re-sent with p = 0.1",
+                   "deliveries": sum(len(fd) for fd, _, _ in reqs),
+                   "merged_tokens": sum(t for _, _, t in reqs)},
+        "ms_per_request": ms / len(reqs),
+        "render_gbs": render_gbs, "render_frac_of_measured_hbm": render_gbs / peak,
+        "render_ms_per_request": kt["render_ms"] / len(reqs),
+        "hash_ms_per_request": (kt["leaf_hash_ms"] + kt["inner_hash_ms"]) / len(reqs),
+        "kernel_launches": kt["leaf_hash_launches"] + kt["inner_hash_launches"] + kt["render_launches"],
+        "clocks": clocks.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    ctx.close()
+    return 0
+
+
 # ---------------------------------------------------------------- GPU arm
 
 def main():
     args = parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.serve:
+        return run_serve(args)
 
     import torch
     import torch.distributed as dist
