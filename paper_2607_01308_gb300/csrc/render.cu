@@ -20,10 +20,10 @@
 // fl64(fl64(x c) - fl64(y s)) (and fl64(fl64(y c) + fl64(x s))), c and s the fp64
 // cosine and sine. The fast path computes z in fp32 with one fma from c and s
 // rounded to fp32 and bounds its distance to the fp64 value by
-// E = 2^-22 (|z| + |x| + |y|) + 2^-146. If z - E and z + E (rounded outward) round
-// to the same bf16, every value between them does (rounding is monotone), the fp64
-// value included, and z's rounding is the answer. Otherwise (about one element in
-// a thousand) a second fp32 level with error-free products and a ~2^-36 bound
+// E = (1 + 2^-9) 2^-24 (|z| + |x||c| + 2|y||s|) + 2^-148 (|x| + |y|) + 2^-146 (see
+// err_bound). If z - E and z + E (rounded outward) round to the same bf16, every
+// value between them does (rounding is monotone), the fp64 value included, and z's
+// rounding is the answer. Otherwise (about one element in eight thousand) a second fp32 level with error-free products and a ~2^-36 bound
 // decides, and the few it cannot certify are recomputed in fp64 with the operation
 // sequence of the definition and rounded directly to bf16 (fp64 throughput is very
 // low on this part, so it must stay rare). The output is bit-exact either way.
@@ -68,8 +68,18 @@ __device__ uint32_t f64_to_bf16_bits(double z) {
     return sign | ((uint32_t)e << 7) | (uint32_t)(r & 0x7Fu);
 }
 
-__device__ __forceinline__ float err_bound(float z, float xy_abs) {
-    return __fmaf_ru(__fadd_ru(fabsf(z), xy_abs), 0x1p-22f, 0x1p-146f);
+// First-level error bound. With w = fl(y s32) and z = fl(x c32 - w) (one fma),
+// c32 = fl(c1 + c2) within u|c32| + 2^-40 |c| (+2^-150 if subnormal) of c, u = 2^-24:
+//   |z - (x c - y s)| <= u |z| + u |x||c32| + u |w| + u |y||s32| (+ tiny terms)
+//                     <= (1 + 2^-9) u (|z| + |x||c32| + 2 |y||s32|) + 2^-148 (|x| + |y|) + 2^-146,
+// the last two terms covering roundings in the subnormal range (absolute error 2^-150
+// each) and the fp64 value's own distance to x c - y s (below 2^-52 of the products).
+// `rest` is the shared 2^-148 (|x| + |y|) + 2^-146; p1, p2 are the two operands whose
+// products enter the rounded sum (p1 multiplies c, p2 multiplies s).
+__device__ __forceinline__ float err_bound(float z, float p1, float c, float p2, float s,
+                                           float rest) {
+    const float a = __fmaf_ru(2.0f, __fmul_ru(fabsf(p2), fabsf(s)), __fmul_ru(fabsf(p1), fabsf(c)));
+    return __fmaf_ru(__fadd_ru(a, fabsf(z)), 0x1.008p-24f, rest);
 }
 
 // Rotate the pairs (x0, y0), (x1, y1) held in word xw (x0 low, x1 high) and word yw.
@@ -83,10 +93,10 @@ __device__ __forceinline__ void rotate_word(uint32_t xw, uint32_t yw, float c0, 
     const float zx1 = __fmaf_rn(x1, c1, -__fmul_rn(y1, s1));
     const float zy0 = __fmaf_rn(y0, c0, __fmul_rn(x0, s0));
     const float zy1 = __fmaf_rn(y1, c1, __fmul_rn(x1, s1));
-    const float m0 = __fadd_ru(fabsf(x0), fabsf(y0));
-    const float m1 = __fadd_ru(fabsf(x1), fabsf(y1));
-    const float ex0 = err_bound(zx0, m0), ex1 = err_bound(zx1, m1);
-    const float ey0 = err_bound(zy0, m0), ey1 = err_bound(zy1, m1);
+    const float r0 = __fmaf_ru(__fadd_ru(fabsf(x0), fabsf(y0)), 0x1p-148f, 0x1p-146f);
+    const float r1 = __fmaf_ru(__fadd_ru(fabsf(x1), fabsf(y1)), 0x1p-148f, 0x1p-146f);
+    const float ex0 = err_bound(zx0, x0, c0, y0, s0, r0), ex1 = err_bound(zx1, x1, c1, y1, s1, r1);
+    const float ey0 = err_bound(zy0, y0, c0, x0, s0, r0), ey1 = err_bound(zy1, y1, c1, x1, s1, r1);
     const uint32_t bx = pack_bf16x2(__fsub_rd(zx0, ex0), __fsub_rd(zx1, ex1)) ^
                         pack_bf16x2(__fadd_ru(zx0, ex0), __fadd_ru(zx1, ex1));
     const uint32_t by = pack_bf16x2(__fsub_rd(zy0, ey0), __fsub_rd(zy1, ey1)) ^
