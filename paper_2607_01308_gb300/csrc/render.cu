@@ -23,7 +23,8 @@
 // E = (1 + 2^-9) 2^-24 (|z| + |x||c| + 2|y||s|) + 2^-148 (|x| + |y|) + 2^-146 (see
 // err_bound). If z - E and z + E (rounded outward) round to the same bf16, every
 // value between them does (rounding is monotone), the fp64 value included, and z's
-// rounding is the answer. Otherwise (about one element in eight thousand) a second fp32 level with error-free products and a ~2^-36 bound
+// rounding is the answer. Otherwise (about one element in eight thousand) a second
+// fp32 level with error-free products and a ~2^-36 bound
 // decides, and the few it cannot certify are recomputed in fp64 with the operation
 // sequence of the definition and rounded directly to bf16 (fp64 throughput is very
 // low on this part, so it must stay rare). The output is bit-exact either way.
