@@ -244,62 +244,69 @@ inner_hash_kernel(const uint8_t *__restrict__ children, uint64_t num_children,
     store_digest(out + j * kDigestBytes, h);
 }
 
-// Loads of child digests. kCoherent: the children were written by other threads of
-// the same launch, so they are read through L2 (ld.global.cg) instead of the
-// non-coherent path.
-template <bool kCoherent>
-__device__ __forceinline__ uint4 load_child(const uint8_t *p) {
-    if (kCoherent) return __ldcg(reinterpret_cast<const uint4 *>(p));
-    return load_nc(p);
+// Node j of a tree level over the digests at `children` (num_children of them): its
+// 16 * min(16, num_children - 16 j) bytes, at most four 64-byte blocks, staged in the
+// thread's 256-byte slice of shared memory so that one copy of the compression loop
+// serves every level (the tree top runs few warps per SM; unrolled copies of the
+// compression would not fit the instruction cache).
+__device__ __forceinline__ void hash_node_from(uint4 *stage, uint32_t len, uint8_t *out,
+                                               uint64_t j, uint64_t num_nodes, uint32_t depth,
+                                               const TreeParams &tp) {
+    const uint32_t nblocks = (len + 63) / 64;
+    const bool last_node = j + 1 == num_nodes;
+    uint32_t h[8];
+    node_init(h, tp, j, depth);
+#pragma unroll 1
+    for (uint32_t b = 0; b < nblocks; ++b) {
+        const uint4 w0 = stage[4 * b], w1 = stage[4 * b + 1], w2 = stage[4 * b + 2],
+                    w3 = stage[4 * b + 3];
+        const uint32_t m[16] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w,
+                                w2.x, w2.y, w2.z, w2.w, w3.x, w3.y, w3.z, w3.w};
+        const uint32_t end = (b + 1) * 64 < len ? (b + 1) * 64 : len;
+        compress(h, m, end, b + 1 == nblocks, last_node);
+    }
+    store_digest(out + j * kDigestBytes, h);
 }
 
-// Node j of a tree level over the digests at `children` (num_children of them):
-// its 16 * min(16, num_children - 16 j) bytes, at most four 64-byte blocks.
-template <bool kCoherent = false>
-__device__ __forceinline__ void hash_inner_node(const uint8_t *children, uint64_t num_children,
-                                                uint8_t *out, uint64_t j, uint64_t num_nodes,
-                                                uint32_t depth, const TreeParams &tp) {
-    // a node's input is at most 16 digests = 256 bytes: all of it is loaded at once
+// Loads node j's children (zero-padded to 256 bytes) into `stage`; returns their length.
+// kCoherent: the children were written by other threads of the same launch, so they
+// are read through L2 (ld.global.cg) instead of the non-coherent path.
+template <bool kCoherent>
+__device__ __forceinline__ uint32_t stage_children(uint4 *stage, const uint8_t *children,
+                                                   uint64_t num_children, uint64_t j) {
     static_assert(kFanout * kDigestBytes <= 256, "an inner node must fit four blocks");
     const uint64_t first = j * kFanout;
     const uint64_t nc64 = num_children - first;
     const uint32_t nc = nc64 < (uint64_t)kFanout ? (uint32_t)nc64 : (uint32_t)kFanout;
     const uint32_t len = nc * kDigestBytes;
-    const uint32_t nblocks = (len + 63) / 64;
-    const bool last_node = j + 1 == num_nodes;
-    const uint8_t *src = children + first * kDigestBytes;
-    uint32_t h[8];
-    node_init(h, tp, j, depth);
+    const uint4 *src = reinterpret_cast<const uint4 *>(children + first * kDigestBytes);
     uint4 w[16];
 #pragma unroll
-    for (int q = 0; q < 16; ++q)
-        w[q] = (uint32_t)(q * 16) < len ? load_child<kCoherent>(src + q * 16) : make_uint4(0, 0, 0, 0);
-#pragma unroll
-    for (uint32_t b = 0; b < 4; ++b) {
-        if (b < nblocks) {
-            const uint32_t m[16] = {w[4 * b].x,     w[4 * b].y,     w[4 * b].z,     w[4 * b].w,
-                                    w[4 * b + 1].x, w[4 * b + 1].y, w[4 * b + 1].z, w[4 * b + 1].w,
-                                    w[4 * b + 2].x, w[4 * b + 2].y, w[4 * b + 2].z, w[4 * b + 2].w,
-                                    w[4 * b + 3].x, w[4 * b + 3].y, w[4 * b + 3].z, w[4 * b + 3].w};
-            const uint32_t end = (b + 1) * 64 < len ? (b + 1) * 64 : len;
-            compress(h, m, end, b + 1 == nblocks, last_node);
-        }
+    for (int q = 0; q < 16; ++q) {
+        const bool in = (uint32_t)(q * 16) < len;
+        w[q] = in ? (kCoherent ? __ldcg(src + q) : __ldg(src + q)) : make_uint4(0, 0, 0, 0);
     }
-    store_digest(out + j * kDigestBytes, h);
+#pragma unroll
+    for (int q = 0; q < 16; ++q) stage[q] = w[q];
+    return len;
 }
 
 __global__ void __launch_bounds__(kInnerThreads)
 tree_top_kernel(const __grid_constant__ TreeTop t) {
+    __shared__ uint4 stage_all[kInnerThreads][16];
+    uint4 *stage = stage_all[threadIdx.x];
     const uint64_t g = (uint64_t)blockIdx.x * kInnerThreads + threadIdx.x;
     if (g >= t.node_begin[t.count]) return;
     uint32_t fi = 0;
     while (fi + 1 < t.count && g >= t.node_begin[fi + 1]) ++fi;
     const TreeTopFragment &f = t.frag[fi];
     uint64_t j = g - t.node_begin[fi];
-    hash_inner_node<false>(f.level[0], f.size[0], f.level[1], j, f.size[1], 1, f.tree);
-    for (uint32_t k = 1; k + 1 < f.levels; ++k) {
-        // this thread finished node j of level k; the one that finishes the last
-        // child of parent j / 16 hashes the parent
+    uint32_t len = stage_children<false>(stage, f.level[0], f.size[0], j);
+    for (uint32_t k = 1;; ++k) {
+        hash_node_from(stage, len, f.level[k], j, f.size[k], k, f.tree);
+        if (k + 1 >= f.levels) break;
+        // this thread finished node j of level k; the one that finishes the last child of
+        // parent j / 16 hashes the parent
         const uint64_t parent = j / kFanout;
         const uint64_t first = parent * kFanout;
         const uint64_t left = f.size[k] - first;
@@ -308,9 +315,8 @@ tree_top_kernel(const __grid_constant__ TreeTop t) {
         const uint32_t done = atomicAdd(f.arrivals[k + 1] + parent, 1u) + 1;
         if (done != siblings) return;
         __threadfence();                                  // see every sibling's digest
-        hash_inner_node<true>(f.level[k], f.size[k], f.level[k + 1], parent, f.size[k + 1], k + 1,
-                              f.tree);
         j = parent;
+        len = stage_children<true>(stage, f.level[k], f.size[k], j);
     }
 }
 
