@@ -23,12 +23,19 @@
 #include <vector>
 
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include "cm_kernels.h"
 
 namespace {
 
 thread_local std::string g_last_error;
+
+// NVTX range for the duration of a call (the library's phases in a profiler timeline).
+struct TraceRange {
+    explicit TraceRange(const char *name) { nvtxRangePushA(name); }
+    ~TraceRange() { nvtxRangePop(); }
+};
 
 cm_status fail(cm_status st, const std::string &msg) {
     g_last_error = msg;
@@ -630,6 +637,7 @@ cm_status cm_set_destroy(cm_set *set) {
 
 cm_status cm_fragment_id(cm_context *ctx, const cm_fragment *frag, cm_stream_t stream,
                          cm_id *out_id, uint64_t *out_norm_key) {
+    TraceRange trace("cm_fragment_id");
     return guarded([&]() -> cm_status {
         if (!ctx) return fail(CM_ERR_INVALID_ARG, "context is NULL");
         if (!out_id) return fail(CM_ERR_INVALID_ARG, "out_id is NULL");
@@ -656,6 +664,7 @@ cm_status cm_ingest(cm_set *set, const cm_fragment *frag, cm_stream_t stream, cm
 
 cm_status cm_ingest_batch(cm_set *set, const cm_fragment *frags, int32_t n, cm_stream_t stream,
                           cm_id *out_ids, int32_t *out_absorbed) {
+    TraceRange trace("cm_ingest");
     return guarded([&]() -> cm_status {
         if (!set) return fail(CM_ERR_INVALID_ARG, "set is NULL");
         if (n < 0 || (n > 0 && !frags)) return fail(CM_ERR_INVALID_ARG, "need n >= 0 fragments");
@@ -771,6 +780,7 @@ cm_status cm_context_kernel_times(cm_context *ctx, cm_kernel_times *out, int32_t
 }
 
 cm_status cm_union(cm_set *dst, const cm_set *src) {
+    TraceRange trace("cm_union");
     return guarded([&]() -> cm_status {
         if (!dst || !src) return fail(CM_ERR_INVALID_ARG, "set is NULL");
         if (dst == src) return CM_OK;
@@ -822,6 +832,7 @@ cm_status render_set(const cm_set *set, void *k_out, void *v_out, int64_t capaci
                      uint32_t withhold_warp, const cm_id *prev_order = nullptr,
                      int64_t prev_n = 0, int64_t *out_reused_tokens = nullptr,
                      const cm_paged_cache *paged = nullptr) {
+    TraceRange trace("cm_render");
     return guarded([&]() -> cm_status {
         if (!set) return fail(CM_ERR_INVALID_ARG, "set is NULL");
         if (capacity_tokens < 0) return fail(CM_ERR_INVALID_ARG, "capacity_tokens < 0");
@@ -916,6 +927,7 @@ cm_status cm_context_check(cm_context *ctx, cm_stream_t stream) {
 cm_status cm_bagmerge(cm_context *ctx, const cm_fragment *frags, int32_t n, void *k_out,
                       void *v_out, int64_t capacity_tokens, cm_stream_t stream,
                       int64_t *out_seq_len) {
+    TraceRange trace("cm_bagmerge");
     return guarded([&]() -> cm_status {
         if (!ctx) return fail(CM_ERR_INVALID_ARG, "context is NULL");
         if (!frags || n < 1) return fail(CM_ERR_INVALID_ARG, "need n >= 1 fragments");

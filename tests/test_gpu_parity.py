@@ -351,3 +351,36 @@ def test_long_fragment_and_large_offsets(ctx):
     assert np.array_equal(synthetic.to_bits(v_out), V_ref)
     assert assert_k_parity(synthetic.to_bits(k_out), K_ref) == 0
     S.close()
+
+
+# ---------------------------------------------------------------- rotation stress
+
+@pytest.mark.parametrize("theta", [1.0e4, 1.0e6, 5.0e5, 1.0e40])
+def test_rotation_stress_random_bit_patterns(theta):
+    # every finite bf16 bit pattern is a possible key; many slots give many (cos, sin)
+    # pairs, including tiny sines when theta is huge
+    c = cm.Context(0, theta)
+    L, H, d = 1, 2, 128
+    rng = np.random.default_rng(int(theta) % 1000 + 1)
+    frags, bits_list = [], []
+    for i in range(12):
+        T = int(rng.integers(1, 90))
+        bits = rng.integers(0, 1 << 16, size=(L, H, T, d), dtype=np.uint64).astype(np.uint16)
+        bits[((bits & 0x7F80) == 0x7F80)] &= 0xBF7F          # no inf / NaN
+        K = torch.from_numpy(bits.view(np.int16)).to("cuda:0").view(torch.bfloat16)
+        V = torch.from_numpy(rng.integers(0, 1 << 15, size=bits.shape).astype(np.int16)).to(
+            "cuda:0").view(torch.bfloat16)
+        frags.append((K.contiguous(), V.contiguous()))
+        bits_list.append(bits)
+    total = sum(f[0].shape[2] for f in frags)
+    k_out, v_out = empty_out(L, H, total, d)
+    n = c.bagmerge(frags, k_out, v_out)
+    torch.cuda.synchronize()
+    kb = synthetic.to_bits(k_out)
+    s = 0
+    for bits in bits_list:
+        T = bits.shape[2]
+        want = oracle.rotate_k(bits, s, theta)
+        assert assert_k_parity(kb[:, :, s:s + T], want, f"slot@{s}") == 0
+        s += T
+    c.close()
