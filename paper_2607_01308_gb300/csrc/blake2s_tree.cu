@@ -193,6 +193,21 @@ leaf_hash_kernel(const __grid_constant__ LeafLaunch a) {
     StreamCursor cur = cursor_at(a, begin);
     NormState ns{0.0};
 
+    if (!norm_leaf && len == (uint32_t)kLeafBytes && cur.left >= (uint64_t)kLeafBytes) {
+        // the whole leaf lies in one K or V segment, away from the routing layer
+        const uint8_t *p = cur.ptr;
+#pragma unroll 1
+        for (uint32_t b = 0; b < 16; ++b) {
+            const uint4 w0 = load_nc(p + 64 * b), w1 = load_nc(p + 64 * b + 16),
+                        w2 = load_nc(p + 64 * b + 32), w3 = load_nc(p + 64 * b + 48);
+            const uint32_t m[16] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w,
+                                    w2.x, w2.y, w2.z, w2.w, w3.x, w3.y, w3.z, w3.w};
+            compress(h, m, (b + 1) * 64, b == 15, last_node);
+        }
+        store_digest(a.digests + leaf * kDigestBytes, h);
+        return;
+    }
+
     for (uint32_t b = 0; b < nblocks; ++b) {
         uint4 w[4];
 #pragma unroll
