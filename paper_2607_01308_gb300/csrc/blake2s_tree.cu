@@ -306,6 +306,12 @@ __device__ __forceinline__ uint32_t stage_children(uint4 *stage, const uint8_t *
     return len;
 }
 
+__device__ __forceinline__ uint32_t arrive_acq_rel(uint32_t *counter) {
+    uint32_t old;
+    asm volatile("atom.add.acq_rel.gpu.u32 %0, [%1], 1;" : "=r"(old) : "l"(counter) : "memory");
+    return old;
+}
+
 __global__ void __launch_bounds__(kInnerThreads)
 tree_top_kernel(const __grid_constant__ TreeTop t) {
     __shared__ uint4 stage_all[kInnerThreads][16];
@@ -326,10 +332,10 @@ tree_top_kernel(const __grid_constant__ TreeTop t) {
         const uint64_t first = parent * kFanout;
         const uint64_t left = f.size[k] - first;
         const uint32_t siblings = left < (uint64_t)kFanout ? (uint32_t)left : (uint32_t)kFanout;
-        __threadfence();                                  // publish this node's digest
-        const uint32_t done = atomicAdd(f.arrivals[k + 1] + parent, 1u) + 1;
+        // one acquire-release add: it publishes this node's digest and, for the thread
+        // that counts the last sibling, makes every sibling's digest visible
+        const uint32_t done = arrive_acq_rel(f.arrivals[k + 1] + parent) + 1;
         if (done != siblings) return;
-        __threadfence();                                  // see every sibling's digest
         j = parent;
         len = stage_children<true>(stage, f.level[k], f.size[k], j);
     }

@@ -384,3 +384,44 @@ def test_rotation_stress_random_bit_patterns(theta):
         assert assert_k_parity(kb[:, :, s:s + T], want, f"slot@{s}") == 0
         s += T
     c.close()
+
+
+# ---------------------------------------------------------------- concurrent use of one context
+
+def test_two_threads_share_a_context(ctx):
+    import threading
+    results, errors = {}, []
+
+    def worker(name, seed):
+        try:
+            stream = torch.cuda.Stream()
+            with torch.cuda.stream(stream):
+                frags = [((torch.randn((3, 2, T, 64), device="cuda:0") * (0.5 + 0.2 * i)).to(torch.bfloat16),
+                          torch.randn((3, 2, T, 64), device="cuda:0").to(torch.bfloat16))
+                         for i, T in enumerate([40 + seed, 77, 12 + seed])]
+                outs = []
+                for rep in range(5):
+                    S = cm.FragmentSet(ctx)
+                    S.ingest_batch(frags, stream)
+                    k, v = empty_out(3, 2, S.seq_len(), 64)
+                    S.render(k, v, stream)
+                    stream.synchronize()
+                    outs.append((synthetic.to_bits(k), synthetic.to_bits(v), S.ids()))
+                    S.close()
+            results[name] = (frags, outs)
+        except Exception as e:     # surfaced below
+            errors.append(e)
+
+    threads = [threading.Thread(target=worker, args=(f"t{i}", i)) for i in range(2)]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    assert not errors, errors
+    for name, (frags, outs) in results.items():
+        ref = oracle.from_deliveries([oracle_fragment(K, V) for K, V in frags])
+        K_ref, V_ref, _ = oracle.render(ref, THETA)
+        for kb, vb, ids in outs:
+            assert ids == ref.ids()
+            assert np.array_equal(vb, V_ref)
+            assert assert_k_parity(kb, K_ref) == 0
