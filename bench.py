@@ -420,6 +420,33 @@ def main():
     ingest_ms = sum(t["ingest"][0].elapsed_time(t["ingest"][1]) for t in step_timers) / args.steps
     elapsed_ms = max_over_ranks(elapsed_ms, dev)
 
+    # paged render of the same merge into per-layer block pools [L][blocks][16][H][d] through a
+    # shuffled block table (timed apart from the steps, same algorithmic bytes)
+    paged_ms = None
+    if args.workload == WORKLOAD:
+        import numpy as np
+        bs = 16
+        nblk = -(-total_T // bs)
+        pool_k = torch.empty((L, nblk, bs, H, d), dtype=torch.bfloat16, device=dev)
+        pool_v = torch.empty_like(pool_k)
+        table = torch.from_numpy(np.random.default_rng(0).permutation(nblk).astype(np.int32)).to(dev)
+        cache = cm.cm_paged_cache(pool_k.data_ptr(), pool_v.data_ptr(), table.data_ptr(), nblk, bs,
+                                  stride_block=bs * H * d, stride_layer=nblk * bs * H * d,
+                                  stride_head=d, stride_token=H * d)
+        ps = cm.cm_set_create(ctx.handle)
+        cm.cm_ingest_batch(ps, fdesc, stream)
+        for _ in range(3):
+            cm.cm_render_paged(ps, cache, stream)
+        pe = [(ev(), ev()) for _ in range(10)]
+        for a_, b_ in pe:
+            a_.record(stream)
+            cm.cm_render_paged(ps, cache, stream)
+            b_.record(stream)
+        torch.cuda.synchronize(dev)
+        paged_ms = sum(a_.elapsed_time(b_) for a_, b_ in pe) / len(pe)
+        cm.cm_set_destroy(ps)
+        del pool_k, pool_v
+
     # end to end through the C ABI with host buffers: pinned inputs copied in and the
     # merged cache copied out inside the timed region, every step
     e2e_steps = args.e2e_steps or min(args.steps, 10)
@@ -505,6 +532,7 @@ def main():
             "render_frac_of_measured_hbm": render_gbs / peak,
             "render_frac_of_8tbs": render_gbs / NOMINAL_HBM_GBS,
             "render_ms": render_ms,
+            "paged_render_gbs": (render_bytes / (paged_ms * 1e-3) / 1e9) if paged_ms else None,
             "ingest_ms_per_merge": ingest_ms,
             "ingest_gbs": hash_bytes / (ingest_ms * 1e-3) / 1e9,
             "roofline": hash_roof if dominant != "render" else render_roof,
