@@ -470,6 +470,9 @@ cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t 
             p->paged = 1;
             p->block_table = paged->block_table;
             p->block_size = paged->block_size;
+            p->log2_block_size = is_pow2(paged->block_size)
+                                     ? (int32_t)__builtin_ctzll((unsigned long long)paged->block_size)
+                                     : -1;
             p->stride_block = paged->stride_block;
             p->stride_layer = paged->stride_layer;
             p->stride_head = paged->stride_head;

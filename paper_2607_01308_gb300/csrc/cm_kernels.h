@@ -114,6 +114,8 @@ struct RenderParams {
     // (element strides, head_dim contiguous); k_out / v_out are the pools
     const int32_t *block_table; // device
     int64_t block_size;
+    int32_t log2_block_size;    // >= 0 when block_size is a power of two, else -1
+    int32_t pad3_;
     int64_t stride_block, stride_layer, stride_head, stride_token;
     RenderSlot slot[kMaxSlots];
     double cs[2 * kMaxTablePairs];   // (cos a, sin a) of a = s * theta^(-2j/d), interleaved

@@ -289,9 +289,20 @@ template <bool kPaged>
 __device__ __forceinline__ uint4 *row_dst(const RenderParams &p, const Item &it, int r) {
     if (!kPaged) return reinterpret_cast<uint4 *>(it.dst) + (int64_t)r * (p.head_dim >> 3);
     const int64_t pos = it.pos0 + r;
-    const int64_t blk = __ldg(p.block_table + pos / p.block_size);
-    return reinterpret_cast<uint4 *>(it.dst +
-                                     (blk * p.stride_block + (pos % p.block_size) * p.stride_token) * 2);
+    int64_t b, o;
+    if (p.log2_block_size >= 0) {                       // the usual case: shifts
+        b = pos >> p.log2_block_size;
+        o = pos & ((1ll << p.log2_block_size) - 1);
+    } else if (pos < 0x80000000ll && p.block_size < 0x80000000ll) {   // 32-bit division
+        const uint32_t q = (uint32_t)pos / (uint32_t)p.block_size;
+        b = q;
+        o = pos - (int64_t)q * p.block_size;
+    } else {
+        b = pos / p.block_size;
+        o = pos - b * p.block_size;
+    }
+    const int64_t blk = __ldg(p.block_table + b);
+    return reinterpret_cast<uint4 *>(it.dst + (blk * p.stride_block + o * p.stride_token) * 2);
 }
 
 // Byte copy of one staged item: shared memory -> registers -> 16-byte streaming stores.
