@@ -137,6 +137,9 @@ struct cm_context {
     std::vector<cudaEvent_t> event_pool;
     double time_ms[3] = {0, 0, 0};
     int64_t launches[3] = {0, 0, 0};
+    // RoPE frequencies theta^(-2j/d), j < d/2, for the last head_dim rendered
+    std::vector<double> omega;
+    int32_t omega_d = 0;
 };
 
 struct cm_set {
@@ -279,6 +282,14 @@ cm_status fragments_digest(cm_context *ctx, const cm_fragment *const *frags, siz
         l.tp = tree_params(f->num_layers, f->num_kv_heads, f->head_dim, f->seq_len);
     }
     const size_t host_bytes = off;     // roots and norm keys, copied back in one piece
+    // arrival counters of every node at levels >= 2 follow the norm keys, so that one
+    // memset zeroes both before the launches
+    std::vector<size_t> arr_off(n);
+    for (size_t i = 0; i < n; ++i) {
+        arr_off[i] = off;
+        for (size_t k = 2; k < lay[i].sizes.size(); ++k) off += (size_t)lay[i].sizes[k] * 4;
+    }
+    const size_t zero_end = off;
     off = (off + 255) & ~(size_t)255;
     for (size_t i = 0; i < n; ++i) {
         Layout &l = lay[i];
@@ -289,23 +300,12 @@ cm_status fragments_digest(cm_context *ctx, const cm_fragment *const *frags, siz
             off += ((size_t)l.sizes[k] * cm::kDigestBytes + 255) & ~(size_t)255;
         }
     }
-    // arrival counters of every node at levels >= 2, zeroed before the tree-top launch
-    const size_t arrivals_off = off;
-    std::vector<size_t> arr_off(n);
-    for (size_t i = 0; i < n; ++i) {
-        arr_off[i] = off;
-        for (size_t k = 2; k < lay[i].sizes.size(); ++k) off += (size_t)lay[i].sizes[k] * 4;
-    }
-    const size_t arrivals_bytes = off - arrivals_off;
     cm_status st = ensure_scratch(ctx, off, host_bytes);
     if (st != CM_OK) return st;
     uint8_t *base = ctx->d_scratch;
 
-    CM_CUDA_TRY(cudaMemsetAsync(base + roots_bytes, 0, host_bytes - roots_bytes, stream),
-                "zeroing the norm keys");
-    if (arrivals_bytes)
-        CM_CUDA_TRY(cudaMemsetAsync(base + arrivals_off, 0, arrivals_bytes, stream),
-                    "zeroing the arrival counters");
+    CM_CUDA_TRY(cudaMemsetAsync(base + roots_bytes, 0, zero_end - roots_bytes, stream),
+                "zeroing the norm keys and arrival counters");
     for (size_t i = 0; i < n; ++i) {
         const cm_fragment *f = frags[i];
         const Layout &l = lay[i];
@@ -426,6 +426,11 @@ cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t 
     const uint64_t planes = 2ull * L * H;
     int log2_pairs = 0;
     while ((1 << log2_pairs) < d / 16) ++log2_pairs;
+    if (ctx->omega_d != d) {
+        ctx->omega.resize((size_t)half);
+        for (int j = 0; j < half; ++j) ctx->omega[(size_t)j] = std::pow(ctx->theta, -(2.0 * j) / d);
+        ctx->omega_d = d;
+    }
     std::unique_ptr<cm::RenderParams> p(new cm::RenderParams);
     for (size_t g0 = 0; g0 < slots.size(); g0 += (size_t)max_group) {
         const size_t n = std::min(slots.size() - g0, (size_t)max_group);
@@ -453,12 +458,14 @@ cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t 
             rs.chunk_begin = (uint32_t)chunk;
             rs.chunks_per_plane = (uint32_t)cpp;
             chunk += cpp * planes;
-            // delta angle a_j = s * theta^(-2j/d) in fp64 (Section 2.3 / Eq. bagmerge-k)
-            for (int j = 0; j < half; ++j) {
-                const double w = std::pow(ctx->theta, -(2.0 * j) / d);
-                const double a = (double)s.offset * w;
-                p->cs[2 * (i * half + j)] = std::cos(a);
-                p->cs[2 * (i * half + j) + 1] = std::sin(a);
+            // delta angle a_j = s * theta^(-2j/d) in fp64 (Section 2.3 / Eq. bagmerge-k);
+            // the slot at offset 0 is copied and needs no table
+            if (rs.rotate) {
+                for (int j = 0; j < half; ++j) {
+                    const double a = (double)s.offset * ctx->omega[(size_t)j];
+                    p->cs[2 * (i * half + j)] = std::cos(a);
+                    p->cs[2 * (i * half + j) + 1] = std::sin(a);
+                }
             }
         }
         if (chunk > 0xFFFFFFFFull)
