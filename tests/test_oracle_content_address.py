@@ -116,3 +116,20 @@ def test_id_sensitive_to_every_byte_and_to_shape():
 def test_id_as_int_is_big_endian():
     assert ca.id_as_int(bytes([1] + [0] * 15)) == 1 << 120
     assert ca.id_as_int(bytes([0] * 15 + [1])) == 1
+
+
+def test_salt_and_personalisation_byte_layout():
+    # salt = (L, H, d, dtype code 1 = bf16) as four little-endian uint16; person = T as a
+    # little-endian uint64 (the documented parameter layout of every tree node)
+    assert ca.tree_salt(28, 8, 128) == bytes([28, 0, 8, 0, 128, 0, 1, 0])
+    assert ca.tree_salt(300, 2, 64) == bytes([0x2C, 0x01, 2, 0, 64, 0, 1, 0])
+    assert ca.tree_person(4096) == bytes([0, 0x10, 0, 0, 0, 0, 0, 0])
+    assert ca.tree_person((1 << 40) + 3) == bytes([3, 0, 0, 0, 0, 1, 0, 0])
+    # and the parameter block the nodes are hashed with carries them at bytes 16..31
+    pb = ref.param_block(16, fanout=ca.FANOUT, depth=ca.DEPTH, leaf_size=ca.LEAF_SIZE,
+                         node_offset=5, node_depth=2, inner_size=16,
+                         salt=ca.tree_salt(28, 8, 128), person=ca.tree_person(4096))
+    assert pb[0:4] == bytes([16, 0, 16, 255]) and pb[4:8] == (1024).to_bytes(4, "little")
+    assert pb[8:14] == (5).to_bytes(6, "little") and pb[14:16] == bytes([2, 16])
+    assert pb[16:24] == bytes([28, 0, 8, 0, 128, 0, 1, 0])
+    assert pb[24:32] == bytes([0, 0x10, 0, 0, 0, 0, 0, 0])
