@@ -10,11 +10,11 @@
 // turned by one constant angle a_j = s * theta^(-2j/d) per frequency j (the delta
 // formula of Section 2.3), pairing element j with element j + d/2.
 //
-// Work item: up to 32 KiB of one source plane. A persistent grid of one CTA per SM
-// walks the items; 1-D TMA bulk copies stage them through shared memory (see
-// render_kernel). For a rotated K item a thread takes vector v of a row's first
-// half and vector v of its second half: 8 (x, y) pairs that share the thread's
-// 8 (cos, sin) values for the whole item.
+// Work item: up to 4 KiB of rows of one source plane. A persistent grid of one CTA
+// per SM walks the items, every warp with its own pipeline of 1-D TMA bulk copies
+// through shared memory (see render_kernel). For a rotated K item a lane takes
+// vector v of a row's first half and vector v of its second half: 8 (x, y) pairs
+// that share the lane's 8 (cos, sin) values for the whole item.
 //
 // Rounding. The result must equal round-to-nearest-even-bf16 of
 // fl64(fl64(x c) - fl64(y s)) (and fl64(fl64(y c) + fl64(x s))), c and s the fp64
@@ -24,10 +24,10 @@
 // err_bound). If z - E and z + E (rounded outward) round to the same bf16, every
 // value between them does (rounding is monotone), the fp64 value included, and z's
 // rounding is the answer. Otherwise (about one element in eight thousand) a second
-// fp32 level with error-free products and a ~2^-36 bound
-// decides, and the few it cannot certify are recomputed in fp64 with the operation
-// sequence of the definition and rounded directly to bf16 (fp64 throughput is very
-// low on this part, so it must stay rare). The output is bit-exact either way.
+// fp32 level with error-free products and a ~2^-36 bound decides, and the few it
+// cannot certify are recomputed in fp64 with the operation sequence of the
+// definition and rounded directly to bf16 (fp64 throughput is very low on this part,
+// so it must stay rare). The output is bit-exact either way.
 #include "cm_kernels.h"
 
 namespace cm {
@@ -381,12 +381,13 @@ __device__ __forceinline__ float2 split16(double c) {
 // pipeline over its own items, with no block-wide barrier after set-up. Items come
 // in (K, V) pairs of the same (slot, layer, head, row chunk); a warp takes pairs
 // warp id + m * total warps and does the K item, then the V item, so rotation work
-// and pure copies alternate within every warp. Lane 0 keeps up to kStages items in flight as
-// 1-D TMA bulk loads into the warp's stages (completion on one mbarrier per
-// stage); all lanes wait for an item, move it from shared memory to its place in
-// the output (rotating K rows of slots at a nonzero offset), and lane 0 refills the
-// stage with the warp's next item. Every wait is bounded: on timeout the warp
-// records an error, waits (bounded) for its own copies in flight and returns.
+// and pure copies alternate within every warp. Lane 0 keeps up to kStages items in
+// flight as 1-D TMA bulk loads into the warp's stages (completion on one mbarrier
+// per stage); all lanes wait for an item, move it from shared memory to its place
+// in the output (rotating K rows of slots at a nonzero offset; kPaged: each row's
+// place comes from the block table), and lane 0 refills the stage with the warp's
+// next item. Every wait is bounded: on timeout the warp records an error, waits
+// (bounded) for its own copies in flight and returns.
 template <bool kPaged>
 __global__ void __launch_bounds__(kThreads, 1)
 render_kernel(const __grid_constant__ RenderParams p) {
