@@ -142,17 +142,28 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
+def kernel_source_digest(source: str) -> str:
+    """sha256 of a kernel's source file and the shared kernel header, with comments and
+    whitespace removed (comment edits do not change the kernel)."""
+    csrc = os.path.join(ROOT, "paper_2607_01308_gb300", "csrc")
+    text = ""
+    for name in (source, "cm_kernels.h"):
+        t = open(os.path.join(csrc, name)).read()
+        t = re.sub(r"/\*.*?\*/", "", t, flags=re.S)
+        t = re.sub(r"//[^\n]*", "", t)
+        text += re.sub(r"\s+", "", t)
+    return hashlib.sha256(text.encode()).hexdigest()
+
+
 def profile_traffic(source: str, summary: str):
-    """DRAM bytes per full launch from a committed ncu summary, if that summary was taken
-    on the current kernel source (the source's sha256 is recorded in it); else None."""
-    src = os.path.join(ROOT, "paper_2607_01308_gb300", "csrc", source)
+    """DRAM bytes per full launch from a committed ncu summary, if that summary was taken on
+    the current kernel code (its kernel source digest is recorded in it); else None."""
     summ = os.path.join(ROOT, "profiles", summary)
     try:
-        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()
         text = open(summ).read()
-        m_sha = re.search(re.escape(source) + r" sha256:\s*([0-9a-f]{64})", text)
+        m_sha = re.search(r"kernel source digest:\s*([0-9a-f]{64})", text)
         m_tr = re.search(r"dram_bytes_per_full_launch:\s*([0-9.eE+]+)", text)
-        if m_sha and m_tr and m_sha.group(1) == sha:
+        if m_sha and m_tr and m_sha.group(1) == kernel_source_digest(source):
             return float(m_tr.group(1))
     except OSError:
         pass
