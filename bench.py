@@ -207,7 +207,7 @@ def oracle_sample_seconds(layers=1, w=None):
     return dt, nbytes
 
 
-def cpu_baseline_entry(layers=2):
+def cpu_baseline_entry(layers=24):
     import synthetic
     w = synthetic.WORKLOADS[WORKLOAD]
     dt, _ = oracle_sample_seconds(layers, w)
