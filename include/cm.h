@@ -193,7 +193,8 @@ cm_status cm_set_ids(const cm_set *set, cm_id *out, int64_t capacity);
  *   out_order        nullable HOST array of set-size ids: the canonical order
  * The output bytes are a pure function of the set: identical for every delivery
  * order and re-delivery. An empty set renders to length 0 and launches nothing
- * (k_out and v_out may then be NULL). */
+ * (k_out and v_out may then be NULL). k_out and v_out must not overlap each other
+ * or any fragment of the set (the render reads the fragments while it writes). */
 cm_status cm_render(const cm_set *set, void *k_out, void *v_out, int64_t capacity_tokens,
                     cm_stream_t stream, int64_t *out_seq_len, cm_id *out_order);
 
