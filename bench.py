@@ -2,8 +2,9 @@
 
 One step = one whole merge of the Qwen3-4B-shaped workload (36 layers, 8 KV
 heads, head_dim 128, RoPE theta 1e6, 4 fragments x 4096 tokens, bf16):
-  replica A ingests fragments 0 and 1, replica B ingests fragments 2 and 3
-  (content address + routing-layer norm key on the GPU, membership on the host),
+  replica A ingests fragments 0 and 1, replica B ingests fragments 2 and 3 in one
+  cm_ingest_many call (content address + routing-layer norm key on the GPU in one
+  pass over the four fragments, membership on the host),
   A := A u B (set union), then A is rendered (canonical order on the host, one
   fused copy-and-rotate kernel) into a preallocated [36, 8, 16384, 128] K/V cache.
 
@@ -61,6 +62,8 @@ def parse_args():
     p.add_argument("--serve", action="store_true",
                    help="run the serving sweep (64 requests of 3 Qwen3-4B-shaped fragments with "
                         "re-deliveries) instead of the single-merge benchmark")
+    p.add_argument("--group", type=int, default=8,
+                   help="serving sweep: requests per cm_ingest_many / cm_render_many call")
     p.add_argument("--workload", default=WORKLOAD, choices=["q4b", "q4b_t512", "q17_n2", "tiny"],
                    help="single-request workload (q4b is the benchmark; the others are small "
                         "cases for profiling)")
@@ -274,7 +277,10 @@ def whole_job_rate(world: int, steps_per_rank: int, max_elapsed_ms: float) -> fl
 def run_serve(args):
     """64 independent merge requests on the Qwen3-4B shape: each delivers its 3 fragments
     (lengths U{512..4096}, each re-sent with probability 0.1, in shuffled order) into a fresh
-    set with one batched ingest, then renders. Every delivery is its own device buffer."""
+    set, which is then rendered. Every delivery is its own device buffer. Timed twice: one
+    request at a time (a batched ingest and a render per request), and `--group` requests at
+    a time (one cm_ingest_many and one cm_render_many per group, each request rendering into
+    its own output buffer)."""
     import torch
     import paper_2607_01308_gb300 as cm
     import synthetic
@@ -295,51 +301,84 @@ def run_serve(args):
         reqs.append(([cm.fragment_from_tensors(K, V) for K, V in msgs], msgs,
                      sum(sp.seq_len for sp in specs)))
     cap = max(t for _, _, t in reqs)
-    k_out = torch.empty((w.num_layers, w.num_kv_heads, cap, w.head_dim), dtype=torch.bfloat16,
-                        device=dev)
-    v_out = torch.empty_like(k_out)
+    G = max(1, args.group)
+    outs = []
+    for _ in range(G):
+        k_out = torch.empty((w.num_layers, w.num_kv_heads, cap, w.head_dim), dtype=torch.bfloat16,
+                            device=dev)
+        outs.append((k_out, torch.empty_like(k_out)))
     ctx = cm.Context(0, synthetic.ROPE_THETA)
     stream = torch.cuda.current_stream(dev)
 
     def one(req):
-        fd, _, total = req
+        fd, _, _ = req
         s = cm.cm_set_create(ctx.handle)
         cm.cm_ingest_batch(s, fd, stream)
-        cm.cm_render(s, k_out.data_ptr(), v_out.data_ptr(), cap, stream)
+        cm.cm_render(s, outs[0][0].data_ptr(), outs[0][1].data_ptr(), cap, stream)
         cm.cm_set_destroy(s)
 
-    for req in reqs[:3]:
-        one(req)
-    torch.cuda.synchronize(dev)
-    cm.cm_context_kernel_times(ctx.handle, reset=True)
-    cm.cm_context_set_timing(ctx.handle, True)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with ClockSampler(0) as clocks:
-        e0.record(stream)
-        for req in reqs:
-            one(req)
-        e1.record(stream)
+    def grouped(group):
+        sets = [cm.cm_set_create(ctx.handle) for _ in group]
+        owners, fds = [], []
+        for s, (fd, _, _) in zip(sets, group):
+            owners += [s] * len(fd)
+            fds += fd
+        cm.cm_ingest_many(owners, fds, stream)
+        cm.cm_render_many([cm.cm_render_job(s, k.data_ptr(), v.data_ptr(), cap)
+                           for s, (k, v) in zip(sets, outs)], stream)
+        for s in sets:
+            cm.cm_set_destroy(s)
+
+    def timed(run_all):
+        run_all(reqs)                           # warm-up: grows the scratch to its steady size
         torch.cuda.synchronize(dev)
-    cm.cm_context_set_timing(ctx.handle, False)
-    kt = cm.cm_context_kernel_times(ctx.handle, reset=True)
-    ms = e0.elapsed_time(e1)
+        cm.cm_context_kernel_times(ctx.handle, reset=True)
+        cm.cm_context_set_timing(ctx.handle, True)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with ClockSampler(0) as clocks:
+            e0.record(stream)
+            run_all(reqs)
+            e1.record(stream)
+            torch.cuda.synchronize(dev)
+        cm.cm_context_set_timing(ctx.handle, False)
+        kt = cm.cm_context_kernel_times(ctx.handle, reset=True)
+        return e0.elapsed_time(e1), kt, clocks.summary()
+
+    def per_request(rs):
+        for req in rs:
+            one(req)
+
+    def per_group(rs):
+        for g0 in range(0, len(rs), G):
+            grouped(rs[g0:g0 + G])
+
     render_bytes = sum(2 * t * w.bytes_per_token for _, _, t in reqs)
-    peak, peak_src = hbm_peak()
-    render_gbs = render_bytes / (kt["render_ms"] * 1e-3) / 1e9
+    peak, _ = hbm_peak()
+
+    def summary(ms, kt):
+        render_gbs = render_bytes / (kt["render_ms"] * 1e-3) / 1e9
+        return {"value": len(reqs) / (ms * 1e-3), "ms_per_request": ms / len(reqs),
+                "render_gbs": render_gbs, "render_frac_of_measured_hbm": render_gbs / peak,
+                "render_ms_per_request": kt["render_ms"] / len(reqs),
+                "hash_ms_per_request": (kt["leaf_hash_ms"] + kt["inner_hash_ms"]) / len(reqs),
+                "kernel_launches": kt["leaf_hash_launches"] + kt["inner_hash_launches"]
+                + kt["render_launches"]}
+
+    ms1, kt1, clocks1 = timed(per_request)
+    msg, ktg, clocksg = timed(per_group)
+    single = summary(ms1, kt1)
+    group = summary(msg, ktg)
     line = {
-        "mode": "serving sweep", "metric": METRIC, "value": len(reqs) / (ms * 1e-3), "unit": UNIT,
+        "mode": "serving sweep", "metric": METRIC, "value": group["value"], "unit": UNIT,
         "n_gpus": 1, "requests": len(reqs), "higher_is_better": True, "dtype": "bf16",
         "data": "synthetic",
         "config": {"workload": "serving sweep on the Qwen3-4B shape: 64 requests x 3 fragments, "
                                "T ~ U{512..4096}, each delivery re-sent with p = 0.1",
                    "deliveries": sum(len(fd) for fd, _, _ in reqs),
-                   "merged_tokens": sum(t for _, _, t in reqs)},
-        "ms_per_request": ms / len(reqs),
-        "render_gbs": render_gbs, "render_frac_of_measured_hbm": render_gbs / peak,
-        "render_ms_per_request": kt["render_ms"] / len(reqs),
-        "hash_ms_per_request": (kt["leaf_hash_ms"] + kt["inner_hash_ms"]) / len(reqs),
-        "kernel_launches": kt["leaf_hash_launches"] + kt["inner_hash_launches"] + kt["render_launches"],
-        "clocks": clocks.summary(),
+                   "merged_tokens": sum(t for _, _, t in reqs),
+                   "group": G},
+        "grouped": dict(group, clocks=clocksg),
+        "per_request": dict(single, clocks=clocks1),
     }
     print(json.dumps(line), flush=True)
     ctx.close()
@@ -391,8 +430,9 @@ def main():
         half = (len(fd) + 1) // 2
         if timers is not None:
             timers["ingest"][0].record(stream)
-        cm.cm_ingest_batch(a, fd[:half], stream)    # replica A
-        cm.cm_ingest_batch(b, fd[half:], stream)    # replica B
+        # replica A takes the first half of the deliveries, replica B the rest: one
+        # cm_ingest_many call, so one GPU pass and one synchronisation for both
+        cm.cm_ingest_many([a] * half + [b] * (len(fd) - half), fd, stream)
         if timers is not None:
             timers["ingest"][1].record(stream)
         cm.cm_union(a, b)   # replica exchange: A := A u B
@@ -520,6 +560,10 @@ def main():
             "algorithmic_ops_per_launch": HASH_ALU_OPS_PER_BYTE * frag_bytes,
             "bytes_hashed_per_launch": frag_bytes, "ms_per_launch": leaf_ms,
             "hash_gbs": frag_bytes / (leaf_ms * 1e-3) / 1e9,
+            "hash_frac_of_measured_hbm": frag_bytes / (leaf_ms * 1e-3) / 1e9 / peak,
+            # against every integer lane of an SM (ALU and FMA pipes, 128 per clock); only
+            # the ALU pipe's 64 can take the xors and rotates, which is what binds
+            "frac_of_128_int_lanes": hash_tops / (alu_peak * 128 / ALU_OPS_PER_CLK_PER_SM),
         }
         per_step = {"leaf_hash": ktimes["leaf_hash_ms"] / args.steps,
                     "inner_hash": ktimes["inner_hash_ms"] / args.steps,

@@ -44,7 +44,7 @@
 extern "C" {
 #endif
 
-#define CM_ABI_VERSION 1
+#define CM_ABI_VERSION 2
 
 /* Same type as cudaStream_t (a CUDA runtime stream handle); NULL is the legacy default stream. */
 typedef struct CUstream_st *cm_stream_t;
@@ -165,6 +165,21 @@ cm_status cm_ingest(cm_set *set, const cm_fragment *frag, cm_stream_t stream, cm
 cm_status cm_ingest_batch(cm_set *set, const cm_fragment *frags, int32_t n, cm_stream_t stream,
                           cm_id *out_ids, int32_t *out_absorbed);
 
+/* Ingest of n deliveries into several sets (Algorithm 2, Ingest, applied to each
+ * delivery): delivery i goes into sets[i]; entries may repeat, so one call can feed
+ * many serving requests. The result is that of calling cm_ingest for i = 0..n-1 in
+ * order; the GPU work for all deliveries is one pass (as in cm_ingest_batch) with a
+ * single synchronisation of `stream`. All sets must come from one context
+ * (CM_ERR_INVALID_ARG); each delivery must have its set's shape, where a set that is
+ * empty takes the shape of its first delivery (CM_ERR_SHAPE_MISMATCH). Different sets
+ * may have different shapes. Nothing is inserted if validation fails.
+ *   sets          HOST array of n set pointers
+ *   frags         HOST array of n descriptors (n >= 0)
+ *   out_ids       nullable HOST array of n ids
+ *   out_absorbed  nullable HOST array of n flags */
+cm_status cm_ingest_many(cm_set *const *sets, const cm_fragment *frags, int32_t n,
+                         cm_stream_t stream, cm_id *out_ids, int32_t *out_absorbed);
+
 /* Merge of Algorithm 2 (Eq. setunion): dst := dst u src. Host only, no GPU work.
  * Both sets must come from the same context (CM_ERR_INVALID_ARG otherwise) and have
  * the same shape unless one is empty (CM_ERR_SHAPE_MISMATCH). On equal ids dst keeps
@@ -180,6 +195,19 @@ cm_status cm_set_seq_len(const cm_set *set, int64_t *out);
 /* The set's ids in ascending order (bytes compared as a big-endian integer).
  * Writes min(size, capacity) ids to the HOST array out. */
 cm_status cm_set_ids(const cm_set *set, cm_id *out, int64_t capacity);
+
+/* Membership of ids in the set (Section 4.4: the state is the set of fragment
+ * identities). out_present[i] = 1 if ids[i] is in the set, else 0. With cm_set_ids
+ * this lets two replicas exchange ids first and ship only the fragments the other
+ * side lacks; the union that results is the same as shipping the whole state
+ * (Eq. setunion). Host only.
+ *   ids, out_present  HOST arrays of n entries (n >= 0) */
+cm_status cm_set_contains(const cm_set *set, const cm_id *ids, int64_t n, uint8_t *out_present);
+
+/* The inclusion order of Section 4.4: *out = 1 if every id of a is in b (a is below
+ * b in the join-semilattice), else 0. The sets may come from different contexts.
+ * Host only. */
+cm_status cm_set_leq(const cm_set *a, const cm_set *b, int32_t *out);
 
 /* Render(S) of Algorithm 2 = CanonicalMerge (Algorithm 1) of the set's fragments:
  * order them by descending routing-layer mean K-norm over the last T* = min seq_len
@@ -197,6 +225,29 @@ cm_status cm_set_ids(const cm_set *set, cm_id *out, int64_t capacity);
  * or any fragment of the set (the render reads the fragments while it writes). */
 cm_status cm_render(const cm_set *set, void *k_out, void *v_out, int64_t capacity_tokens,
                     cm_stream_t stream, int64_t *out_seq_len, cm_id *out_order);
+
+/* One render job of cm_render_many: a set and its contiguous output, with the
+ * meaning of the arguments of the same names in cm_render. */
+typedef struct cm_render_job {
+    const cm_set *set;
+    void *k_out;                  /* DEVICE, 16-byte aligned, [L][H][capacity_tokens][d] bf16 */
+    void *v_out;
+    int64_t capacity_tokens;
+} cm_render_job;
+
+/* Render(S) of Algorithm 2 for several sets in one pass: jobs[i].set is rendered
+ * into jobs[i].k_out / v_out exactly as cm_render would (the same bytes), but the
+ * slots of all sets are packed into shared launches of the render kernel instead
+ * of at least one launch per set, which keeps the GPU full when the sets are small
+ * (many concurrent serving requests). All sets must come from one context
+ * (CM_ERR_INVALID_ARG) and every non-empty set must have the same (L, H, d)
+ * (CM_ERR_SHAPE_MISMATCH); each job is validated as in cm_render before anything
+ * is launched. Outputs must not overlap one another or any fragment of any job.
+ * Enqueued on `stream`; returns without waiting.
+ *   jobs          HOST array of n jobs (n >= 0)
+ *   out_seq_lens  nullable HOST array of n: the rendered length of each set */
+cm_status cm_render_many(const cm_render_job *jobs, int32_t n, cm_stream_t stream,
+                         int64_t *out_seq_lens);
 
 /* Incremental Render(S) (addresses the lazy O(m) re-render of Section 7): k_out and
  * v_out already hold the render of an earlier state whose canonical order was

@@ -71,6 +71,11 @@ class cm_paged_cache(ctypes.Structure):
                 ("stride_token", ctypes.c_int64)]
 
 
+class cm_render_job(ctypes.Structure):
+    _fields_ = [("set", ctypes.c_void_p), ("k_out", ctypes.c_void_p), ("v_out", ctypes.c_void_p),
+                ("capacity_tokens", ctypes.c_int64)]
+
+
 _c = ctypes
 _P = ctypes.c_void_p
 _SIGS = {
@@ -90,6 +95,12 @@ _SIGS = {
                                          _c.POINTER(_c.c_uint64)]),
     "cm_ingest_batch": (_c.c_int, [_P, _c.POINTER(cm_fragment), _c.c_int32, _P,
                                    _c.POINTER(cm_id), _c.POINTER(_c.c_int32)]),
+    "cm_ingest_many": (_c.c_int, [_c.POINTER(_P), _c.POINTER(cm_fragment), _c.c_int32, _P,
+                                  _c.POINTER(cm_id), _c.POINTER(_c.c_int32)]),
+    "cm_render_many": (_c.c_int, [_c.POINTER(cm_render_job), _c.c_int32, _P,
+                                  _c.POINTER(_c.c_int64)]),
+    "cm_set_contains": (_c.c_int, [_P, _c.POINTER(cm_id), _c.c_int64, _c.POINTER(_c.c_uint8)]),
+    "cm_set_leq": (_c.c_int, [_P, _P, _c.POINTER(_c.c_int32)]),
     "cm_context_set_timing": (_c.c_int, [_P, _c.c_int32]),
     "cm_context_kernel_times": (_c.c_int, [_P, _c.POINTER(cm_kernel_times), _c.c_int32]),
     "cm_union": (_c.c_int, [_P, _P]),
@@ -205,6 +216,43 @@ def cm_ingest_batch(s: int, frags: Sequence[cm_fragment], stream=None) -> List[T
     absorbed = (ctypes.c_int32 * max(n, 1))()
     _check(lib.cm_ingest_batch(s, arr, n, _stream_handle(stream), ids, absorbed))
     return [(ids[i].to_bytes(), bool(absorbed[i])) for i in range(n)]
+
+
+def cm_ingest_many(sets: Sequence[int], frags: Sequence[cm_fragment],
+                   stream=None) -> List[Tuple[bytes, bool]]:
+    n = len(frags)
+    if len(sets) != n:
+        raise ValueError("one set per delivery")
+    set_arr = (_P * max(n, 1))(*sets)
+    arr = (cm_fragment * max(n, 1))(*frags)
+    ids = (cm_id * max(n, 1))()
+    absorbed = (ctypes.c_int32 * max(n, 1))()
+    _check(lib.cm_ingest_many(set_arr, arr, n, _stream_handle(stream), ids, absorbed))
+    return [(ids[i].to_bytes(), bool(absorbed[i])) for i in range(n)]
+
+
+def cm_render_many(jobs: Sequence[cm_render_job], stream=None) -> List[int]:
+    n = len(jobs)
+    arr = (cm_render_job * max(n, 1))(*jobs)
+    seq = (ctypes.c_int64 * max(n, 1))()
+    _check(lib.cm_render_many(arr, n, _stream_handle(stream), seq))
+    return [seq[i] for i in range(n)]
+
+
+def cm_set_contains(s: int, ids: Sequence[bytes]) -> List[bool]:
+    n = len(ids)
+    arr = (cm_id * max(n, 1))()
+    for i, fid in enumerate(ids):
+        arr[i].b[:] = list(fid)
+    out = (ctypes.c_uint8 * max(n, 1))()
+    _check(lib.cm_set_contains(s, arr, n, out))
+    return [bool(out[i]) for i in range(n)]
+
+
+def cm_set_leq(a: int, b: int) -> bool:
+    out = ctypes.c_int32()
+    _check(lib.cm_set_leq(a, b, ctypes.byref(out)))
+    return bool(out.value)
 
 
 def cm_context_set_timing(ctx: int, enable: bool) -> None:
@@ -373,6 +421,14 @@ class FragmentSet:
     def __len__(self) -> int:
         return cm_set_size(self.handle)
 
+    def contains(self, ids: Sequence[bytes]) -> List[bool]:
+        """Membership of each id (for replica exchange: ship only what the other lacks)."""
+        return cm_set_contains(self.handle, ids)
+
+    def __le__(self, other: "FragmentSet") -> bool:
+        """The inclusion order of Section 4.4: every id of self is in other."""
+        return cm_set_leq(self.handle, other.handle)
+
     def ids(self) -> List[bytes]:
         return cm_set_ids(self.handle)
 
@@ -388,3 +444,22 @@ class FragmentSet:
         return cm_render(self.handle, k_out.data_ptr() if k_out is not None else 0,
                          v_out.data_ptr() if v_out is not None else 0,
                          k_out.shape[2] if k_out is not None else 0, stream)
+
+
+def ingest_many(deliveries, stream=None) -> List[Tuple[bytes, bool]]:
+    """Ingest [(FragmentSet, K, V), ...] in order, one GPU pass and one synchronisation
+    for all of them; deliveries may go to different sets."""
+    res = cm_ingest_many([S.handle for S, _, _ in deliveries],
+                         [fragment_from_tensors(K, V) for _, K, V in deliveries], stream)
+    for (fid, absorbed), (S, K, V) in zip(res, deliveries):
+        if not absorbed:
+            S._keep.setdefault(fid, (K, V))
+    return res
+
+
+def render_many(jobs, stream=None) -> List[int]:
+    """Render [(FragmentSet, k_out, v_out), ...] in shared launches; returns the lengths."""
+    return cm_render_many([cm_render_job(S.handle, k.data_ptr() if k is not None else 0,
+                                         v.data_ptr() if v is not None else 0,
+                                         k.shape[2] if k is not None else 0)
+                           for S, k, v in jobs], stream)

@@ -20,6 +20,7 @@
 #include <mutex>
 #include <new>
 #include <string>
+#include <unordered_map>
 #include <vector>
 
 #include <cuda_runtime.h>
@@ -157,10 +158,13 @@ int32_t routing_layer_for(const cm_context *ctx, int32_t L) {
 
 cm_status ensure_scratch(cm_context *ctx, size_t dev_bytes, size_t host_bytes) {
     if (dev_bytes > ctx->scratch_bytes) {
+        const size_t old_dev = ctx->scratch_bytes;
         if (ctx->d_scratch) cudaFree(ctx->d_scratch);
         ctx->d_scratch = nullptr;
         ctx->scratch_bytes = 0;
-        const size_t want = std::max(dev_bytes, (size_t)1 << 20);
+        // grown by at least half its size, so a stream of slowly growing requests
+        // reallocates (a device-wide synchronisation) only O(log) times
+        const size_t want = std::max({dev_bytes, old_dev + old_dev / 2, (size_t)1 << 20});
         cudaError_t e = cudaMalloc(&ctx->d_scratch, want);
         if (e != cudaSuccess) {
             cudaGetLastError();
@@ -170,10 +174,11 @@ cm_status ensure_scratch(cm_context *ctx, size_t dev_bytes, size_t host_bytes) {
         ctx->scratch_bytes = want;
     }
     if (host_bytes > ctx->pinned_bytes) {
+        const size_t old_host = ctx->pinned_bytes;
         if (ctx->h_pinned) cudaFreeHost(ctx->h_pinned);
         ctx->h_pinned = nullptr;
         ctx->pinned_bytes = 0;
-        const size_t want = std::max(host_bytes, (size_t)1 << 16);
+        const size_t want = std::max({host_bytes, old_host + old_host / 2, (size_t)1 << 16});
         cudaError_t e = cudaHostAlloc(reinterpret_cast<void **>(&ctx->h_pinned), want,
                                       cudaHostAllocDefault);
         if (e != cudaSuccess) {
@@ -407,19 +412,24 @@ cm_status bytes_equal(cm_context *ctx, const cm_fragment *f, const Record &r, cu
     return CM_OK;
 }
 
-// One slot of a render: a fragment and its output offset.
+// One slot of a render: a fragment, its output offset and its set's contiguous
+// output (ignored for paged outputs).
 struct Slot {
     const void *k;
     const void *v;
     int64_t T;
     int64_t offset;
+    void *k_out;
+    void *v_out;
+    int64_t capacity;
 };
 
 // Fused copy-and-rotate of slots already in order (offsets set), in launch groups
-// of at most kMaxSlots slots and kMaxTablePairs (cos, sin) pairs.
+// of at most kMaxSlots slots and kMaxTablePairs (cos, sin) pairs. The slots may
+// belong to several sets of one shape: each slot carries its own output.
 cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t L, int32_t H,
-                       int32_t d, void *k_out, void *v_out, int64_t capacity, cudaStream_t stream,
-                       uint32_t withhold_warp = 0, const cm_paged_cache *paged = nullptr) {
+                       int32_t d, cudaStream_t stream, uint32_t withhold_warp = 0,
+                       const cm_paged_cache *paged = nullptr) {
     const int rows_per_chunk = cm::kChunkBytes / (2 * d);
     const int half = d / 2;
     const int max_group = std::min<int>(cm::kMaxSlots, cm::kMaxTablePairs / half);
@@ -435,9 +445,6 @@ cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t 
     for (size_t g0 = 0; g0 < slots.size(); g0 += (size_t)max_group) {
         const size_t n = std::min(slots.size() - g0, (size_t)max_group);
         std::memset(p.get(), 0, sizeof(cm::RenderParams));
-        p->k_out = k_out;
-        p->v_out = v_out;
-        p->capacity = capacity;
         p->num_layers = L;
         p->num_heads = H;
         p->head_dim = d;
@@ -450,6 +457,9 @@ cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t 
             cm::RenderSlot &rs = p->slot[i];
             rs.k = s.k;
             rs.v = s.v;
+            rs.k_out = s.k_out;
+            rs.v_out = s.v_out;
+            rs.capacity = s.capacity;
             rs.seq_len = s.T;
             rs.offset = s.offset;
             rs.rotate = s.offset != 0;
@@ -458,7 +468,7 @@ cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t 
             rs.chunk_begin = (uint32_t)chunk;
             rs.chunks_per_plane = (uint32_t)cpp;
             chunk += cpp * planes;
-            // delta angle a_j = s * theta^(-2j/d) in fp64 (Section 2.3 / Eq. bagmerge-k);
+            // delta angle a_j = s * theta^(-2j/d) in fp64 (Section 4.2, Eq. bagmerge-k);
             // the slot at offset 0 is copied and needs no table
             if (rs.rotate) {
                 for (int j = 0; j < half; ++j) {
@@ -475,6 +485,8 @@ cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t 
         p->withhold_warp = g0 == 0 ? withhold_warp : 0;
         if (paged) {
             p->paged = 1;
+            p->k_pool = paged->k_pool;
+            p->v_pool = paged->v_pool;
             p->block_table = paged->block_table;
             p->block_size = paged->block_size;
             p->log2_block_size = is_pow2(paged->block_size)
@@ -546,6 +558,85 @@ cm_status guarded(F &&f) {
     } catch (...) {
         return fail(CM_ERR_INVALID_ARG, "unexpected internal error");
     }
+}
+
+// Ingest (Algorithm 2) of n deliveries, delivery i into sets[i] (several entries
+// may name one set): one GPU pass for all of them, then the insertions in delivery
+// order, so a delivery whose id its set already holds (before the batch or from an
+// earlier delivery of it) is absorbed. Nothing is inserted if validation fails.
+cm_status ingest_deliveries(cm_set *const *sets, const cm_fragment *frags, int32_t n,
+                            cm_stream_t stream, cm_id *out_ids, int32_t *out_absorbed) {
+    if (n == 0) return CM_OK;
+    cm_context *ctx = sets[0]->ctx;
+    struct Shape {
+        bool has;
+        int32_t L, H, d;
+    };
+    std::unordered_map<const cm_set *, Shape> shape;
+    std::vector<const cm_fragment *> fp((size_t)n);
+    for (int32_t i = 0; i < n; ++i) {
+        const cm_set *set = sets[i];
+        if (set->ctx != ctx) return fail(CM_ERR_INVALID_ARG, "sets belong to different contexts");
+        const cm_fragment *f = &frags[i];
+        cm_status st = validate_fragment(f);
+        if (st != CM_OK) return st;
+        auto it = shape.find(set);
+        if (it == shape.end())
+            it = shape.emplace(set, Shape{set->has_shape, set->L, set->H, set->d}).first;
+        Shape &sh = it->second;
+        if (!sh.has) {
+            sh = Shape{true, f->num_layers, f->num_kv_heads, f->head_dim};
+        } else if (f->num_layers != sh.L || f->num_kv_heads != sh.H || f->head_dim != sh.d) {
+            return fail(CM_ERR_SHAPE_MISMATCH,
+                        "fragment (layers, kv_heads, head_dim) differ from the set's");
+        }
+        if (routing_layer_for(ctx, f->num_layers) >= f->num_layers)
+            return fail(CM_ERR_INVALID_ARG, "routing layer >= num_layers");
+        fp[(size_t)i] = f;
+    }
+    std::lock_guard<std::mutex> lock(ctx->mu);
+    DeviceScope scope(ctx->device);
+    if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
+    const cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+    std::vector<cm_id> ids((size_t)n);
+    std::vector<std::vector<uint64_t>> Qs((size_t)n);
+    cm_status st = fragments_digest(ctx, fp.data(), (size_t)n, cs, ids.data(), Qs.data());
+    if (st != CM_OK) return st;
+    for (int32_t i = 0; i < n; ++i) {
+        cm_set *set = sets[i];
+        const cm_fragment *f = fp[(size_t)i];
+        if (out_ids) out_ids[i] = ids[(size_t)i];
+        const IdKey key = key_of(ids[(size_t)i]);
+        auto it = set->items.find(key);
+        if (it != set->items.end()) {
+            if (ctx->verify) {
+                bool equal = false;
+                st = bytes_equal(ctx, f, *it->second, cs, &equal);
+                if (st != CM_OK) return st;
+                if (!equal) return fail(CM_ERR_COLLISION, "content address hit with different bytes");
+            }
+            if (out_absorbed) out_absorbed[i] = 1;
+            continue;
+        }
+        auto rec = std::make_shared<Record>();
+        rec->id = ids[(size_t)i];
+        rec->L = f->num_layers;
+        rec->H = f->num_kv_heads;
+        rec->T = f->seq_len;
+        rec->d = f->head_dim;
+        rec->k = f->k;
+        rec->v = f->v;
+        rec->Q = std::move(Qs[(size_t)i]);
+        set->items.emplace(key, std::move(rec));
+        if (!set->has_shape) {
+            set->has_shape = true;
+            set->L = f->num_layers;
+            set->H = f->num_kv_heads;
+            set->d = f->head_dim;
+        }
+        if (out_absorbed) out_absorbed[i] = 0;
+    }
+    return CM_OK;
 }
 
 }  // namespace
@@ -678,75 +769,23 @@ cm_status cm_ingest_batch(cm_set *set, const cm_fragment *frags, int32_t n, cm_s
     return guarded([&]() -> cm_status {
         if (!set) return fail(CM_ERR_INVALID_ARG, "set is NULL");
         if (n < 0 || (n > 0 && !frags)) return fail(CM_ERR_INVALID_ARG, "need n >= 0 fragments");
-        if (n == 0) return CM_OK;
-        cm_context *ctx = set->ctx;
-        bool has_shape = set->has_shape;
-        int32_t L = set->L, H = set->H, d = set->d;
-        std::vector<const cm_fragment *> fp((size_t)n);
-        for (int32_t i = 0; i < n; ++i) {
-            const cm_fragment *f = &frags[i];
-            cm_status st = validate_fragment(f);
-            if (st != CM_OK) return st;
-            if (!has_shape) {
-                has_shape = true;
-                L = f->num_layers;
-                H = f->num_kv_heads;
-                d = f->head_dim;
-            } else if (f->num_layers != L || f->num_kv_heads != H || f->head_dim != d) {
-                return fail(CM_ERR_SHAPE_MISMATCH,
-                            "fragment (layers, kv_heads, head_dim) differ from the set's");
-            }
-            if (routing_layer_for(ctx, f->num_layers) >= f->num_layers)
-                return fail(CM_ERR_INVALID_ARG, "routing layer >= num_layers");
-            fp[(size_t)i] = f;
-        }
-        std::lock_guard<std::mutex> lock(ctx->mu);
-        DeviceScope scope(ctx->device);
-        if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
-        const cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
-        std::vector<cm_id> ids((size_t)n);
-        std::vector<std::vector<uint64_t>> Qs((size_t)n);
-        cm_status st = fragments_digest(ctx, fp.data(), (size_t)n, cs, ids.data(), Qs.data());
-        if (st != CM_OK) return st;
-        // Ingest in order: a later delivery with an id already present (in the set or
-        // earlier in this batch) is absorbed.
-        for (int32_t i = 0; i < n; ++i) {
-            const cm_fragment *f = fp[(size_t)i];
-            if (out_ids) out_ids[i] = ids[(size_t)i];
-            const IdKey key = key_of(ids[(size_t)i]);
-            auto it = set->items.find(key);
-            if (it != set->items.end()) {
-                if (ctx->verify) {
-                    bool equal = false;
-                    st = bytes_equal(ctx, f, *it->second, cs, &equal);
-                    if (st != CM_OK) return st;
-                    if (!equal)
-                        return fail(CM_ERR_COLLISION, "content address hit with different bytes");
-                }
-                if (out_absorbed) out_absorbed[i] = 1;
-                continue;
-            }
-            auto rec = std::make_shared<Record>();
-            rec->id = ids[(size_t)i];
-            rec->L = f->num_layers;
-            rec->H = f->num_kv_heads;
-            rec->T = f->seq_len;
-            rec->d = f->head_dim;
-            rec->k = f->k;
-            rec->v = f->v;
-            rec->Q = std::move(Qs[(size_t)i]);
-            set->items.emplace(key, std::move(rec));
-            if (!set->has_shape) {
-                set->has_shape = true;
-                set->L = f->num_layers;
-                set->H = f->num_kv_heads;
-                set->d = f->head_dim;
-            }
-            if (out_absorbed) out_absorbed[i] = 0;
-        }
-        return CM_OK;
+        const std::vector<cm_set *> sets((size_t)n, set);
+        return ingest_deliveries(sets.data(), frags, n, stream, out_ids, out_absorbed);
     });
 }
+
+cm_status cm_ingest_many(cm_set *const *sets, const cm_fragment *frags, int32_t n,
+                         cm_stream_t stream, cm_id *out_ids, int32_t *out_absorbed) {
+    TraceRange trace("cm_ingest");
+    return guarded([&]() -> cm_status {
+        if (n < 0 || (n > 0 && (!frags || !sets)))
+            return fail(CM_ERR_INVALID_ARG, "need n >= 0 fragments and their sets");
+        for (int32_t i = 0; i < n; ++i)
+            if (!sets[i]) return fail(CM_ERR_INVALID_ARG, "a set is NULL");
+        return ingest_deliveries(sets, frags, n, stream, out_ids, out_absorbed);
+    });
+}
+
 
 cm_status cm_context_set_timing(cm_context *ctx, int32_t enable) {
     if (!ctx) return fail(CM_ERR_INVALID_ARG, "context is NULL");
@@ -879,7 +918,8 @@ cm_status render_set(const cm_set *set, void *k_out, void *v_out, int64_t capaci
             if (i < keep)
                 reused += order[i]->T;
             else
-                slots.push_back({order[i]->k, order[i]->v, order[i]->T, s});
+                slots.push_back({order[i]->k, order[i]->v, order[i]->T, s, k_out, v_out,
+                                 capacity_tokens});
             s += order[i]->T;
         }
         if (out_reused_tokens) *out_reused_tokens = reused;
@@ -888,7 +928,7 @@ cm_status render_set(const cm_set *set, void *k_out, void *v_out, int64_t capaci
         std::lock_guard<std::mutex> lock(ctx->mu);
         DeviceScope scope(ctx->device);
         if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
-        return launch_slots(ctx, slots, set->L, set->H, set->d, k_out, v_out, capacity_tokens,
+        return launch_slots(ctx, slots, set->L, set->H, set->d,
                             reinterpret_cast<cudaStream_t>(stream), withhold_warp, paged);
     });
 }
@@ -898,6 +938,77 @@ cm_status render_set(const cm_set *set, void *k_out, void *v_out, int64_t capaci
 cm_status cm_render(const cm_set *set, void *k_out, void *v_out, int64_t capacity_tokens,
                     cm_stream_t stream, int64_t *out_seq_len, cm_id *out_order) {
     return render_set(set, k_out, v_out, capacity_tokens, stream, out_seq_len, out_order, 0);
+}
+
+cm_status cm_render_many(const cm_render_job *jobs, int32_t n, cm_stream_t stream,
+                         int64_t *out_seq_lens) {
+    TraceRange trace("cm_render");
+    return guarded([&]() -> cm_status {
+        if (n < 0 || (n > 0 && !jobs)) return fail(CM_ERR_INVALID_ARG, "need n >= 0 jobs");
+        cm_context *ctx = nullptr;
+        bool has_shape = false;
+        int32_t L = 0, H = 0, d = 0;
+        std::vector<int64_t> totals((size_t)n);
+        for (int32_t i = 0; i < n; ++i) {
+            const cm_render_job &j = jobs[i];
+            if (!j.set) return fail(CM_ERR_INVALID_ARG, "a job's set is NULL");
+            if (j.capacity_tokens < 0) return fail(CM_ERR_INVALID_ARG, "capacity_tokens < 0");
+            if (ctx && j.set->ctx != ctx)
+                return fail(CM_ERR_INVALID_ARG, "sets belong to different contexts");
+            ctx = j.set->ctx;
+            int64_t total = 0;
+            for (const auto &kv : j.set->items) total += kv.second->T;
+            cm_status st = validate_outputs(j.k_out, j.v_out, j.capacity_tokens, total);
+            if (st != CM_OK) return st;
+            totals[(size_t)i] = total;
+            if (total == 0) continue;
+            if (!has_shape) {
+                has_shape = true;
+                L = j.set->L;
+                H = j.set->H;
+                d = j.set->d;
+            } else if (j.set->L != L || j.set->H != H || j.set->d != d) {
+                return fail(CM_ERR_SHAPE_MISMATCH, "sets of one cm_render_many call differ in shape");
+            }
+        }
+        std::vector<Slot> slots;
+        for (int32_t i = 0; i < n; ++i) {
+            const cm_render_job &j = jobs[i];
+            int64_t s = 0;
+            for (const auto &r : canonical_order(j.set)) {
+                slots.push_back({r->k, r->v, r->T, s, j.k_out, j.v_out, j.capacity_tokens});
+                s += r->T;
+            }
+        }
+        if (out_seq_lens)
+            for (int32_t i = 0; i < n; ++i) out_seq_lens[i] = totals[(size_t)i];
+        if (slots.empty()) return CM_OK;
+        std::lock_guard<std::mutex> lock(ctx->mu);
+        DeviceScope scope(ctx->device);
+        if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
+        return launch_slots(ctx, slots, L, H, d, reinterpret_cast<cudaStream_t>(stream));
+    });
+}
+
+cm_status cm_set_contains(const cm_set *set, const cm_id *ids, int64_t n, uint8_t *out_present) {
+    if (!set) return fail(CM_ERR_INVALID_ARG, "set is NULL");
+    if (n < 0 || (n > 0 && (!ids || !out_present)))
+        return fail(CM_ERR_INVALID_ARG, "need n >= 0 ids and an output array");
+    for (int64_t i = 0; i < n; ++i)
+        out_present[i] = set->items.count(key_of(ids[i])) ? 1 : 0;
+    return CM_OK;
+}
+
+cm_status cm_set_leq(const cm_set *a, const cm_set *b, int32_t *out) {
+    if (!a || !b || !out) return fail(CM_ERR_INVALID_ARG, "a, b or out is NULL");
+    int32_t leq = 1;
+    for (const auto &kv : a->items)
+        if (!b->items.count(kv.first)) {
+            leq = 0;
+            break;
+        }
+    *out = leq;
+    return CM_OK;
 }
 
 cm_status cm_render_incremental(const cm_set *set, void *k_out, void *v_out,
@@ -957,7 +1068,8 @@ cm_status cm_bagmerge(cm_context *ctx, const cm_fragment *frags, int32_t n, void
         std::vector<Slot> slots;
         int64_t s = 0;
         for (int32_t i = 0; i < n; ++i) {
-            slots.push_back({frags[i].k, frags[i].v, frags[i].seq_len, s});
+            slots.push_back({frags[i].k, frags[i].v, frags[i].seq_len, s, k_out, v_out,
+                             capacity_tokens});
             s += frags[i].seq_len;
         }
         if (out_seq_len) *out_seq_len = total;
@@ -965,8 +1077,7 @@ cm_status cm_bagmerge(cm_context *ctx, const cm_fragment *frags, int32_t n, void
         DeviceScope scope(ctx->device);
         if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
         return launch_slots(ctx, slots, frags[0].num_layers, frags[0].num_kv_heads,
-                            frags[0].head_dim, k_out, v_out, capacity_tokens,
-                            reinterpret_cast<cudaStream_t>(stream));
+                            frags[0].head_dim, reinterpret_cast<cudaStream_t>(stream));
     });
 }
 

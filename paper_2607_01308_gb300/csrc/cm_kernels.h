@@ -84,6 +84,9 @@ constexpr int kChunkBytes = 4096;      // bytes of one source plane handled per 
 struct RenderSlot {
     const void *k;              // source K [L][H][T][d], device
     const void *v;              // source V
+    void *k_out;                // contiguous output of the slot's set, [L][H][capacity][d]
+    void *v_out;                // (unused for paged outputs)
+    int64_t capacity;           // token rows per (layer, head) plane of k_out / v_out
     int64_t seq_len;            // T
     int64_t offset;             // s: first output position of this slot
     uint32_t chunk_begin;       // first global work item of this slot
@@ -94,9 +97,8 @@ struct RenderSlot {
 
 // Passed by value (kernel parameter space, < 32 KiB), so a launch owns its table.
 struct RenderParams {
-    void *k_out;                // [L][H][capacity][d], device
-    void *v_out;
-    int64_t capacity;
+    void *k_pool;               // paged outputs only: the block pools (see below)
+    void *v_pool;
     int32_t num_layers;
     int32_t num_heads;
     int32_t head_dim;
@@ -111,7 +113,7 @@ struct RenderParams {
     int32_t paged;              // 1: outputs are block pools addressed through block_table
     // paged output: token pos of (layer l, head h) lives at pool + block_table[pos / block_size]
     // * stride_block + l * stride_layer + h * stride_head + (pos % block_size) * stride_token
-    // (element strides, head_dim contiguous); k_out / v_out are the pools
+    // (element strides, head_dim contiguous)
     const int32_t *block_table; // device
     int64_t block_size;
     int32_t log2_block_size;    // >= 0 when block_size is a power of two, else -1

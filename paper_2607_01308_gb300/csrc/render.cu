@@ -270,11 +270,11 @@ __device__ __forceinline__ Item item_of(const RenderParams &p, uint32_t g) {
     it.src = static_cast<const uint8_t *>(is_v ? S.v : S.k) + (lh * S.seq_len + row0) * row_bytes;
     if (p.paged) {
         const int64_t l = lh / p.num_heads, h = lh - l * p.num_heads;
-        it.dst = static_cast<uint8_t *>(is_v ? p.v_out : p.k_out) +
+        it.dst = static_cast<uint8_t *>(is_v ? p.v_pool : p.k_pool) +
                  (l * p.stride_layer + h * p.stride_head) * 2;
     } else {
-        it.dst = static_cast<uint8_t *>(is_v ? p.v_out : p.k_out) +
-                 (lh * p.capacity + S.offset + row0) * row_bytes;
+        it.dst = static_cast<uint8_t *>(is_v ? S.v_out : S.k_out) +
+                 (lh * S.capacity + S.offset + row0) * row_bytes;
     }
     it.pos0 = S.offset + row0;
     it.bytes = (uint32_t)(rows * row_bytes);

@@ -20,6 +20,18 @@ int main(void) {
     memset(&pc, 0, sizeof pc);
     if (cm_render_paged(NULL, &pc, NULL, NULL, NULL) != CM_ERR_INVALID_ARG) return 5;
     if (cm_testing_render_withheld_load(NULL, NULL, NULL, 0, NULL) != CM_ERR_INVALID_ARG) return 6;
+    /* the calls over several sets: zero items is a no-op, a NULL set is refused */
+    if (cm_render_many(NULL, 0, NULL, NULL) != CM_OK) return 7;
+    if (cm_ingest_many(NULL, NULL, 0, NULL, NULL, NULL) != CM_OK) return 8;
+    cm_render_job job;
+    memset(&job, 0, sizeof job);
+    if (cm_render_many(&job, 1, NULL, NULL) != CM_ERR_INVALID_ARG) return 9;
+    cm_set *no_set = NULL;
+    if (cm_ingest_many(&no_set, &f, 1, NULL, NULL, NULL) != CM_ERR_INVALID_ARG) return 10;
+    uint8_t present = 0;
+    int32_t leq = 0;
+    if (cm_set_contains(NULL, &id, 1, &present) != CM_ERR_INVALID_ARG) return 11;
+    if (cm_set_leq(NULL, NULL, &leq) != CM_ERR_INVALID_ARG) return 12;
     printf("ok %s\n", cm_last_error_message());
     return 0;
 }

@@ -31,7 +31,8 @@ def test_header_declares_the_documented_calls():
             "cm_set_seq_len", "cm_set_ids", "cm_render", "cm_bagmerge", "cm_status_string",
             "cm_last_error_message", "cm_context_check", "cm_ingest_batch",
             "cm_context_set_timing", "cm_context_kernel_times", "cm_fragment_id_static",
-            "cm_render_incremental", "cm_render_paged"}
+            "cm_render_incremental", "cm_render_paged", "cm_ingest_many", "cm_render_many",
+            "cm_set_contains", "cm_set_leq"}
     assert want <= set(_declared_functions())
 
 
@@ -43,7 +44,7 @@ def test_library_exports_every_declared_symbol(cm):
 
 
 def test_abi_version_and_status_strings(cm):
-    assert cm.cm_abi_version() == 1
+    assert cm.cm_abi_version() == 2
     for st in cm.Status:
         assert cm.cm_status_string(int(st)) == "CM_" + st.name
     assert cm.cm_status_string(99) == "CM_ERR_UNKNOWN"

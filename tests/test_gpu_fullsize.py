@@ -68,8 +68,9 @@ def test_q4b_full_size_bench_configuration(ctx):
     frags = [synthetic.make_fragment_torch(sp, w.num_layers, w.num_kv_heads, w.head_dim, "cuda:0")
              for sp in specs]
     A, B = cm.FragmentSet(ctx), cm.FragmentSet(ctx)
-    ra = A.ingest_batch(frags[:2])
-    rb = B.ingest_batch(frags[2:])
+    # the bench's launch configuration: one cm_ingest_many call feeds both replicas
+    res = cm.ingest_many([(A, *frags[0]), (A, *frags[1]), (B, *frags[2]), (B, *frags[3])])
+    ra, rb = res[:2], res[2:]
     A.union(B)
     total = sum(sp.seq_len for sp in specs)
     k_out, v_out = empty_out(w.num_layers, w.num_kv_heads, total, w.head_dim)
