@@ -423,7 +423,8 @@ def main():
 
     ev = lambda: torch.cuda.Event(enable_timing=True)
 
-    def one_merge(timers=None, inputs=None):
+    def one_merge(timers=None, inputs=None, out=None):
+        k_dst, v_dst = out or (k_out, v_out)
         a = cm.cm_set_create(ctx.handle)
         b = cm.cm_set_create(ctx.handle)
         fd = inputs or fdesc
@@ -438,7 +439,7 @@ def main():
         cm.cm_union(a, b)   # replica exchange: A := A u B
         if timers is not None:
             timers["render"][0].record(stream)
-        n, _ = cm.cm_render(a, k_out.data_ptr(), v_out.data_ptr(), total_T, stream)
+        n, _ = cm.cm_render(a, k_dst.data_ptr(), v_dst.data_ptr(), total_T, stream)
         if timers is not None:
             timers["render"][1].record(stream)
         cm.cm_set_destroy(b)
@@ -498,39 +499,93 @@ def main():
         cm.cm_set_destroy(ps)
         del pool_k, pool_v
 
-    # end to end through the C ABI with host buffers: pinned inputs copied in and the
-    # merged cache copied out inside the timed region, every step
-    e2e_steps = args.e2e_steps or min(args.steps, 10)
+    # end to end through the C ABI with host buffers: every step copies its inputs in from
+    # pinned host memory and the whole merged cache out to pinned host memory
+    e2e_steps = args.e2e_steps or min(args.steps, 20)
     host_in = [(K.cpu().pin_memory(), V.cpu().pin_memory()) for K, V in frags]
-    dev_in = [(torch.empty_like(K), torch.empty_like(V)) for K, V in frags]
-    dev_desc = [cm.fragment_from_tensors(K, V) for K, V in dev_in]
     host_out = (torch.empty(k_out.shape, dtype=k_out.dtype, pin_memory=True),
                 torch.empty(v_out.shape, dtype=v_out.dtype, pin_memory=True))
     h2d = sum(K.numel() * 2 + V.numel() * 2 for K, V in host_in)
     d2h = 2 * k_out.numel() * 2
+    # two device copies of the inputs and of the output: while step i merges, step i+1's
+    # inputs stream in and step i-1's merged cache streams out (the host link carries both
+    # directions at once faster than one after the other)
+    dev_in = [[(torch.empty_like(K), torch.empty_like(V)) for K, V in frags] for _ in range(2)]
+    dev_desc = [[cm.fragment_from_tensors(K, V) for K, V in di] for di in dev_in]
+    dev_out = [(k_out, v_out), (torch.empty_like(k_out), torch.empty_like(v_out))]
+    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    mk = lambda: torch.cuda.Event()
+    in_ready, in_free = [mk(), mk()], [mk(), mk()]
+    out_ready, out_free = [mk(), mk()], [mk(), mk()]
 
-    def e2e_step():
-        for (hk, hv), (dk, dv) in zip(host_in, dev_in):
+    def copy_in(i):
+        b = i % 2
+        s_in.wait_event(in_free[b])
+        with torch.cuda.stream(s_in):
+            for (hk, hv), (dk, dv) in zip(host_in, dev_in[b]):
+                dk.copy_(hk, non_blocking=True)
+                dv.copy_(hv, non_blocking=True)
+        in_ready[b].record(s_in)
+
+    def merge(i):
+        b = i % 2
+        stream.wait_event(in_ready[b])
+        stream.wait_event(out_free[b])
+        one_merge(inputs=dev_desc[b], out=dev_out[b])
+        in_free[b].record(stream)
+        out_ready[b].record(stream)
+
+    def copy_out(i):
+        b = i % 2
+        s_out.wait_event(out_ready[b])
+        with torch.cuda.stream(s_out):
+            host_out[0].copy_(dev_out[b][0], non_blocking=True)
+            host_out[1].copy_(dev_out[b][1], non_blocking=True)
+        out_free[b].record(s_out)
+
+    def pipelined(n_steps):
+        for e in in_free + out_free:
+            e.record(stream)
+        s_in.wait_stream(stream)
+        s_out.wait_stream(stream)
+        copy_in(0)
+        for i in range(n_steps):
+            if i + 1 < n_steps:
+                copy_in(i + 1)      # enqueued before merge(i) blocks on its ingest
+            merge(i)
+            copy_out(i)
+        stream.wait_stream(s_out)
+        stream.wait_stream(s_in)
+
+    def serial_step():
+        for (hk, hv), (dk, dv) in zip(host_in, dev_in[0]):
             dk.copy_(hk, non_blocking=True)
             dv.copy_(hv, non_blocking=True)
-        one_merge(inputs=dev_desc)
+        one_merge(inputs=dev_desc[0])
         host_out[0].copy_(k_out, non_blocking=True)
         host_out[1].copy_(v_out, non_blocking=True)
 
-    e2e_step()
-    torch.cuda.synchronize(dev)
-    if world > 1:
-        dist.barrier()
-    e0, e1 = ev(), ev()
-    e0.record(stream)
-    for _ in range(e2e_steps):
-        e2e_step()
-    e1.record(stream)
-    torch.cuda.synchronize(dev)
-    e2e_ms = e0.elapsed_time(e1)
-    e2e_ms = max_over_ranks(e2e_ms, dev)
-    if world > 1:
-        dist.barrier()
+    def timed_e2e(run):
+        torch.cuda.synchronize(dev)
+        if world > 1:
+            dist.barrier()
+        e0, e1 = ev(), ev()
+        e0.record(stream)
+        run()
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        ms = max_over_ranks(e0.elapsed_time(e1), dev)
+        if world > 1:
+            dist.barrier()
+        return ms
+
+    pipelined(2)                                   # warm-up
+    e2e_ms = timed_e2e(lambda: pipelined(e2e_steps))
+    # the host copy of the last step's result is that step's merged cache
+    assert torch.equal(host_out[0][:, :, -8:].view(torch.int16).to(dev),
+                       dev_out[(e2e_steps - 1) % 2][0][:, :, -8:].view(torch.int16))
+    serial_step()
+    e2e_serial_ms = timed_e2e(lambda: [serial_step() for _ in range(e2e_steps)])
 
     if rank == 0:
         peak, peak_src = hbm_peak()
@@ -596,8 +651,12 @@ def main():
             "kernel_ms_per_step": per_step,
             "dominant_kernel": dominant,
             "e2e": {"value": whole_job_rate(world, e2e_steps, e2e_ms), "unit": UNIT,
-                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                    "timing": "CUDA events around the steps; copies and merge in order on one stream"},
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e2e_steps,
+                    "timing": "CUDA events around all steps; step i+1's inputs copy in and step "
+                              "i-1's merged cache copies out while step i merges (double-buffered "
+                              "on the device, three streams)",
+                    "serial": {"value": whole_job_rate(world, e2e_steps, e2e_serial_ms),
+                               "timing": "copy in, merge, copy out, in order on one stream"}},
             "gpu_launches": int(round(launches_per_step * args.steps)),
             "clocks": clocks.summary(),
         }
