@@ -185,40 +185,70 @@ def sm_max_mhz():
 
 def oracle_sample_seconds(layers=1, w=None):
     """The oracle as it stands on a bounded sample of the workload: the first `layers`
-    layers of each of the 4 fragments (T = 4096), full ingest (id + norm key), union
-    and render; returns (seconds, bytes of that sample's fragments)."""
+    layers of each of the 4 fragments (T = 4096). Returns the seconds of one full merge
+    estimated from it: the content address and the render cost the same per layer, so
+    their sample times are scaled by num_layers / layers; the routing-layer norm key
+    covers one layer of each fragment in a full merge as in the sample, so its time is
+    taken as it is."""
     import numpy as np
     import oracle
     import synthetic
+    from oracle.content_address import fragment_id
+    from oracle.norm import norm_key
     w = w or synthetic.WORKLOADS[WORKLOAD]
     specs = synthetic.fragment_specs(w)
     frags = [synthetic.make_fragment_bits(s, layers, w.num_kv_heads, w.head_dim) for s in specs]
-    t0 = time.perf_counter()
+    t_layers = t_norm = 0.0
     A = oracle.FragmentSet()
     B = oracle.FragmentSet()
     for i, (K, V) in enumerate(frags):
-        f = oracle.make_fragment(K, V, routing_layer=layers // 2)
+        t0 = time.perf_counter()
+        fid = fragment_id(K, V)
+        t1 = time.perf_counter()
+        Q = norm_key(K, layers // 2)
+        t2 = time.perf_counter()
+        f = oracle.Fragment(K, V, fid, Q)
         if i < 2:
             A = oracle.ingest(A, f)
         else:
             B = oracle.ingest(B, f)
+        t3 = time.perf_counter()
+        t_layers += (t1 - t0) + (t3 - t2)
+        t_norm += t2 - t1
+    t0 = time.perf_counter()
     S = oracle.union(A, B)
     K_out, V_out, _ = oracle.render(S, synthetic.ROPE_THETA)
-    dt = time.perf_counter() - t0
-    nbytes = sum(K.nbytes + V.nbytes for K, V in frags)
+    t_layers += time.perf_counter() - t0
     assert K_out.shape[2] == sum(s.seq_len for s in specs)
-    return dt, nbytes
+    return t_layers * w.num_layers / layers + t_norm, t_layers + t_norm
+
+
+def host_cpu():
+    """Model name of the host CPU (lscpu) and the number of cores the OS reports."""
+    model = None
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().lower().startswith("model name"):
+                model = line.split(":", 1)[1].strip()
+                break
+    except Exception:
+        pass
+    return {"model": model, "os_cpu_count": os.cpu_count()}
 
 
 def cpu_baseline_entry(layers=24):
     import synthetic
     w = synthetic.WORKLOADS[WORKLOAD]
-    dt, _ = oracle_sample_seconds(layers, w)
-    per_merge = dt * w.num_layers / layers
+    per_merge, dt = oracle_sample_seconds(layers, w)
+    merged = sum(s.seq_len for s in synthetic.fragment_specs(w))
     return {"value": 1.0 / per_merge, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "render_bytes_gbs": 2 * merged * w.bytes_per_token / per_merge / 1e9,
+            "host": host_cpu(),
             "sample": f"one merge restricted to the first {layers} of {w.num_layers} layers "
                       f"(4 fragments x 4096 tokens; ingest + union + render), timed once "
-                      f"({dt:.2f} s) and scaled by {w.num_layers}/{layers} to a full merge; "
+                      f"({dt:.2f} s); content address and render scaled by {w.num_layers}/{layers}, "
+                      f"the routing-layer norm key (one layer per fragment either way) unscaled; "
                       f"single thread (numpy fp64 + hashlib)",
             "seconds_per_merge": per_merge}
 
@@ -235,8 +265,7 @@ def run_reference(args):
         oracle_sample_seconds(layers, w)
     total = 0.0
     for _ in range(args.steps):
-        dt, _ = oracle_sample_seconds(layers, w)
-        total += dt * w.num_layers / layers
+        total += oracle_sample_seconds(layers, w)[0]
     value = args.steps / total
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
@@ -245,9 +274,11 @@ def run_reference(args):
         "scaling": "weak", "vs_baseline": None, "dtype": "u16 bits / f64", "data": "synthetic",
         "config": workload_config(w),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "host": host_cpu(),
                          "sample": f"each step: one merge restricted to the first {layers} of "
-                                   f"{w.num_layers} layers, scaled by {w.num_layers} to a full "
-                                   f"merge; single thread"},
+                                   f"{w.num_layers} layers; content address and render scaled by "
+                                   f"{w.num_layers}, the routing-layer norm key unscaled; single "
+                                   f"thread"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
