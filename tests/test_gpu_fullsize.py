@@ -1,5 +1,6 @@
 """GPU parity at the benchmark's full sizes, in the launch configuration bench.py
-times (two replicas batch-ingest half the fragments each, union, render).
+times (one cm_ingest_many call feeds two replicas half the fragments each, union,
+render), and at the full sizes of the other workloads.
 
 The oracle computes every content address and norm key in full (hashlib over all
 bytes) and the render on sampled (slot, layer, head) planes: each output plane
@@ -7,6 +8,8 @@ depends only on its source plane and the slot's offset, so a sampled plane is
 checked exactly as a full render would check it. V planes are compared bit for
 bit, K planes within 1 bf16 ulp with the non-exact count asserted to be 0.
 """
+import itertools
+
 import numpy as np
 import pytest
 import torch
@@ -142,6 +145,53 @@ def test_arity_batch_matches_sequential_ingest_and_oracle(ctx):
     _check_sampled_planes(frags, order, outs[0][0], outs[0][1], layers=[0, 14, 27], heads=[0, 5])
     S1.close()
     S2.close()
+
+
+def test_arity_all_120_orders_render_identically_at_full_length(ctx):
+    # the arity configuration at its real lengths (T ~ U{256..2048}): every order of the
+    # five distinct fragments, as unions of single-fragment sets, renders the same bytes;
+    # so do 20 random orders of the eight deliveries (duplicates included)
+    w = synthetic.WORKLOADS["q17_arity"]
+    specs = synthetic.fragment_specs(w)
+    frags = [synthetic.make_fragment_torch(sp, w.num_layers, w.num_kv_heads, w.head_dim, "cuda:0")
+             for sp in specs]
+    total = sum(sp.seq_len for sp in specs)
+    singles = []
+    for K, V in frags:
+        S = cm.FragmentSet(ctx)
+        S.ingest(K, V)
+        singles.append(S)
+    k0, v0 = empty_out(w.num_layers, w.num_kv_heads, total, w.head_dim)
+    ref = None
+    for perm in itertools.permutations(range(5)):
+        U = cm.FragmentSet(ctx)
+        for i in perm:
+            U.union(singles[i])
+        n, order_ids = U.render(k0, v0)
+        if ref is None:
+            ref = (k0.clone(), v0.clone(), order_ids)
+        else:
+            assert order_ids == ref[2]
+            assert torch.equal(k0.view(torch.int16), ref[0].view(torch.int16))
+            assert torch.equal(v0.view(torch.int16), ref[1].view(torch.int16))
+        U.close()
+    sched = synthetic.delivery_schedule(w)
+    msgs = [(frags[i][0].clone(), frags[i][1].clone()) for i in sched]
+    rng = np.random.default_rng(120)
+    for _ in range(20):
+        S = cm.FragmentSet(ctx)
+        res = S.ingest_batch([msgs[j] for j in rng.permutation(len(msgs))])
+        assert sum(a for _, a in res) == 3 and len(S) == 5
+        S.render(k0, v0)
+        assert torch.equal(k0.view(torch.int16), ref[0].view(torch.int16))
+        assert torch.equal(v0.view(torch.int16), ref[1].view(torch.int16))
+        S.close()
+    keys = _oracle_keys(frags, w.num_layers // 2)
+    order = _oracle_order(keys, [sp.seq_len for sp in specs])
+    assert ref[2] == [keys[i][0] for i in order]
+    _check_sampled_planes(frags, order, ref[0], ref[1], layers=[0, 14, 27], heads=[0, 7])
+    for S in singles:
+        S.close()
 
 
 def test_kernel_timing_counts_every_launch(ctx):
