@@ -506,7 +506,7 @@ def main():
     # paged render of the same merge into per-layer block pools [L][blocks][16][H][d] through a
     # shuffled block table (timed apart from the steps, same algorithmic bytes)
     paged_ms = None
-    if args.workload == WORKLOAD:
+    if args.workload in (WORKLOAD, "q4b_t512"):
         import numpy as np
         bs = 16
         nblk = -(-total_T // bs)

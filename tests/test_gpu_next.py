@@ -125,8 +125,13 @@ def _paged_check(ctx, frags, block_size, layout, seed):
     S.close()
 
 
+# block sizes: powers of two no smaller than an item's rows (one table lookup per block an
+# item touches: 16 at d = 128, 32 at d = 64 where the rows equal the block, 128 at d = 256)
+# and the per-row lookups otherwise (12: not a power of two; 1 and 64 at d = 16: an item
+# of 128 rows spans several blocks)
 @pytest.mark.parametrize("layout,block_size,d", [("per_layer", 16, 128), ("block_major", 12, 64),
-                                                 ("per_layer", 1, 16), ("block_major", 128, 256)])
+                                                 ("per_layer", 1, 16), ("block_major", 128, 256),
+                                                 ("per_layer", 32, 64), ("block_major", 64, 16)])
 def test_paged_render_matches_contiguous_render(ctx, layout, block_size, d):
     L, H = 3, 2
     frags = [_frag(L, H, T, d, 0.5 + 0.4 * i, 10 + i) for i, T in enumerate([37, 200, 5, 129])]
