@@ -480,6 +480,8 @@ def main():
     for _ in range(args.warmup):
         one_merge()
     torch.cuda.synchronize(dev)
+    # register-only integer-ALU rates of this GPU (the ceiling of the content address)
+    xor3_tops, compress_tops = cm.cm_measure_int_alu(local_rank)
 
     step_timers = [{"ingest": (ev(), ev()), "render": (ev(), ev())} for _ in range(args.steps)]
     start, end = ev(), ev()
@@ -650,6 +652,10 @@ def main():
             # against every integer lane of an SM (ALU and FMA pipes, 128 per clock); only
             # the ALU pipe's 64 can take the xors and rotates, which is what binds
             "frac_of_128_int_lanes": hash_tops / (alu_peak * 128 / ALU_OPS_PER_CLK_PER_SM),
+            # measured on this GPU before the timed steps (cm_measure_int_alu): three-input
+            # xors alone, and the same compression function on register data alone
+            "measured_xor3_tops": xor3_tops, "measured_compress_tops": compress_tops,
+            "frac_of_measured_compress": hash_tops / compress_tops,
         }
         per_step = {"leaf_hash": ktimes["leaf_hash_ms"] / args.steps,
                     "inner_hash": ktimes["inner_hash_ms"] / args.steps,

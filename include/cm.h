@@ -329,6 +329,16 @@ cm_status cm_context_set_timing(cm_context *ctx, int32_t enable);
  * context's totals and report the totals; reset != 0 zeroes them afterwards. */
 cm_status cm_context_kernel_times(cm_context *ctx, cm_kernel_times *out, int32_t reset);
 
+/* Integer-ALU throughput of `device`, measured with two register-only kernels (a
+ * profiling aid for the roofline of the content-address kernels; the paper has no
+ * counterpart): chains of three-input xors (one integer-ALU instruction each), and the
+ * BLAKE2s compression function of the content address applied to register data, counted
+ * as 808 integer-ALU operations per 64-byte block (10 rounds x 8 G x 10 + 8). Both are
+ * reported in 10^12 operations per second, best of three timed launches of four full
+ * waves each. Synchronous; allocates and frees a small device buffer; takes a few ms.
+ * The calling thread's current device is restored on return. */
+cm_status cm_measure_int_alu(int32_t device, double *xor3_tops, double *compress_tops);
+
 /* Static name of a status code. */
 const char *cm_status_string(cm_status status);
 

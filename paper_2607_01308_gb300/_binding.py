@@ -101,6 +101,7 @@ _SIGS = {
                                   _c.POINTER(_c.c_int64)]),
     "cm_set_contains": (_c.c_int, [_P, _c.POINTER(cm_id), _c.c_int64, _c.POINTER(_c.c_uint8)]),
     "cm_set_leq": (_c.c_int, [_P, _P, _c.POINTER(_c.c_int32)]),
+    "cm_measure_int_alu": (_c.c_int, [_c.c_int32, _c.POINTER(_c.c_double), _c.POINTER(_c.c_double)]),
     "cm_context_set_timing": (_c.c_int, [_P, _c.c_int32]),
     "cm_context_kernel_times": (_c.c_int, [_P, _c.POINTER(cm_kernel_times), _c.c_int32]),
     "cm_union": (_c.c_int, [_P, _P]),
@@ -253,6 +254,13 @@ def cm_set_leq(a: int, b: int) -> bool:
     out = ctypes.c_int32()
     _check(lib.cm_set_leq(a, b, ctypes.byref(out)))
     return bool(out.value)
+
+
+def cm_measure_int_alu(device: int = 0) -> Tuple[float, float]:
+    """(xor3_tops, compress_tops): register-only integer-ALU throughput of the device."""
+    x, c = ctypes.c_double(), ctypes.c_double()
+    _check(lib.cm_measure_int_alu(device, ctypes.byref(x), ctypes.byref(c)))
+    return x.value, c.value
 
 
 def cm_context_set_timing(ctx: int, enable: bool) -> None:

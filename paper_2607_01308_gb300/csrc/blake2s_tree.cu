@@ -503,3 +503,112 @@ extern "C" cm_status cm_fragment_id_static(const cm_fragment *frag, int32_t rout
         return report_error(CM_ERR_OOM, "host allocation failed");
     }
 }
+
+// ---------------------------------------------------------------- integer-ALU throughput
+//
+// Register-only kernels that measure the ceiling of the content-address kernels on the
+// current GPU (a profiling aid for their roofline): chains of three-input xors, one
+// integer-ALU instruction each, and the compression function above applied to register
+// data with no memory traffic.
+
+namespace cm {
+namespace {
+
+__global__ void __launch_bounds__(kLeafThreads)
+xor3_probe_kernel(uint32_t *out, int iters) {
+    const uint32_t tid = blockIdx.x * blockDim.x + threadIdx.x;
+    uint32_t a[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) a[i] = tid * (2u * i + 3u);
+    for (int it = 0; it < iters; ++it) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) a[i] = a[i] ^ a[(i + 1) & 7] ^ a[(i + 3) & 7];
+    }
+    uint32_t x = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) x ^= a[i];
+    out[tid] = x;
+}
+
+__global__ void __launch_bounds__(kLeafThreads)
+compress_probe_kernel(uint32_t *out, int blocks) {
+    const uint32_t tid = blockIdx.x * blockDim.x + threadIdx.x;
+    uint32_t h[8], m[16];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) h[i] = tid * 2654435761u + (uint32_t)i;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) m[i] = tid ^ ((uint32_t)i * 0x9E3779B9u);
+    for (int b = 0; b < blocks; ++b) {
+        compress(h, m, (uint64_t)(b + 1) * 64, false, false);
+        m[0] ^= h[0];
+        m[7] ^= h[3];
+        m[11] ^= h[6];
+    }
+    out[tid] = h[0] ^ h[1] ^ h[2] ^ h[3] ^ h[4] ^ h[5] ^ h[6] ^ h[7];
+}
+
+}  // namespace
+}  // namespace cm
+
+extern "C" cm_status cm_measure_int_alu(int32_t device, double *xor3_tops, double *compress_tops) {
+    using namespace cm;
+    if (!xor3_tops || !compress_tops)
+        return report_error(CM_ERR_INVALID_ARG, "xor3_tops and compress_tops are required");
+    int prev = 0;
+    cudaError_t e = cudaGetDevice(&prev);
+    if (e != cudaSuccess) return report_error(CM_ERR_CUDA, cudaGetErrorString(e));
+    e = cudaSetDevice(device);
+    if (e != cudaSuccess) return report_error(CM_ERR_CUDA, cudaGetErrorString(e));
+    cm_status st = CM_OK;
+    uint32_t *out = nullptr;
+    cudaEvent_t e0 = nullptr, e1 = nullptr;
+    auto check = [&](cudaError_t err) {
+        if (err != cudaSuccess && st == CM_OK) st = report_error(CM_ERR_CUDA, cudaGetErrorString(err));
+        return err == cudaSuccess;
+    };
+    int sms = 0, per_sm_x = 0, per_sm_c = 0;
+    if (check(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device)) &&
+        check(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm_x, xor3_probe_kernel,
+                                                            kLeafThreads, 0)) &&
+        check(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm_c, compress_probe_kernel,
+                                                            kLeafThreads, 0))) {
+        // four full waves of each kernel
+        const int grid_x = 4 * sms * per_sm_x, grid_c = 4 * sms * per_sm_c;
+        const int grid = grid_x > grid_c ? grid_x : grid_c;
+        const int xor_iters = 4096, comp_blocks = 64;
+        if (check(cudaMalloc(&out, (size_t)grid * kLeafThreads * sizeof(uint32_t))) &&
+            check(cudaEventCreate(&e0)) && check(cudaEventCreate(&e1))) {
+            auto best_ms = [&](auto launch) {
+                float best = 0.0f;
+                for (int rep = 0; rep < 4 && st == CM_OK; ++rep) {   // rep 0 warms up
+                    check(cudaEventRecord(e0));
+                    launch();
+                    check(cudaGetLastError());
+                    check(cudaEventRecord(e1));
+                    float ms = 0.0f;
+                    if (check(cudaEventSynchronize(e1)) && check(cudaEventElapsedTime(&ms, e0, e1)) &&
+                        rep > 0 && (best == 0.0f || ms < best))
+                        best = ms;
+                }
+                return (double)best;
+            };
+            const double ms_x = best_ms([&] {
+                xor3_probe_kernel<<<grid_x, kLeafThreads>>>(out, xor_iters);
+            });
+            const double ms_c = best_ms([&] {
+                compress_probe_kernel<<<grid_c, kLeafThreads>>>(out, comp_blocks);
+            });
+            if (st == CM_OK) {
+                const double ops_x = (double)grid_x * kLeafThreads * xor_iters * 8;
+                const double ops_c = (double)grid_c * kLeafThreads * comp_blocks * 808;
+                *xor3_tops = ops_x / (ms_x * 1e-3) / 1e12;
+                *compress_tops = ops_c / (ms_c * 1e-3) / 1e12;
+            }
+        }
+    }
+    if (e0) cudaEventDestroy(e0);
+    if (e1) cudaEventDestroy(e1);
+    if (out) cudaFree(out);
+    cudaSetDevice(prev);
+    return st;
+}

@@ -14,6 +14,7 @@
 #include <array>
 #include <cmath>
 #include <cstdio>
+#include <cstddef>
 #include <cstring>
 #include <map>
 #include <memory>
@@ -141,6 +142,8 @@ struct cm_context {
     // RoPE frequencies theta^(-2j/d), j < d/2, for the last head_dim rendered
     std::vector<double> omega;
     int32_t omega_d = 0;
+    // launch parameters of the render kernel (about 31 KB), reused by every launch
+    std::unique_ptr<cm::RenderParams> render_params;
 };
 
 struct cm_set {
@@ -441,10 +444,14 @@ cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t 
         for (int j = 0; j < half; ++j) ctx->omega[(size_t)j] = std::pow(ctx->theta, -(2.0 * j) / d);
         ctx->omega_d = d;
     }
-    std::unique_ptr<cm::RenderParams> p(new cm::RenderParams);
+    if (!ctx->render_params) ctx->render_params.reset(new cm::RenderParams);
+    cm::RenderParams *p = ctx->render_params.get();
     for (size_t g0 = 0; g0 < slots.size(); g0 += (size_t)max_group) {
         const size_t n = std::min(slots.size() - g0, (size_t)max_group);
-        std::memset(p.get(), 0, sizeof(cm::RenderParams));
+        // the kernel reads the header, slot[0, n) and the (cos, sin) pairs of those slots
+        // that rotate, all written below; the rest of the block keeps older values
+        std::memset(p, 0, offsetof(cm::RenderParams, slot));
+        std::memset(p->slot, 0, n * sizeof(cm::RenderSlot));
         p->num_layers = L;
         p->num_heads = H;
         p->head_dim = d;
@@ -535,8 +542,18 @@ std::vector<std::shared_ptr<const Record>> canonical_order(const cm_set *set) {
     std::vector<Keyed> keyed;
     keyed.reserve(recs.size());
     for (auto &r : recs) {
+        // each Q[t] is at most H (2^44 - 1): when H T* (2^44 - 1) < 2^64 the tail sum
+        // cannot wrap in 64 bits, and a plain 64-bit sum (which vectorises) is exact
+        const uint64_t *q = r->Q.data() + (r->T - t_star);
         unsigned __int128 S = 0;
-        for (int64_t t = r->T - t_star; t < r->T; ++t) S += r->Q[(size_t)t];
+        if ((unsigned __int128)r->H * (uint64_t)t_star * ((1ull << 44) - 1) <
+            ((unsigned __int128)1 << 64)) {
+            uint64_t s64 = 0;
+            for (int64_t t = 0; t < t_star; ++t) s64 += q[t];
+            S = s64;
+        } else {
+            for (int64_t t = 0; t < t_star; ++t) S += q[t];
+        }
         keyed.push_back({S, key_of(r->id), r});
     }
     std::sort(keyed.begin(), keyed.end(), [](const Keyed &a, const Keyed &b) {

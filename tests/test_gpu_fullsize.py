@@ -194,6 +194,15 @@ def test_arity_all_120_orders_render_identically_at_full_length(ctx):
         S.close()
 
 
+def test_integer_alu_probe_is_plausible(ctx):
+    # the xor chains run on the integer ALU pipe (64 lanes per SM per clock on this
+    # part); the compression rate cannot exceed it by more than timing noise
+    xor3, comp = cm.cm_measure_int_alu(0)
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    assert sms * 64 * 0.5e9 / 1e12 < xor3 < sms * 64 * 3.0e9 / 1e12
+    assert 0.5 * xor3 < comp < 1.05 * xor3
+
+
 def test_kernel_timing_counts_every_launch(ctx):
     w, L, H, d = None, 4, 2, 64
     g = torch.Generator(device="cuda:0").manual_seed(5)
