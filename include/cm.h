@@ -311,6 +311,17 @@ cm_status cm_bagmerge(cm_context *ctx, const cm_fragment *frags, int32_t n, void
  * the output of the affected render is incomplete. CM_OK otherwise. */
 cm_status cm_context_check(cm_context *ctx, cm_stream_t stream);
 
+/* Width of the render kernel's CTAs for every later render launched from ctx (a
+ * scheduling aid; the paper has no counterpart). The render is one persistent CTA per
+ * SM. warps = 16 (the default) gives it the whole register file of each SM: the fastest
+ * render when it runs alone. warps = 8 leaves half of each SM's registers free, so that
+ * the content-address kernels of a later cm_ingest* call on another stream run beside
+ * the render instead of after it (the render is bound by HBM, hashing by the integer
+ * ALU): a serving loop that renders one group of requests while hashing the next gains
+ * throughput, at some cost to a render that runs alone. The rendered bytes are the same.
+ * CM_ERR_INVALID_ARG for any other value. */
+cm_status cm_context_set_render_warps(cm_context *ctx, int32_t warps);
+
 /* Device time per kernel, accumulated while timing is on (a profiling aid). */
 typedef struct cm_kernel_times {
     double leaf_hash_ms;          /* content address, level 0 (one launch per fragment) */

@@ -144,6 +144,7 @@ struct cm_context {
     int32_t omega_d = 0;
     // launch parameters of the render kernel (about 31 KB), reused by every launch
     std::unique_ptr<cm::RenderParams> render_params;
+    int32_t render_warps = 16;   // warps per render CTA (cm_context_set_render_warps)
 };
 
 struct cm_set {
@@ -506,7 +507,7 @@ cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t 
         }
         const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(chunk, ctx->num_sms));
         CM_CUDA_TRY(timed_launch(ctx, kTimeRender, stream,
-                                 [&] { return cm::launch_render(*p, grid, stream); }),
+                                 [&] { return cm::launch_render(*p, grid, ctx->render_warps, stream); }),
                     "render launch");
     }
     return CM_OK;
@@ -803,6 +804,14 @@ cm_status cm_ingest_many(cm_set *const *sets, const cm_fragment *frags, int32_t 
     });
 }
 
+
+cm_status cm_context_set_render_warps(cm_context *ctx, int32_t warps) {
+    if (!ctx) return fail(CM_ERR_INVALID_ARG, "context is NULL");
+    if (warps != 8 && warps != 16) return fail(CM_ERR_INVALID_ARG, "render warps must be 8 or 16");
+    std::lock_guard<std::mutex> lock(ctx->mu);
+    ctx->render_warps = warps;
+    return CM_OK;
+}
 
 cm_status cm_context_set_timing(cm_context *ctx, int32_t enable) {
     if (!ctx) return fail(CM_ERR_INVALID_ARG, "context is NULL");

@@ -123,9 +123,9 @@ struct RenderParams {
     double cs[2 * kMaxTablePairs];   // (cos a, sin a) of a = s * theta^(-2j/d), interleaved
 };
 
-// One CTA per SM; render_prepare() once per device before the first launch.
-cudaError_t launch_render(const RenderParams &p, int grid, cudaStream_t stream);
-int render_threads_per_block();
+// One CTA of `warps` warps (16, or 8 to leave half of each SM's registers to kernels of
+// other streams) per SM; render_prepare() once per device before the first launch.
+cudaError_t launch_render(const RenderParams &p, int grid, int warps, cudaStream_t stream);
 cudaError_t render_prepare();
 
 }  // namespace cm

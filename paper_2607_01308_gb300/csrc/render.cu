@@ -33,7 +33,6 @@
 namespace cm {
 namespace {
 
-constexpr int kThreads = 512;
 static_assert(sizeof(RenderParams) <= 32764, "render parameters exceed the kernel parameter limit");
 
 __device__ __forceinline__ void st_stream(uint4 *p, const uint4 &v) { __stcs(p, v); }
@@ -231,11 +230,12 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-constexpr int kWarps = kThreads / 32;
 constexpr int kStages = 3;                          // per warp
 constexpr uint32_t kItemBytes = 4096;               // one work item = one stage
 constexpr size_t kTableBytes = sizeof(float4) * kMaxTablePairs;
-constexpr size_t kDynSmem = (size_t)kWarps * kStages * kItemBytes + kTableBytes;
+// Dynamic shared memory of a CTA of kW warps: the warps' stages, then the (cos, sin) table.
+template <int kW>
+constexpr size_t dyn_smem() { return (size_t)kW * kStages * kItemBytes + kTableBytes; }
 static_assert(kChunkBytes == (int)kItemBytes, "host and kernel disagree on the work item size");
 
 // One work item: up to kItemBytes of one source plane and where it goes.
@@ -377,7 +377,9 @@ __device__ __forceinline__ float2 split16(double c) {
     return make_float2(c1, __double2float_rn(c - (double)c1));
 }
 
-// Persistent kernel, one CTA of kWarps warps per SM; every warp runs its own
+// Persistent kernel, one CTA of kW warps per SM (16: the whole register file at 128
+// registers a thread; 8: half of it, leaving room for kernels of another stream on
+// the same SMs); every warp runs its own
 // pipeline over its own items, with no block-wide barrier after set-up. Items come
 // in (K, V) pairs of the same (slot, layer, head, row chunk); a warp takes pairs
 // warp id + m * total warps and does the K item, then the V item, so rotation work
@@ -388,13 +390,14 @@ __device__ __forceinline__ float2 split16(double c) {
 // place comes from the block table), and lane 0 refills the stage with the warp's
 // next item. Every wait is bounded: on timeout the warp records an error, waits
 // (bounded) for its own copies in flight and returns.
-template <bool kPaged>
-__global__ void __launch_bounds__(kThreads, 1)
+template <bool kPaged, int kW>
+__global__ void __launch_bounds__(kW * 32, 16 / kW)
 render_kernel(const __grid_constant__ RenderParams p) {
+    constexpr int kThreads = kW * 32;
     extern __shared__ __align__(128) uint8_t smem[];
-    __shared__ __align__(8) uint64_t full[kWarps][kStages];
-    __shared__ Item items[kWarps][kStages];
-    float4 *tab = reinterpret_cast<float4 *>(smem + (size_t)kWarps * kStages * kItemBytes);
+    __shared__ __align__(8) uint64_t full[kW][kStages];
+    __shared__ Item items[kW][kStages];
+    float4 *tab = reinterpret_cast<float4 *>(smem + (size_t)kW * kStages * kItemBytes);
 
     const int half = p.head_dim >> 1;
     const int n_table = p.num_slots * half;
@@ -409,8 +412,8 @@ render_kernel(const __grid_constant__ RenderParams p) {
     }
     __syncthreads();
 
-    const uint32_t first = blockIdx.x * kWarps + warp;
-    const uint32_t stride = gridDim.x * kWarps;
+    const uint32_t first = blockIdx.x * kW + warp;
+    const uint32_t stride = gridDim.x * kW;
     const uint32_t npairs = p.total_chunks / 2;
     const uint32_t n = npairs > first ? 2 * ((npairs - first + stride - 1) / stride) : 0;
     const int lane_v = lane & ((p.head_dim >> 4) - 1);
@@ -457,25 +460,34 @@ render_kernel(const __grid_constant__ RenderParams p) {
     }
 }
 
-}  // namespace
-
-int render_threads_per_block() { return kThreads; }
-
-cudaError_t render_prepare() {
-    cudaError_t e = cudaFuncSetAttribute(render_kernel<false>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kDynSmem);
-    if (e != cudaSuccess) return e;
-    return cudaFuncSetAttribute(render_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)kDynSmem);
+template <bool kPaged, int kW>
+cudaError_t set_smem_attribute() {
+    return cudaFuncSetAttribute(render_kernel<kPaged, kW>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn_smem<kW>());
 }
 
-cudaError_t launch_render(const RenderParams &p, int grid, cudaStream_t stream) {
-    if (p.total_chunks == 0) return cudaSuccess;
+template <int kW>
+cudaError_t launch_width(const RenderParams &p, int grid, cudaStream_t stream) {
     if (p.paged)
-        render_kernel<true><<<grid, kThreads, kDynSmem, stream>>>(p);
+        render_kernel<true, kW><<<grid, kW * 32, dyn_smem<kW>(), stream>>>(p);
     else
-        render_kernel<false><<<grid, kThreads, kDynSmem, stream>>>(p);
+        render_kernel<false, kW><<<grid, kW * 32, dyn_smem<kW>(), stream>>>(p);
     return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t render_prepare() {
+    cudaError_t e = set_smem_attribute<false, 16>();
+    if (e == cudaSuccess) e = set_smem_attribute<true, 16>();
+    if (e == cudaSuccess) e = set_smem_attribute<false, 8>();
+    if (e == cudaSuccess) e = set_smem_attribute<true, 8>();
+    return e;
+}
+
+cudaError_t launch_render(const RenderParams &p, int grid, int warps, cudaStream_t stream) {
+    if (p.total_chunks == 0) return cudaSuccess;
+    return warps == 8 ? launch_width<8>(p, grid, stream) : launch_width<16>(p, grid, stream);
 }
 
 }  // namespace cm

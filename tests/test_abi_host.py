@@ -32,7 +32,8 @@ def test_header_declares_the_documented_calls():
             "cm_last_error_message", "cm_context_check", "cm_ingest_batch",
             "cm_context_set_timing", "cm_context_kernel_times", "cm_fragment_id_static",
             "cm_render_incremental", "cm_render_paged", "cm_ingest_many", "cm_render_many",
-            "cm_set_contains", "cm_set_leq", "cm_measure_int_alu"}
+            "cm_set_contains", "cm_set_leq", "cm_measure_int_alu",
+            "cm_context_set_render_warps"}
     assert want <= set(_declared_functions())
 
 

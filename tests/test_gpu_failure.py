@@ -17,10 +17,12 @@ pytestmark = pytest.mark.gpu
 cm = pytest.importorskip("paper_2607_01308_gb300")
 
 
-def test_withheld_copy_times_out_and_the_context_recovers():
+@pytest.mark.parametrize("warps", [16, 8])
+def test_withheld_copy_times_out_and_the_context_recovers(warps):
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
     ctx = cm.Context(0, THETA)
+    cm.cm_context_set_render_warps(ctx.handle, warps)
     w, frags, _ = gpu_fragments("tiny")
     S = cm.FragmentSet(ctx)
     S.ingest_batch(frags)

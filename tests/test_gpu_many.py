@@ -231,3 +231,62 @@ def test_replica_exchange_by_ids(ctx):
     assert A.contains([]) == []
     for S in (A, B, empty):
         S.close()
+
+
+def test_eight_warp_render_writes_the_same_bytes(ctx):
+    # cm_context_set_render_warps(8) halves the render CTA; every layout must come out
+    # byte-identical to the default 16-warp render (and so to the oracle)
+    ctx8 = cm.Context(0, THETA)
+    cm.cm_context_set_render_warps(ctx8.handle, 8)
+    for bad in (0, 4, 12, 32):
+        with pytest.raises(cm.CMError) as e:
+            cm.cm_context_set_render_warps(ctx8.handle, bad)
+        assert e.value.status == cm.Status.ERR_INVALID_ARG
+    for d in (16, 64, 128, 512):
+        L, H = 3, 2
+        frags = _fragments(8000 + d, [1, 129, 70, 600], L, H, d)
+        outs = []
+        for c in (ctx, ctx8):
+            S = cm.FragmentSet(c)
+            S.ingest_batch(frags)
+            k, v = empty_out(L, H, S.seq_len() + 3, d, fill=CANARY)
+            S.render(k, v)
+            torch.cuda.synchronize()
+            outs.append((k, v))
+            S.close()
+        assert torch.equal(outs[0][0].view(torch.int16), outs[1][0].view(torch.int16))
+        assert torch.equal(outs[0][1].view(torch.int16), outs[1][1].view(torch.int16))
+        if d == 128:
+            _check_against_oracle(frags, outs[1][0], outs[1][1], sum([1, 129, 70, 600]))
+    # paged output and BagMerge through the 8-warp kernel
+    L, H, d, bs = 2, 2, 64, 16
+    frags = _fragments(8100, [37, 200, 5], L, H, d)
+    total = sum(f[0].shape[2] for f in frags)
+    nblk = -(-total // bs)
+    table = torch.randperm(nblk, generator=torch.Generator().manual_seed(1)).to(torch.int32).cuda()
+    pools = []
+    for c in (ctx, ctx8):
+        S = cm.FragmentSet(c)
+        S.ingest_batch(frags)
+        kp = torch.zeros((L, nblk, bs, H, d), dtype=torch.bfloat16, device="cuda:0")
+        vp = torch.zeros_like(kp)
+        cache = cm.cm_paged_cache(kp.data_ptr(), vp.data_ptr(), table.data_ptr(), nblk, bs,
+                                  stride_block=bs * H * d, stride_layer=nblk * bs * H * d,
+                                  stride_head=d, stride_token=H * d)
+        cm.cm_render_paged(S.handle, cache)
+        torch.cuda.synchronize()
+        pools.append((kp, vp))
+        S.close()
+    assert torch.equal(pools[0][0].view(torch.int16), pools[1][0].view(torch.int16))
+    assert torch.equal(pools[0][1].view(torch.int16), pools[1][1].view(torch.int16))
+    seq = frags + frags[:1]
+    n_tok = sum(f[0].shape[2] for f in seq)
+    bag = []
+    for c in (ctx, ctx8):
+        kb, vb = empty_out(L, H, n_tok, d)
+        c.bagmerge(seq, kb, vb)
+        torch.cuda.synchronize()
+        bag.append((kb, vb))
+    assert torch.equal(bag[0][0].view(torch.int16), bag[1][0].view(torch.int16))
+    assert torch.equal(bag[0][1].view(torch.int16), bag[1][1].view(torch.int16))
+    ctx8.close()
