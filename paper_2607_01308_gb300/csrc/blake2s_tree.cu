@@ -14,7 +14,7 @@
 // integer atomic: integer addition is associative, so Q does not depend on the
 // order the atomics land in. Rows never straddle leaves because head_dim is a
 // power of two with rows of at most 1024 bytes.
-#include "cm_kernels.h"
+#include "cm_hash_kernels.h"
 
 #include <vector>
 

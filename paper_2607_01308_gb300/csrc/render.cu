@@ -28,7 +28,7 @@
 // cannot certify are recomputed in fp64 with the operation sequence of the
 // definition and rounded directly to bf16 (fp64 throughput is very low on this part,
 // so it must stay rare). The output is bit-exact either way.
-#include "cm_kernels.h"
+#include "cm_render_kernels.h"
 
 namespace cm {
 namespace {
