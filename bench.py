@@ -37,6 +37,7 @@ if ROOT not in sys.path:
 METRIC = "cm_render merged-cache GB/s and % of HBM peak; merges/sec (ingest+union+render)"
 UNIT = "merges/s"
 WORKLOAD = "q4b"
+BASE_SEED_REDELIVER = 42 + 997   # delivery order of the re-delivery sweep
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 # Integer-ALU roofline of the content-address kernel: a BLAKE2s block (64 bytes) is
@@ -59,6 +60,10 @@ def parse_args():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--e2e-steps", type=int, default=None)
+    p.add_argument("--redeliver", type=int, default=0, metavar="R",
+                   help="re-delivery sweep: every fragment of the Qwen3-4B-shaped merge arrives R "
+                        "times as separate copies; merges/s with the byte-comparison fast path "
+                        "off and on")
     p.add_argument("--serve", action="store_true",
                    help="run the serving sweep (64 requests of 3 Qwen3-4B-shaped fragments with "
                         "re-deliveries) instead of the single-merge benchmark")
@@ -313,6 +318,75 @@ def whole_job_rate(world: int, steps_per_rank: int, max_elapsed_ms: float) -> fl
 
 # ---------------------------------------------------------------- serving sweep
 
+def run_redeliver(args):
+    """Re-delivery (the fault model of Section 5.9): one replica receives each of the 4
+    Qwen3-4B-shaped fragments R times, every delivery its own byte-identical copy, in a
+    shuffled order, with one cm_ingest_batch call, then renders the set. Timed with the
+    re-delivery fast path (cm_context_set_dedup_by_bytes) off and on; the rendered bytes
+    are compared between the two."""
+    import numpy as np
+    import torch
+    import paper_2607_01308_gb300 as cm
+    import synthetic
+    R = args.redeliver
+    w = synthetic.WORKLOADS[WORKLOAD]
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    specs = synthetic.fragment_specs(w)
+    frags = [synthetic.make_fragment_torch(sp, w.num_layers, w.num_kv_heads, w.head_dim, dev)
+             for sp in specs]
+    order = np.random.default_rng(BASE_SEED_REDELIVER).permutation(len(frags) * R)
+    copies = [(K.clone(), V.clone()) for K, V in frags for _ in range(R)]
+    msgs = [copies[int(i)] for i in order]
+    fd = [cm.fragment_from_tensors(K, V) for K, V in msgs]
+    total = sum(sp.seq_len for sp in specs)
+    outs = [torch.empty((w.num_layers, w.num_kv_heads, total, w.head_dim), dtype=torch.bfloat16,
+                        device=dev) for _ in range(4)]
+    ctx = cm.Context(0, synthetic.ROPE_THETA)
+    stream = torch.cuda.current_stream(dev)
+
+    def merge(k_out, v_out):
+        s = cm.cm_set_create(ctx.handle)
+        res = cm.cm_ingest_batch(s, fd, stream)
+        cm.cm_render(s, k_out.data_ptr(), v_out.data_ptr(), total, stream)
+        cm.cm_set_destroy(s)
+        return res
+
+    line = {"mode": "re-delivery sweep", "metric": METRIC, "unit": UNIT, "n_gpus": 1,
+            "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": WORKLOAD_TEXT[WORKLOAD], "redeliveries": R,
+                       "deliveries": len(fd), "distinct": len(frags)}}
+    for name, on, (k_out, v_out) in (("fast_path_off", False, outs[:2]), ("fast_path_on", True, outs[2:])):
+        cm.cm_context_set_dedup_by_bytes(ctx.handle, on)
+        for _ in range(3):
+            res = merge(k_out, v_out)
+        assert sum(a for _, a in res) == len(fd) - len(frags)
+        torch.cuda.synchronize(dev)
+        cm.cm_context_kernel_times(ctx.handle, reset=True)
+        cm.cm_context_set_timing(ctx.handle, True)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        n = 20
+        with ClockSampler(0) as clocks:
+            e0.record(stream)
+            for _ in range(n):
+                merge(k_out, v_out)
+            e1.record(stream)
+            torch.cuda.synchronize(dev)
+        cm.cm_context_set_timing(ctx.handle, False)
+        kt = cm.cm_context_kernel_times(ctx.handle, reset=True)
+        ms = e0.elapsed_time(e1) / n
+        line[name] = {"value": 1000.0 / ms, "ms_per_merge": ms,
+                      "leaf_hash_launches_per_merge": kt["leaf_hash_launches"] / n,
+                      "hash_ms_per_merge": (kt["leaf_hash_ms"] + kt["inner_hash_ms"]) / n,
+                      "clocks": clocks.summary()}
+    assert torch.equal(outs[0].view(torch.int16), outs[2].view(torch.int16))
+    assert torch.equal(outs[1].view(torch.int16), outs[3].view(torch.int16))
+    line["value"] = line["fast_path_on"]["value"]
+    print(json.dumps(line), flush=True)
+    ctx.close()
+    return 0
+
+
 def run_serve(args):
     """64 independent merge requests on the Qwen3-4B shape: each delivers its 3 fragments
     (lengths U{512..4096}, each re-sent with probability 0.1, in shuffled order) into a fresh
@@ -459,6 +533,8 @@ def main():
     args = parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.redeliver:
+        return run_redeliver(args)
     if args.serve:
         return run_serve(args)
 

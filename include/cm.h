@@ -311,6 +311,21 @@ cm_status cm_bagmerge(cm_context *ctx, const cm_fragment *frags, int32_t n, void
  * the output of the affected render is incomplete. CM_OK otherwise. */
 cm_status cm_context_check(cm_context *ctx, cm_stream_t stream);
 
+/* Re-delivery fast path for every later cm_ingest, cm_ingest_batch and cm_ingest_many
+ * on ctx (off by default). The content address is a function of a fragment's bytes,
+ * shapes and dtype (Section 4.3), so a delivery byte-identical to a fragment whose id is
+ * known has that id without hashing it. With the path on, each delivery is first
+ * compared byte for byte with at most 16 fragments of its exact shape and length: the
+ * records its set holds, then the earlier deliveries of the same call (identical (k, v)
+ * pointers count as equal without reading them). A delivery found equal takes that
+ * fragment's id and norm key and is not hashed; the others are hashed as usual. Results
+ * (ids, absorption, the set) are identical with the path on or off. The candidates'
+ * first 4 KiB are compared first; only the first candidate whose prefix matches is then
+ * compared in full, reading both fragments at HBM speed. This costs one more stream
+ * synchronisation per call that has candidates (two if a prefix matches): turn it on
+ * where re-deliveries are common (gossip, retries). The paper has no counterpart. */
+cm_status cm_context_set_dedup_by_bytes(cm_context *ctx, int32_t enable);
+
 /* Width of the render kernel's CTAs for every later render launched from ctx (a
  * scheduling aid; the paper has no counterpart). The render is one persistent CTA per
  * SM. warps = 16 (the default) gives it the whole register file of each SM: the fastest

@@ -103,6 +103,7 @@ _SIGS = {
     "cm_set_leq": (_c.c_int, [_P, _P, _c.POINTER(_c.c_int32)]),
     "cm_measure_int_alu": (_c.c_int, [_c.c_int32, _c.POINTER(_c.c_double), _c.POINTER(_c.c_double)]),
     "cm_context_set_render_warps": (_c.c_int, [_P, _c.c_int32]),
+    "cm_context_set_dedup_by_bytes": (_c.c_int, [_P, _c.c_int32]),
     "cm_context_set_timing": (_c.c_int, [_P, _c.c_int32]),
     "cm_context_kernel_times": (_c.c_int, [_P, _c.POINTER(cm_kernel_times), _c.c_int32]),
     "cm_union": (_c.c_int, [_P, _P]),
@@ -262,6 +263,10 @@ def cm_measure_int_alu(device: int = 0) -> Tuple[float, float]:
     x, c = ctypes.c_double(), ctypes.c_double()
     _check(lib.cm_measure_int_alu(device, ctypes.byref(x), ctypes.byref(c)))
     return x.value, c.value
+
+
+def cm_context_set_dedup_by_bytes(ctx: int, enable: bool) -> None:
+    _check(lib.cm_context_set_dedup_by_bytes(ctx, int(enable)))
 
 
 def cm_context_set_render_warps(ctx: int, warps: int) -> None:

@@ -4,6 +4,7 @@ Three translation units compiled in parallel, then one shared-library link:
   csrc/cm_host.cpp       host core (g++, C++17, no floating-point contraction)
   csrc/blake2s_tree.cu   content-address kernels (nvcc, sm_103a)
   csrc/render.cu         render kernel (nvcc, sm_103a)
+  csrc/dedup.cu          byte comparison of the re-delivery fast path (nvcc, sm_103a)
 The CUDA runtime is linked statically into libcm.so and only the cm_* symbols
 are exported (csrc/libcm.map).
 """
@@ -27,7 +28,7 @@ NVCC_FLAGS = ["-std=c++17", "-O3", "-lineinfo", "-fmad=false", "-Xcompiler", "-f
 CXX_FLAGS = ["-std=c++17", "-O2", "-fPIC", "-ffp-contract=off", "-Wall", "-Wextra",
              "-I" + INCLUDE, "-I" + CSRC]
 
-CUDA_SOURCES = ["blake2s_tree.cu", "render.cu"]
+CUDA_SOURCES = ["blake2s_tree.cu", "render.cu", "dedup.cu"]
 CXX_SOURCES = ["cm_host.cpp"]
 
 

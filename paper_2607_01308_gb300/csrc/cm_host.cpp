@@ -145,6 +145,7 @@ struct cm_context {
     // launch parameters of the render kernel (about 31 KB), reused by every launch
     std::unique_ptr<cm::RenderParams> render_params;
     int32_t render_warps = 16;   // warps per render CTA (cm_context_set_render_warps)
+    bool dedup_bytes = false;    // re-delivery fast path (cm_context_set_dedup_by_bytes)
 };
 
 struct cm_set {
@@ -578,6 +579,134 @@ cm_status guarded(F &&f) {
     }
 }
 
+// Re-delivery fast path: the deliveries of one ingest call that are byte-identical to
+// a fragment their set already holds or to an earlier delivery of the call. A
+// delivery is compared with at most kMaxCandidates fragments of its shape and length
+// (the set's records first, then the call's earlier deliveries, the latest first):
+// their first 4 KiB in one pass, then all bytes of the first candidate whose prefix
+// matched; identical (k, v) pointers count as equal without a comparison. Results:
+// rec[i] is the equal record, else from[i] the equal earlier delivery, else neither
+// (hash it).
+constexpr int kMaxCandidates = 16;
+
+cm_status find_redeliveries(cm_context *ctx, cm_set *const *sets,
+                            const std::vector<const cm_fragment *> &fp, cudaStream_t stream,
+                            std::vector<std::shared_ptr<const Record>> &rec,
+                            std::vector<int32_t> &from) {
+    const size_t n = fp.size();
+    rec.assign(n, nullptr);
+    from.assign(n, -1);
+    struct Cand {
+        size_t delivery;
+        std::shared_ptr<const Record> r;   // a record, or null for delivery `other`
+        size_t other;
+    };
+    std::vector<Cand> cands;
+    auto same_shape = [](const cm_fragment *f, int32_t L, int32_t H, int32_t T, int32_t d) {
+        return f->num_layers == L && f->num_kv_heads == H && f->seq_len == T && f->head_dim == d;
+    };
+    for (size_t i = 0; i < n; ++i) {
+        const cm_fragment *f = fp[i];
+        int found = 0;
+        bool same_buffers = false;
+        for (const auto &kv : sets[i]->items) {
+            const Record &r = *kv.second;
+            if (!same_shape(f, r.L, r.H, r.T, r.d)) continue;
+            if (r.k == f->k && r.v == f->v) {
+                rec[i] = kv.second;
+                same_buffers = true;
+                break;
+            }
+            if (found < kMaxCandidates) {
+                cands.push_back({i, kv.second, 0});
+                ++found;
+            }
+        }
+        for (size_t j = i; j-- > 0 && !same_buffers;) {
+            const cm_fragment *g = fp[j];
+            if (!same_shape(f, g->num_layers, g->num_kv_heads, g->seq_len, g->head_dim)) continue;
+            if (g->k == f->k && g->v == f->v) {
+                from[i] = (int32_t)j;
+                same_buffers = true;
+                break;
+            }
+            if (found < kMaxCandidates) {
+                cands.push_back({i, nullptr, j});
+                ++found;
+            }
+        }
+        if (same_buffers)
+            while (!cands.empty() && cands.back().delivery == i) cands.pop_back();
+    }
+    if (cands.empty()) return CM_OK;
+    // one comparison pass over a list of candidate pairs: differ[c] = 1 if pair c differs
+    // (its first 4 KiB of K only, or all of it)
+    auto compare = [&](const std::vector<size_t> &which, bool full,
+                       std::vector<uint32_t> &differ) -> cm_status {
+        differ.assign(which.size(), 1u);
+        cm_status st = ensure_scratch(ctx, which.size() * 4, which.size() * 4);
+        if (st != CM_OK) return st;
+        auto *d_differ = reinterpret_cast<uint32_t *>(ctx->d_scratch);
+        CM_CUDA_TRY(cudaMemsetAsync(d_differ, 0, which.size() * 4, stream), "comparison flags reset");
+        for (size_t c0 = 0; c0 < which.size(); c0 += (size_t)cm::kMaxComparePairs) {
+            cm::CompareLaunch cl;
+            std::memset(&cl, 0, sizeof cl);
+            const size_t cn = std::min(which.size() - c0, (size_t)cm::kMaxComparePairs);
+            for (size_t q = 0; q < cn; ++q) {
+                const Cand &c = cands[which[c0 + q]];
+                const cm_fragment *f = fp[c.delivery];
+                const void *bk = c.r ? c.r->k : fp[c.other]->k;
+                const void *bv = c.r ? c.r->v : fp[c.other]->v;
+                const uint64_t vecs =
+                    (uint64_t)f->num_layers * f->num_kv_heads * f->seq_len * f->head_dim * 2 / 16;
+                cl.pair[q] = {static_cast<const uint4 *>(f->k), static_cast<const uint4 *>(f->v),
+                              static_cast<const uint4 *>(bk), static_cast<const uint4 *>(bv), vecs};
+                cl.chunk_begin[q + 1] =
+                    cl.chunk_begin[q] + 2 * ceil_div(vecs, (uint64_t)cm::kCompareChunkVecs);
+            }
+            cl.count = (uint32_t)cn;
+            cl.differ = d_differ + c0;
+            CM_CUDA_TRY(full ? cm::launch_compare_full(cl, ctx->num_sms, stream)
+                             : cm::launch_compare_prefix(cl, stream),
+                        "comparison launch");
+        }
+        CM_CUDA_TRY(cudaMemcpyAsync(ctx->h_pinned, d_differ, which.size() * 4,
+                                    cudaMemcpyDeviceToHost, stream),
+                    "comparison flags copy");
+        CM_CUDA_TRY(cudaStreamSynchronize(stream), "comparison synchronisation");
+        std::memcpy(differ.data(), ctx->h_pinned, which.size() * 4);
+        return CM_OK;
+    };
+    // first the 4 KiB prefixes of every pair, then the whole of one pair per delivery:
+    // its first candidate whose prefix matched (one full comparison suffices, and
+    // re-deliveries of one fragment would otherwise all be compared with each other)
+    std::vector<size_t> all(cands.size());
+    for (size_t c = 0; c < cands.size(); ++c) all[c] = c;
+    std::vector<uint32_t> prefix_differ, full_differ;
+    cm_status st = compare(all, false, prefix_differ);
+    if (st != CM_OK) return st;
+    std::vector<size_t> chosen;
+    std::vector<bool> has_choice(n, false);
+    for (size_t c = 0; c < cands.size(); ++c) {
+        const size_t i = cands[c].delivery;
+        if (prefix_differ[c] != 0 || has_choice[i]) continue;
+        has_choice[i] = true;
+        chosen.push_back(c);
+    }
+    if (chosen.empty()) return CM_OK;
+    st = compare(chosen, true, full_differ);
+    if (st != CM_OK) return st;
+    for (size_t q = 0; q < chosen.size(); ++q) {
+        if (full_differ[q] != 0) continue;
+        const Cand &c = cands[chosen[q]];
+        if (c.r)
+            rec[c.delivery] = c.r;
+        else
+            from[c.delivery] = (int32_t)c.other;
+    }
+    return CM_OK;
+}
+
 // Ingest (Algorithm 2) of n deliveries, delivery i into sets[i] (several entries
 // may name one set): one GPU pass for all of them, then the insertions in delivery
 // order, so a delivery whose id its set already holds (before the batch or from an
@@ -616,18 +745,57 @@ cm_status ingest_deliveries(cm_set *const *sets, const cm_fragment *frags, int32
     DeviceScope scope(ctx->device);
     if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
     const cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+    // with the re-delivery fast path on, deliveries byte-identical to a known fragment
+    // take its id and norm key and are not hashed
+    std::vector<std::shared_ptr<const Record>> same_rec;
+    std::vector<int32_t> same_as;
+    cm_status st = CM_OK;
+    if (ctx->dedup_bytes) {
+        st = find_redeliveries(ctx, sets, fp, cs, same_rec, same_as);
+        if (st != CM_OK) return st;
+    } else {
+        same_rec.assign((size_t)n, nullptr);
+        same_as.assign((size_t)n, -1);
+    }
+    std::vector<const cm_fragment *> to_hash;
+    std::vector<size_t> hashed_as((size_t)n, 0);
+    for (int32_t i = 0; i < n; ++i)
+        if (!same_rec[(size_t)i] && same_as[(size_t)i] < 0) {
+            hashed_as[(size_t)i] = to_hash.size();
+            to_hash.push_back(fp[(size_t)i]);
+        }
+    std::vector<cm_id> hashed_ids(to_hash.size());
+    std::vector<std::vector<uint64_t>> hashed_Q(to_hash.size());
+    if (!to_hash.empty()) {
+        st = fragments_digest(ctx, to_hash.data(), to_hash.size(), cs, hashed_ids.data(),
+                              hashed_Q.data());
+        if (st != CM_OK) return st;
+    }
+    // ids in delivery order; Qsrc[i] is where delivery i's norm key lives once delivery i
+    // has been processed (its own record, a record it matched, or a hashed result)
     std::vector<cm_id> ids((size_t)n);
-    std::vector<std::vector<uint64_t>> Qs((size_t)n);
-    cm_status st = fragments_digest(ctx, fp.data(), (size_t)n, cs, ids.data(), Qs.data());
-    if (st != CM_OK) return st;
+    std::vector<const std::vector<uint64_t> *> Qsrc((size_t)n, nullptr);
     for (int32_t i = 0; i < n; ++i) {
         cm_set *set = sets[i];
         const cm_fragment *f = fp[(size_t)i];
+        std::vector<uint64_t> *own = nullptr;
+        if (same_rec[(size_t)i]) {
+            ids[(size_t)i] = same_rec[(size_t)i]->id;
+            Qsrc[(size_t)i] = &same_rec[(size_t)i]->Q;
+        } else if (same_as[(size_t)i] >= 0) {
+            ids[(size_t)i] = ids[(size_t)same_as[(size_t)i]];
+            Qsrc[(size_t)i] = Qsrc[(size_t)same_as[(size_t)i]];
+        } else {
+            ids[(size_t)i] = hashed_ids[hashed_as[(size_t)i]];
+            own = &hashed_Q[hashed_as[(size_t)i]];
+            Qsrc[(size_t)i] = own;
+        }
         if (out_ids) out_ids[i] = ids[(size_t)i];
         const IdKey key = key_of(ids[(size_t)i]);
         auto it = set->items.find(key);
         if (it != set->items.end()) {
-            if (ctx->verify) {
+            // a byte match against this very record needs no second look at the bytes
+            if (ctx->verify && same_rec[(size_t)i] != it->second) {
                 bool equal = false;
                 st = bytes_equal(ctx, f, *it->second, cs, &equal);
                 if (st != CM_OK) return st;
@@ -644,7 +812,11 @@ cm_status ingest_deliveries(cm_set *const *sets, const cm_fragment *frags, int32
         rec->d = f->head_dim;
         rec->k = f->k;
         rec->v = f->v;
-        rec->Q = std::move(Qs[(size_t)i]);
+        if (own)
+            rec->Q = std::move(*own);
+        else
+            rec->Q = *Qsrc[(size_t)i];
+        Qsrc[(size_t)i] = &rec->Q;
         set->items.emplace(key, std::move(rec));
         if (!set->has_shape) {
             set->has_shape = true;
@@ -804,6 +976,13 @@ cm_status cm_ingest_many(cm_set *const *sets, const cm_fragment *frags, int32_t 
     });
 }
 
+
+cm_status cm_context_set_dedup_by_bytes(cm_context *ctx, int32_t enable) {
+    if (!ctx) return fail(CM_ERR_INVALID_ARG, "context is NULL");
+    std::lock_guard<std::mutex> lock(ctx->mu);
+    ctx->dedup_bytes = enable != 0;
+    return CM_OK;
+}
 
 cm_status cm_context_set_render_warps(cm_context *ctx, int32_t warps) {
     if (!ctx) return fail(CM_ERR_INVALID_ARG, "context is NULL");

@@ -34,6 +34,7 @@ int main(void) {
     if (cm_set_leq(NULL, NULL, &leq) != CM_ERR_INVALID_ARG) return 12;
     if (cm_measure_int_alu(0, NULL, NULL) != CM_ERR_INVALID_ARG) return 13;
     if (cm_context_set_render_warps(NULL, 8) != CM_ERR_INVALID_ARG) return 14;
+    if (cm_context_set_dedup_by_bytes(NULL, 1) != CM_ERR_INVALID_ARG) return 15;
     printf("ok %s\n", cm_last_error_message());
     return 0;
 }

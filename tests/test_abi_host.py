@@ -33,7 +33,7 @@ def test_header_declares_the_documented_calls():
             "cm_context_set_timing", "cm_context_kernel_times", "cm_fragment_id_static",
             "cm_render_incremental", "cm_render_paged", "cm_ingest_many", "cm_render_many",
             "cm_set_contains", "cm_set_leq", "cm_measure_int_alu",
-            "cm_context_set_render_warps"}
+            "cm_context_set_render_warps", "cm_context_set_dedup_by_bytes"}
     assert want <= set(_declared_functions())
 
 
