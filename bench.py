@@ -390,11 +390,12 @@ def run_redeliver(args):
 def run_serve(args):
     """64 independent merge requests on the Qwen3-4B shape: each delivers its 3 fragments
     (lengths U{512..4096}, each re-sent with probability 0.1, in shuffled order) into a fresh
-    set, which is then rendered. Every delivery is its own device buffer. Timed three ways:
+    set, which is then rendered. Every delivery is its own device buffer. Timed four ways:
     one request at a time (a batched ingest and a render per request); `--group` requests at
     a time (one cm_ingest_many and one cm_render_many per group, each request rendering into
-    its own output buffer); and grouped with each group's render (8-warp CTAs) running while
-    the next group hashes on a second stream (the line's value)."""
+    its own output buffer); grouped with each group's render (8-warp CTAs) running while
+    the next group hashes on a second stream; and that with the re-delivery fast path on
+    (the line's value)."""
     import torch
     import paper_2607_01308_gb300 as cm
     import synthetic
@@ -503,12 +504,16 @@ def run_serve(args):
     msg, ktg, clocksg = timed(per_group)
     cm.cm_context_set_render_warps(ctx.handle, 8)
     mso, kto, clockso = timed(overlapped)
+    cm.cm_context_set_dedup_by_bytes(ctx.handle, True)
+    msd, ktd, clocksd = timed(overlapped)
+    cm.cm_context_set_dedup_by_bytes(ctx.handle, False)
     cm.cm_context_set_render_warps(ctx.handle, 16)
     single = summary(ms1, kt1)
     group = summary(msg, ktg)
     ovl = summary(mso, kto)
+    ovl_dedup = summary(msd, ktd)
     line = {
-        "mode": "serving sweep", "metric": METRIC, "value": ovl["value"], "unit": UNIT,
+        "mode": "serving sweep", "metric": METRIC, "value": ovl_dedup["value"], "unit": UNIT,
         "n_gpus": 1, "requests": len(reqs), "higher_is_better": True, "dtype": "bf16",
         "data": "synthetic",
         "config": {"workload": "serving sweep on the Qwen3-4B shape: 64 requests x 3 fragments, "
@@ -519,6 +524,9 @@ def run_serve(args):
         "grouped_overlapped": dict(ovl, clocks=clockso,
                                    note="8-warp render CTAs; group g renders while group g+1 "
                                         "hashes on a second stream, so the kernel times overlap"),
+        "grouped_overlapped_dedup": dict(ovl_dedup, clocks=clocksd,
+                                         note="as grouped_overlapped, with the re-delivery fast "
+                                              "path on (re-sent copies are compared, not hashed)"),
         "grouped": dict(group, clocks=clocksg),
         "per_request": dict(single, clocks=clocks1),
     }
