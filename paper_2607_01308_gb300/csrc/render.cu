@@ -269,7 +269,8 @@ __device__ __forceinline__ Item item_of(const RenderParams &p, uint32_t g) {
     Item it;
     it.src = static_cast<const uint8_t *>(is_v ? S.v : S.k) + (lh * S.seq_len + row0) * row_bytes;
     if (p.paged) {
-        const int64_t l = lh / p.num_heads, h = lh - l * p.num_heads;
+        const uint32_t l32 = lhp / (uint32_t)p.num_heads;      // 32-bit: lhp < 2^32
+        const int64_t l = l32, h = (int64_t)(lhp - l32 * (uint32_t)p.num_heads);
         it.dst = static_cast<uint8_t *>(is_v ? p.v_pool : p.k_pool) +
                  (l * p.stride_layer + h * p.stride_head) * 2;
     } else {
@@ -284,10 +285,44 @@ __device__ __forceinline__ Item item_of(const RenderParams &p, uint32_t g) {
     return it;
 }
 
+// Paged outputs: where the rows of one item go. When the block size is a power of two
+// no smaller than the item's row count, the item's positions lie in at most two logical
+// blocks: rows [0, split) in the first at a + r * stride, the rest in the next at
+// b + r * stride (b is offset back by split rows so that one formula serves both), and
+// the block table is read once per item instead of once per row.
+struct PagedRows {
+    uint8_t *a;
+    uint8_t *b;
+    int64_t stride;  // bytes between consecutive positions of a block
+    int split;       // rows in the item's first block
+    bool fast;
+};
+
+__device__ __forceinline__ PagedRows paged_rows(const RenderParams &p, const Item &it) {
+    PagedRows pr;
+    pr.fast = p.log2_block_size >= 0 && (int64_t)it.rows <= p.block_size;
+    pr.a = pr.b = it.dst;
+    pr.stride = p.stride_token * 2;
+    pr.split = it.rows;
+    if (pr.fast) {
+        const int64_t b0 = it.pos0 >> p.log2_block_size;
+        const int64_t o0 = it.pos0 & (p.block_size - 1);
+        const int64_t k = p.block_size - o0;                 // rows left in block b0
+        pr.a = it.dst + (int64_t)__ldg(p.block_table + b0) * p.stride_block * 2 + o0 * pr.stride;
+        if (k < it.rows) {
+            pr.split = (int)k;
+            pr.b = it.dst + (int64_t)__ldg(p.block_table + b0 + 1) * p.stride_block * 2 - k * pr.stride;
+        }
+    }
+    return pr;
+}
+
 // Start of output row r of an item: contiguous rows, or the row's slot in its block.
 template <bool kPaged>
-__device__ __forceinline__ uint4 *row_dst(const RenderParams &p, const Item &it, int r) {
+__device__ __forceinline__ uint4 *row_dst(const RenderParams &p, const Item &it, int r,
+                                          const PagedRows &pr) {
     if (!kPaged) return reinterpret_cast<uint4 *>(it.dst) + (int64_t)r * (p.head_dim >> 3);
+    if (pr.fast) return reinterpret_cast<uint4 *>((r < pr.split ? pr.a : pr.b) + (int64_t)r * pr.stride);
     const int64_t pos = it.pos0 + r;
     int64_t b, o;
     if (p.log2_block_size >= 0) {                       // the usual case: shifts
@@ -312,6 +347,8 @@ __device__ __forceinline__ void copy_from_smem(const RenderParams &p, const Item
     constexpr int kU = kItemBytes / 16 / 32;          // 8 vectors per lane
     const int n_vec = (int)(it.bytes >> 4);
     const uint4 *src = reinterpret_cast<const uint4 *>(buf);
+    PagedRows pr{};
+    if (kPaged) pr = paged_rows(p, it);
     uint4 r[kU];
 #pragma unroll
     for (int u = 0; u < kU; ++u)
@@ -327,7 +364,7 @@ __device__ __forceinline__ void copy_from_smem(const RenderParams &p, const Item
 #pragma unroll
         for (int u = 0; u < kU; ++u) {
             const int v = lane + 32 * u;
-            if (v < n_vec) st_stream(row_dst<true>(p, it, v >> log2_vpr) + (v & col_mask), r[u]);
+            if (v < n_vec) st_stream(row_dst<true>(p, it, v >> log2_vpr, pr) + (v & col_mask), r[u]);
         }
     }
 }
@@ -343,6 +380,8 @@ __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const fl
     const int half_vecs = p.head_dim >> 4;
     const int n_pairs = it.rows * half_vecs;
     const int cs_index = it.cs_index + 8 * lane_v;
+    PagedRows pr{};
+    if (kPaged) pr = paged_rows(p, it);
     float c[8], s[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
@@ -364,7 +403,7 @@ __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const fl
         rotate_word(a.z, b.z, c[4], s[4], c[5], s[5], ao.z, bo.z, b2);
         rotate_word(a.w, b.w, c[6], s[6], c[7], s[7], ao.w, bo.w, b3);
         if ((b0 | b1 | b2 | b3) != 0u) fixup_pair(p, tab, cs_index, a, b, b0, b1, b2, b3, ao, bo);
-        uint4 *d = row_dst<kPaged>(p, it, row) + lane_v;
+        uint4 *d = row_dst<kPaged>(p, it, row, pr) + lane_v;
         st_stream(d, ao);
         st_stream(d + half_vecs, bo);
     }
