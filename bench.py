@@ -377,6 +377,7 @@ def run_redeliver(args):
         ms = e0.elapsed_time(e1) / n
         line[name] = {"value": 1000.0 / ms, "ms_per_merge": ms,
                       "leaf_hash_launches_per_merge": kt["leaf_hash_launches"] / n,
+                      "fragments_hashed_per_merge": kt["leaf_hash_fragments"] / n,
                       "hash_ms_per_merge": (kt["leaf_hash_ms"] + kt["inner_hash_ms"]) / n,
                       "clocks": clocks.summary()}
     assert torch.equal(outs[0].view(torch.int16), outs[2].view(torch.int16))
@@ -750,8 +751,11 @@ def main():
         ms_per_step = elapsed_ms / args.steps
         launches_per_step = (ktimes["leaf_hash_launches"] + ktimes["inner_hash_launches"] +
                              ktimes["render_launches"]) / args.steps
+        # one leaf-hash launch covers every fragment of an ingest call (up to 32): the
+        # work of a launch is the bytes of the step's fragments divided by its launches
+        leaf_launches_per_step = max(1, ktimes["leaf_hash_launches"]) / args.steps
         leaf_ms = ktimes["leaf_hash_ms"] / max(1, ktimes["leaf_hash_launches"])
-        frag_bytes = hash_bytes / len(specs)
+        frag_bytes = hash_bytes / leaf_launches_per_step
         hash_tops = HASH_ALU_OPS_PER_BYTE * frag_bytes / (leaf_ms * 1e-3) / 1e12
         alu_peak = NUM_SMS * ALU_OPS_PER_CLK_PER_SM * sm_max_mhz() * 1e6 / 1e12
         kernel_render_ms = ktimes["render_ms"] / max(1, ktimes["render_launches"])
@@ -771,6 +775,7 @@ def main():
             "traffic": profile_traffic("blake2s_tree.cu", "leaf_hash_kernel_q4b.md"),
             "algorithmic_ops_per_launch": HASH_ALU_OPS_PER_BYTE * frag_bytes,
             "bytes_hashed_per_launch": frag_bytes, "ms_per_launch": leaf_ms,
+            "fragments_per_launch": ktimes["leaf_hash_fragments"] / max(1, ktimes["leaf_hash_launches"]),
             "hash_gbs": frag_bytes / (leaf_ms * 1e-3) / 1e9,
             "hash_frac_of_measured_hbm": frag_bytes / (leaf_ms * 1e-3) / 1e9 / peak,
             # against every integer lane of an SM (ALU and FMA pipes, 128 per clock); only

@@ -44,7 +44,7 @@
 extern "C" {
 #endif
 
-#define CM_ABI_VERSION 2
+#define CM_ABI_VERSION 3
 
 /* Same type as cudaStream_t (a CUDA runtime stream handle); NULL is the legacy default stream. */
 typedef struct CUstream_st *cm_stream_t;
@@ -153,8 +153,8 @@ cm_status cm_ingest(cm_set *set, const cm_fragment *frag, cm_stream_t stream, cm
                     int32_t *out_absorbed);
 
 /* Ingest of n deliveries in order (Algorithm 2, Ingest, applied n times): the same
- * result as n calls of cm_ingest, with one pass of GPU work for all of them (the
- * leaf-hash launch of every fragment, then one launch per tree level covering all
+ * result as n calls of cm_ingest, with one pass of GPU work for all of them (one
+ * leaf-hash launch and one launch for the tree levels above the leaves per 32
  * fragments) and a single synchronisation of `stream`. A delivery whose id is
  * already in the set, or equal to an earlier delivery of the same batch, is
  * absorbed. All fragments must have the set's shape (or one common shape if the
@@ -339,12 +339,13 @@ cm_status cm_context_set_render_warps(cm_context *ctx, int32_t warps);
 
 /* Device time per kernel, accumulated while timing is on (a profiling aid). */
 typedef struct cm_kernel_times {
-    double leaf_hash_ms;          /* content address, level 0 (one launch per fragment) */
+    double leaf_hash_ms;          /* content address, level 0 (one launch per up to 32 fragments) */
     int64_t leaf_hash_launches;
     double inner_hash_ms;         /* content address, tree levels above the leaves */
     int64_t inner_hash_launches;
     double render_ms;             /* render / BagMerge */
     int64_t render_launches;
+    int64_t leaf_hash_fragments;  /* fragments hashed by those leaf-hash launches */
 } cm_kernel_times;
 
 /* Turn kernel timing on or off for ctx. While on, every launch the context makes

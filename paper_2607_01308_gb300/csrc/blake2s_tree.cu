@@ -16,6 +16,8 @@
 // power of two with rows of at most 1024 bytes.
 #include "cm_hash_kernels.h"
 
+#include <cstring>
+
 #include <vector>
 
 namespace cm {
@@ -175,11 +177,14 @@ __device__ __forceinline__ const uint8_t *cursor_next(const LeafLaunch &a, Strea
     return p;
 }
 
-constexpr int kLeafThreads = 128;
+constexpr int kLeafThreads = kLeafBlockThreads;
 
 __global__ void __launch_bounds__(kLeafThreads)
-leaf_hash_kernel(const __grid_constant__ LeafLaunch a) {
-    const uint64_t leaf = (uint64_t)blockIdx.x * kLeafThreads + threadIdx.x;
+leaf_hash_kernel(const __grid_constant__ LeafGroup grp) {
+    uint32_t fi = 0;                                   // the block's fragment (uniform)
+    while (fi + 1 < grp.count && blockIdx.x >= grp.block_begin[fi + 1]) ++fi;
+    const LeafLaunch &a = grp.frag[fi];
+    const uint64_t leaf = (uint64_t)(blockIdx.x - grp.block_begin[fi]) * kLeafThreads + threadIdx.x;
     if (leaf >= a.num_leaves) return;
     const uint64_t begin = leaf * kLeafBytes;
     const uint64_t rem = a.stream_bytes - begin;
@@ -354,12 +359,21 @@ __global__ void compare_kernel(const uint4 *__restrict__ a, const uint4 *__restr
 
 }  // namespace
 
-cudaError_t launch_leaf_hash(const LeafLaunch &a, cudaStream_t stream) {
-    if (a.num_leaves == 0) return cudaSuccess;
-    const uint64_t blocks = (a.num_leaves + kLeafThreads - 1) / kLeafThreads;
+cudaError_t launch_leaf_hash_group(const LeafGroup &g, cudaStream_t stream) {
+    const uint64_t blocks = g.block_begin[g.count];
+    if (g.count == 0 || blocks == 0) return cudaSuccess;
     if (blocks > 0x7FFFFFFFull) return cudaErrorInvalidValue;
-    leaf_hash_kernel<<<(unsigned)blocks, kLeafThreads, 0, stream>>>(a);
+    leaf_hash_kernel<<<(unsigned)blocks, kLeafThreads, 0, stream>>>(g);
     return cudaGetLastError();
+}
+
+cudaError_t launch_leaf_hash(const LeafLaunch &a, cudaStream_t stream) {
+    LeafGroup g;
+    std::memset(&g, 0, sizeof g);
+    g.count = 1;
+    g.block_begin[1] = (a.num_leaves + kLeafThreads - 1) / kLeafThreads;   // as the host does
+    g.frag[0] = a;
+    return launch_leaf_hash_group(g, stream);
 }
 
 cudaError_t launch_inner_hash(const uint8_t *children, uint64_t num_children, uint8_t *out,

@@ -38,7 +38,20 @@ struct LeafLaunch {
     TreeParams tree;
 };
 
-// Level 0: one thread per leaf; also accumulates the routing-layer norm key.
+// Level 0 of up to kMaxLeafGroup fragments in one launch: one thread per leaf, the
+// blocks of fragment i being [block_begin[i], block_begin[i + 1]); each thread whose
+// leaf lies in K[l*] also accumulates the routing-layer norm key.
+constexpr int kMaxLeafGroup = 32;
+constexpr int kLeafBlockThreads = 128;   // threads (= leaves) per block of the leaf launch
+struct LeafGroup {
+    uint32_t count;
+    uint32_t pad_;
+    uint64_t block_begin[kMaxLeafGroup + 1];
+    LeafLaunch frag[kMaxLeafGroup];
+};
+cudaError_t launch_leaf_hash_group(const LeafGroup &g, cudaStream_t stream);
+
+// Level 0 of one fragment (a group of one).
 cudaError_t launch_leaf_hash(const LeafLaunch &a, cudaStream_t stream);
 
 // Level `depth` >= 1: node j hashes the digests of children [16 j, 16 j + 16).

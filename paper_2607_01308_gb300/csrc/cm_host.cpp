@@ -139,6 +139,7 @@ struct cm_context {
     std::vector<cudaEvent_t> event_pool;
     double time_ms[3] = {0, 0, 0};
     int64_t launches[3] = {0, 0, 0};
+    int64_t leaf_fragments = 0;   // fragments hashed by the timed leaf-hash launches
     // RoPE frequencies theta^(-2j/d), j < d/2, for the last head_dim rendered
     std::vector<double> omega;
     int32_t omega_d = 0;
@@ -316,23 +317,35 @@ cm_status fragments_digest(cm_context *ctx, const cm_fragment *const *frags, siz
 
     CM_CUDA_TRY(cudaMemsetAsync(base + roots_bytes, 0, zero_end - roots_bytes, stream),
                 "zeroing the norm keys and arrival counters");
-    for (size_t i = 0; i < n; ++i) {
-        const cm_fragment *f = frags[i];
-        const Layout &l = lay[i];
-        cm::LeafLaunch a;
-        a.k = static_cast<const uint8_t *>(f->k);
-        a.v = static_cast<const uint8_t *>(f->v);
-        a.plane_bytes = l.plane;
-        a.stream_bytes = l.stream_bytes;
-        a.num_leaves = l.sizes[0];
-        a.norm_begin = 2ull * (uint64_t)l.rl * l.plane;
-        a.row_bytes = (uint32_t)f->head_dim * 2;
-        a.seq_len = (uint32_t)f->seq_len;
-        a.norm_key = reinterpret_cast<unsigned long long *>(base + l.q_off);
-        a.digests = base + l.level_off[0];
-        a.tree = l.tp;
-        CM_CUDA_TRY(timed_launch(ctx, kTimeLeaf, stream, [&] { return cm::launch_leaf_hash(a, stream); }),
+    // level 0 of up to kMaxLeafGroup fragments per launch
+    std::unique_ptr<cm::LeafGroup> grp(new cm::LeafGroup);
+    for (size_t g0 = 0; g0 < n; g0 += (size_t)cm::kMaxLeafGroup) {
+        const size_t gn = std::min(n - g0, (size_t)cm::kMaxLeafGroup);
+        std::memset(grp.get(), 0, sizeof(cm::LeafGroup));
+        grp->count = (uint32_t)gn;
+        for (size_t q = 0; q < gn; ++q) {
+            const cm_fragment *f = frags[g0 + q];
+            const Layout &l = lay[g0 + q];
+            cm::LeafLaunch &a = grp->frag[q];
+            a.k = static_cast<const uint8_t *>(f->k);
+            a.v = static_cast<const uint8_t *>(f->v);
+            a.plane_bytes = l.plane;
+            a.stream_bytes = l.stream_bytes;
+            a.num_leaves = l.sizes[0];
+            a.norm_begin = 2ull * (uint64_t)l.rl * l.plane;
+            a.row_bytes = (uint32_t)f->head_dim * 2;
+            a.seq_len = (uint32_t)f->seq_len;
+            a.norm_key = reinterpret_cast<unsigned long long *>(base + l.q_off);
+            a.digests = base + l.level_off[0];
+            a.tree = l.tp;
+            grp->block_begin[q + 1] = grp->block_begin[q] + ceil_div(a.num_leaves, (uint64_t)cm::kLeafBlockThreads);
+        }
+        if (grp->block_begin[gn] > 0x7FFFFFFFull)
+            return fail(CM_ERR_UNSUPPORTED, "leaf-hash launch exceeds 2^31 - 1 blocks");
+        CM_CUDA_TRY(timed_launch(ctx, kTimeLeaf, stream,
+                                 [&] { return cm::launch_leaf_hash_group(*grp, stream); }),
                     "leaf hash launch");
+        if (ctx->timing) ctx->leaf_fragments += (int64_t)gn;
     }
     std::unique_ptr<cm::TreeTop> top(new cm::TreeTop);
     std::memset(top.get(), 0, sizeof(cm::TreeTop));
@@ -1018,6 +1031,7 @@ cm_status cm_context_kernel_times(cm_context *ctx, cm_kernel_times *out, int32_t
         if (out) {
             out->leaf_hash_ms = ctx->time_ms[kTimeLeaf];
             out->leaf_hash_launches = ctx->launches[kTimeLeaf];
+            out->leaf_hash_fragments = ctx->leaf_fragments;
             out->inner_hash_ms = ctx->time_ms[kTimeInner];
             out->inner_hash_launches = ctx->launches[kTimeInner];
             out->render_ms = ctx->time_ms[kTimeRender];
@@ -1028,6 +1042,7 @@ cm_status cm_context_kernel_times(cm_context *ctx, cm_kernel_times *out, int32_t
                 ctx->time_ms[k] = 0;
                 ctx->launches[k] = 0;
             }
+            ctx->leaf_fragments = 0;
         }
         return CM_OK;
     });

@@ -99,19 +99,20 @@ def test_duplicates_are_not_hashed(ctxs):
     res, t = _timed(on, lambda: S.ingest_batch([A, c1, c2, B, A]))
     assert [a for _, a in res] == [False, True, True, False, True]
     assert res[1][0] == res[2][0] == res[4][0] == res[0][0]
-    assert t["leaf_hash_launches"] == 2            # A and B only
+    assert t["leaf_hash_fragments"] == 2           # A and B only
     # a later call: a clone of a fragment the set holds is absorbed with no hashing at all
     c3 = _clone(B)
     res2, t2 = _timed(on, lambda: S.ingest_batch([c3]))
     assert res2 == [(res[3][0], True)]
-    assert t2["leaf_hash_launches"] == 0 and t2["inner_hash_launches"] == 0
+    assert t2["leaf_hash_fragments"] == 0 and t2["leaf_hash_launches"] == 0
+    assert t2["inner_hash_launches"] == 0
     # in one call, a clone delivered to another set than its original takes the
     # original's id and norm key: the order of that set's render (which needs the norm
     # key) and its bytes are the oracle's
     U, T = cm.FragmentSet(on), cm.FragmentSet(on)
     res3, t3 = _timed(on, lambda: cm.ingest_many([(U, *B), (T, *_clone(B)), (T, *A)]))
     assert [a for _, a in res3] == [False, False, False]
-    assert t3["leaf_hash_launches"] == 2            # B and A; the clone is not hashed
+    assert t3["leaf_hash_fragments"] == 2          # B and A; the clone is not hashed
     kT, vT = empty_out(3, 2, 81, 64)
     n, order = T.render(kT, vT)
     ref = oracle.from_deliveries([oracle_fragment(*B), oracle_fragment(*A)])

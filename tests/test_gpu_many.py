@@ -109,7 +109,8 @@ def test_ingest_many_equals_sequential_ingest(ctx):
     res = cm.ingest_many([(sets[s], *frags[f]) for s, f in plan])
     cm.cm_context_set_timing(ctx.handle, False)
     t = cm.cm_context_kernel_times(ctx.handle, reset=True)
-    assert t["leaf_hash_launches"] == len(plan) and t["inner_hash_launches"] == 1
+    assert t["leaf_hash_launches"] == 1 and t["inner_hash_launches"] == 1
+    assert t["leaf_hash_fragments"] == len(plan)
     ref = [oracle_fragment(K, V) for K, V in frags]
     ref_sets = [oracle.FragmentSet() for _ in range(3)]
     for (s, f), (fid, absorbed) in zip(plan, res):

@@ -298,6 +298,7 @@ def test_forty_fragments_span_two_render_and_two_tree_launches(ctx):
     cm.cm_context_set_timing(ctx.handle, False)
     t = cm.cm_context_kernel_times(ctx.handle, reset=True)
     assert t["render_launches"] == 2 and t["inner_hash_launches"] == 2
+    assert t["leaf_hash_launches"] == 2 and t["leaf_hash_fragments"] == 40
     ref_frags = [oracle_fragment(K, V) for K, V in frags]
     assert [r[0] for r in res] == [f.fid for f in ref_frags]
     K_ref, V_ref, o_order = oracle.render(oracle.from_deliveries(ref_frags), THETA)
