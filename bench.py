@@ -592,7 +592,8 @@ def main():
         cm.cm_union(a, b)   # replica exchange: A := A u B
         if timers is not None:
             timers["render"][0].record(stream)
-        n, _ = cm.cm_render(a, k_dst.data_ptr(), v_dst.data_ptr(), total_T, stream)
+        n, _ = cm.cm_render(a, k_dst.data_ptr(), v_dst.data_ptr(), total_T, stream,
+                            want_order=False)
         if timers is not None:
             timers["render"][1].record(stream)
         cm.cm_set_destroy(b)

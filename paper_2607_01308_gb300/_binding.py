@@ -308,10 +308,15 @@ def cm_set_ids(s: int) -> List[bytes]:
 
 
 def cm_render(s: int, k_out: int, v_out: int, capacity_tokens: int,
-              stream=None) -> Tuple[int, List[bytes]]:
+              stream=None, want_order: bool = True) -> Tuple[int, Optional[List[bytes]]]:
+    """(rendered length, canonical order); the order is None when want_order is False."""
+    seq = ctypes.c_int64()
+    if not want_order:
+        _check(lib.cm_render(s, k_out, v_out, capacity_tokens, _stream_handle(stream),
+                             ctypes.byref(seq), None))
+        return seq.value, None
     n = cm_set_size(s)
     order = (cm_id * max(n, 1))()
-    seq = ctypes.c_int64()
     _check(lib.cm_render(s, k_out, v_out, capacity_tokens, _stream_handle(stream),
                          ctypes.byref(seq), order))
     return seq.value, [order[i].to_bytes() for i in range(n)]
