@@ -498,7 +498,7 @@ def run_serve(args):
                 "render_gbs": render_gbs, "render_frac_of_measured_hbm": render_gbs / peak,
                 "render_ms_per_request": kt["render_ms"] / len(reqs),
                 "hash_ms_per_request": (kt["leaf_hash_ms"] + kt["inner_hash_ms"]) / len(reqs),
-                "kernel_launches": kt["leaf_hash_launches"] + kt["inner_hash_launches"]
+                "kernel_launches": kt["leaf_hash_launches"] + kt["inner_hash_launches"] + kt["aux_launches"]
                 + kt["render_launches"]}
 
     ms1, kt1, clocks1 = timed(per_request)
@@ -751,7 +751,7 @@ def main():
         render_gbs = render_bytes / (render_ms * 1e-3) / 1e9
         ms_per_step = elapsed_ms / args.steps
         launches_per_step = (ktimes["leaf_hash_launches"] + ktimes["inner_hash_launches"] +
-                             ktimes["render_launches"]) / args.steps
+                             ktimes["render_launches"] + ktimes["aux_launches"]) / args.steps
         # one leaf-hash launch covers every fragment of an ingest call (up to 32): the
         # work of a launch is the bytes of the step's fragments divided by its launches
         leaf_launches_per_step = max(1, ktimes["leaf_hash_launches"]) / args.steps

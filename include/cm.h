@@ -44,7 +44,7 @@
 extern "C" {
 #endif
 
-#define CM_ABI_VERSION 3
+#define CM_ABI_VERSION 4
 
 /* Same type as cudaStream_t (a CUDA runtime stream handle); NULL is the legacy default stream. */
 typedef struct CUstream_st *cm_stream_t;
@@ -346,6 +346,8 @@ typedef struct cm_kernel_times {
     double render_ms;             /* render / BagMerge */
     int64_t render_launches;
     int64_t leaf_hash_fragments;  /* fragments hashed by those leaf-hash launches */
+    int64_t aux_launches;         /* launches of the small kernels (result readback, byte
+                                     comparison), counted, not timed */
 } cm_kernel_times;
 
 /* Turn kernel timing on or off for ctx. While on, every launch the context makes

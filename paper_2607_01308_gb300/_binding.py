@@ -58,7 +58,7 @@ class cm_kernel_times(ctypes.Structure):
     _fields_ = [("leaf_hash_ms", ctypes.c_double), ("leaf_hash_launches", ctypes.c_int64),
                 ("inner_hash_ms", ctypes.c_double), ("inner_hash_launches", ctypes.c_int64),
                 ("render_ms", ctypes.c_double), ("render_launches", ctypes.c_int64),
-                ("leaf_hash_fragments", ctypes.c_int64)]
+                ("leaf_hash_fragments", ctypes.c_int64), ("aux_launches", ctypes.c_int64)]
 
     def as_dict(self) -> dict:
         return {name: getattr(self, name) for name, _ in self._fields_}

@@ -5,6 +5,7 @@ Three translation units compiled in parallel, then one shared-library link:
   csrc/blake2s_tree.cu   content-address kernels (nvcc, sm_103a)
   csrc/render.cu         render kernel (nvcc, sm_103a)
   csrc/dedup.cu          byte comparison of the re-delivery fast path (nvcc, sm_103a)
+  csrc/readback.cu       small device-to-host results written by the SMs (nvcc, sm_103a)
 The CUDA runtime is linked statically into libcm.so and only the cm_* symbols
 are exported (csrc/libcm.map).
 """
@@ -28,7 +29,7 @@ NVCC_FLAGS = ["-std=c++17", "-O3", "-lineinfo", "-fmad=false", "-Xcompiler", "-f
 CXX_FLAGS = ["-std=c++17", "-O2", "-fPIC", "-ffp-contract=off", "-Wall", "-Wextra",
              "-I" + INCLUDE, "-I" + CSRC]
 
-CUDA_SOURCES = ["blake2s_tree.cu", "render.cu", "dedup.cu"]
+CUDA_SOURCES = ["blake2s_tree.cu", "render.cu", "dedup.cu", "readback.cu"]
 CXX_SOURCES = ["cm_host.cpp"]
 
 

@@ -127,6 +127,7 @@ struct cm_context {
     size_t scratch_bytes = 0;
     // pinned host staging for the root digest, Q[t] and the compare flag
     uint8_t *h_pinned = nullptr;
+    void *h_pinned_dev = nullptr;   // its device-mapped address (null: use copy engines)
     size_t pinned_bytes = 0;
     int live_sets = 0;
     // kernel timing (cm_context_set_timing): events bracketing each launch
@@ -140,6 +141,7 @@ struct cm_context {
     double time_ms[3] = {0, 0, 0};
     int64_t launches[3] = {0, 0, 0};
     int64_t leaf_fragments = 0;   // fragments hashed by the timed leaf-hash launches
+    int64_t aux_launches = 0;     // readback and comparison launches while timing is on
     // RoPE frequencies theta^(-2j/d), j < d/2, for the last head_dim rendered
     std::vector<double> omega;
     int32_t omega_d = 0;
@@ -183,18 +185,36 @@ cm_status ensure_scratch(cm_context *ctx, size_t dev_bytes, size_t host_bytes) {
         const size_t old_host = ctx->pinned_bytes;
         if (ctx->h_pinned) cudaFreeHost(ctx->h_pinned);
         ctx->h_pinned = nullptr;
+        ctx->h_pinned_dev = nullptr;
         ctx->pinned_bytes = 0;
         const size_t want = std::max({host_bytes, old_host + old_host / 2, (size_t)1 << 16});
         cudaError_t e = cudaHostAlloc(reinterpret_cast<void **>(&ctx->h_pinned), want,
-                                      cudaHostAllocDefault);
+                                      cudaHostAllocMapped);
         if (e != cudaSuccess) {
             cudaGetLastError();
             return fail(CM_ERR_OOM, std::string("pinned host allocation failed: ") +
                                         cudaGetErrorString(e));
         }
+        // small results are written there by the SMs (readback.cu) when it is mapped
+        if (cudaHostGetDevicePointer(&ctx->h_pinned_dev, ctx->h_pinned, 0) != cudaSuccess) {
+            cudaGetLastError();
+            ctx->h_pinned_dev = nullptr;
+        }
         ctx->pinned_bytes = want;
     }
     return CM_OK;
+}
+
+// Reads a small device result (`bytes` at `src`) into ctx->h_pinned, enqueued on
+// `stream`: stored by the SMs through the buffer's mapped address when both are 4-byte
+// granular (so the read does not wait behind bulk device-to-host copies of other
+// streams on the copy engine), else by a copy.
+cudaError_t read_small(cm_context *ctx, const void *src, size_t bytes, cudaStream_t stream) {
+    if (ctx->h_pinned_dev && bytes % 4 == 0 && (reinterpret_cast<uintptr_t>(src) & 3u) == 0) {
+        if (ctx->timing) ++ctx->aux_launches;
+        return cm::launch_readback(ctx->h_pinned_dev, src, bytes, stream);
+    }
+    return cudaMemcpyAsync(ctx->h_pinned, src, bytes, cudaMemcpyDeviceToHost, stream);
 }
 
 // BLAKE2s parameter block (32 bytes) of the tree, node offset and depth zero,
@@ -376,7 +396,7 @@ cm_status fragments_digest(cm_context *ctx, const cm_fragment *const *frags, siz
         if (top->count == (uint32_t)cm::kMaxGroup) CM_CUDA_TRY(flush(), "tree-top launch");
     }
     CM_CUDA_TRY(flush(), "tree-top launch");
-    CM_CUDA_TRY(cudaMemcpyAsync(ctx->h_pinned, base, host_bytes, cudaMemcpyDeviceToHost, stream),
+    CM_CUDA_TRY(read_small(ctx, base, host_bytes, stream),
                 "digest copy");
     CM_CUDA_TRY(cudaStreamSynchronize(stream), "ingest synchronisation");
     for (size_t i = 0; i < n; ++i) {
@@ -393,8 +413,7 @@ cm_status fragments_digest(cm_context *ctx, const cm_fragment *const *frags, siz
 cm_status take_device_error(cm_context *ctx, cudaStream_t stream) {
     cm_status st = ensure_scratch(ctx, 0, 16);
     if (st != CM_OK) return st;
-    CM_CUDA_TRY(cudaMemcpyAsync(ctx->h_pinned, ctx->d_error, sizeof(unsigned int),
-                                cudaMemcpyDeviceToHost, stream),
+    CM_CUDA_TRY(read_small(ctx, ctx->d_error, sizeof(unsigned int), stream),
                 "error word copy");
     CM_CUDA_TRY(cudaStreamSynchronize(stream), "error word synchronisation");
     unsigned int e;
@@ -420,8 +439,7 @@ cm_status bytes_equal(cm_context *ctx, const cm_fragment *f, const Record &r, cu
     CM_CUDA_TRY(cudaMemsetAsync(flag, 0, sizeof(unsigned int), stream), "flag reset");
     CM_CUDA_TRY(cm::launch_compare(f->k, r.k, bytes, flag, stream), "compare launch");
     CM_CUDA_TRY(cm::launch_compare(f->v, r.v, bytes, flag, stream), "compare launch");
-    CM_CUDA_TRY(cudaMemcpyAsync(ctx->h_pinned, flag, sizeof(unsigned int), cudaMemcpyDeviceToHost,
-                                stream),
+    CM_CUDA_TRY(read_small(ctx, flag, sizeof(unsigned int), stream),
                 "flag copy");
     CM_CUDA_TRY(cudaStreamSynchronize(stream), "compare synchronisation");
     unsigned int h;
@@ -682,9 +700,9 @@ cm_status find_redeliveries(cm_context *ctx, cm_set *const *sets,
             CM_CUDA_TRY(full ? cm::launch_compare_full(cl, ctx->num_sms, stream)
                              : cm::launch_compare_prefix(cl, stream),
                         "comparison launch");
+            if (ctx->timing) ++ctx->aux_launches;
         }
-        CM_CUDA_TRY(cudaMemcpyAsync(ctx->h_pinned, d_differ, which.size() * 4,
-                                    cudaMemcpyDeviceToHost, stream),
+        CM_CUDA_TRY(read_small(ctx, d_differ, which.size() * 4, stream),
                     "comparison flags copy");
         CM_CUDA_TRY(cudaStreamSynchronize(stream), "comparison synchronisation");
         std::memcpy(differ.data(), ctx->h_pinned, which.size() * 4);
@@ -1032,6 +1050,7 @@ cm_status cm_context_kernel_times(cm_context *ctx, cm_kernel_times *out, int32_t
             out->leaf_hash_ms = ctx->time_ms[kTimeLeaf];
             out->leaf_hash_launches = ctx->launches[kTimeLeaf];
             out->leaf_hash_fragments = ctx->leaf_fragments;
+            out->aux_launches = ctx->aux_launches;
             out->inner_hash_ms = ctx->time_ms[kTimeInner];
             out->inner_hash_launches = ctx->launches[kTimeInner];
             out->render_ms = ctx->time_ms[kTimeRender];
@@ -1043,6 +1062,7 @@ cm_status cm_context_kernel_times(cm_context *ctx, cm_kernel_times *out, int32_t
                 ctx->launches[k] = 0;
             }
             ctx->leaf_fragments = 0;
+            ctx->aux_launches = 0;
         }
         return CM_OK;
     });

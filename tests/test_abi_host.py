@@ -45,7 +45,7 @@ def test_library_exports_every_declared_symbol(cm):
 
 
 def test_abi_version_and_status_strings(cm):
-    assert cm.cm_abi_version() == 3
+    assert cm.cm_abi_version() == 4
     for st in cm.Status:
         assert cm.cm_status_string(int(st)) == "CM_" + st.name
     assert cm.cm_status_string(99) == "CM_ERR_UNKNOWN"

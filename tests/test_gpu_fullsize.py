@@ -220,5 +220,6 @@ def test_kernel_timing_counts_every_launch(ctx):
     assert t["leaf_hash_launches"] == 1 and t["leaf_hash_fragments"] == 3   # one grouped launch
     assert t["inner_hash_launches"] == 1
     assert t["render_launches"] == 1
+    assert t["aux_launches"] == 1                  # the ingest's result readback
     assert t["leaf_hash_ms"] > 0 and t["render_ms"] > 0
     S.close()
