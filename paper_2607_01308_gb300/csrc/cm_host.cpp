@@ -190,6 +190,10 @@ cm_status ensure_scratch(cm_context *ctx, size_t dev_bytes, size_t host_bytes) {
         const size_t want = std::max({host_bytes, old_host + old_host / 2, (size_t)1 << 16});
         cudaError_t e = cudaHostAlloc(reinterpret_cast<void **>(&ctx->h_pinned), want,
                                       cudaHostAllocMapped);
+        if (e != cudaSuccess) {                    // no mapped host memory: a plain one
+            cudaGetLastError();
+            e = cudaHostAlloc(reinterpret_cast<void **>(&ctx->h_pinned), want, cudaHostAllocDefault);
+        }
         if (e != cudaSuccess) {
             cudaGetLastError();
             return fail(CM_ERR_OOM, std::string("pinned host allocation failed: ") +
