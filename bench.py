@@ -41,10 +41,11 @@ BASE_SEED_REDELIVER = 42 + 997   # delivery order of the re-delivery sweep
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 # Integer-ALU roofline of the content-address kernel: a BLAKE2s block (64 bytes) is
-# 10 rounds x 8 G x (2 three-input adds + 4 xors + 4 rotates) + 8 xors = 808 ops that
-# must issue on the integer ALU pipe; the pipe takes 16 lanes per SMSP per clock
-# (4 SMSPs -> 64 ops/clk/SM), so the peak is 152 SMs x 64 x the maximum SM clock.
-HASH_ALU_OPS_PER_BYTE = 808.0 / 64.0
+# 10 rounds x 8 G x (4 xors + 4 rotates) + 8 xors = 648 ops that must issue on the
+# integer ALU pipe (G's additions are multiply-adds on the FMA pipe); the pipe takes 16
+# lanes per SMSP per clock (4 SMSPs -> 64 ops/clk/SM), so the peak is 152 SMs x 64 x
+# the maximum SM clock.
+HASH_ALU_OPS_PER_BYTE = 648.0 / 64.0
 ALU_OPS_PER_CLK_PER_SM = 64
 NUM_SMS = 152
 CLOCK_FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"

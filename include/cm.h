@@ -362,7 +362,8 @@ cm_status cm_context_kernel_times(cm_context *ctx, cm_kernel_times *out, int32_t
  * profiling aid for the roofline of the content-address kernels; the paper has no
  * counterpart): chains of three-input xors (one integer-ALU instruction each), and the
  * BLAKE2s compression function of the content address applied to register data, counted
- * as 808 integer-ALU operations per 64-byte block (10 rounds x 8 G x 10 + 8). Both are
+ * as the 648 operations per 64-byte block that issue on the integer ALU pipe (10 rounds x
+ * 8 G x (4 xors + 4 rotations) + 8 xors; G's additions run on the FMA pipe). Both are
  * reported in 10^12 operations per second, best of three timed launches of four full
  * waves each. Synchronous; allocates and frees a small device buffer; takes a few ms.
  * The calling thread's current device is restored on return. */

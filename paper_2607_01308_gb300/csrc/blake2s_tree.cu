@@ -7,13 +7,11 @@
 // digests, shapes and dtype in the salt, seq_len in the personalisation.
 //
 // Level 0 runs one thread per leaf: 16 compressions of 64-byte blocks, loaded as
-// 128-bit vectors straight from the fragment buffers. A thread whose leaf lies in
-// K[l*] also accumulates, row by row, the squared norm of each key in fp64 in
-// ascending element order, and adds the quantised norm of every finished row
-// (round-half-even of 2^20 * sqrt, saturated at 2^44 - 1) into Q[t] with a 64-bit
-// integer atomic: integer addition is associative, so Q does not depend on the
-// order the atomics land in. Rows never straddle leaves because head_dim is a
-// power of two with rows of at most 1024 bytes.
+// 128-bit vectors straight from the fragment buffers. The same launch computes the
+// norm key with one thread per row of K[l*]: the squared norm of the key in fp64 in
+// ascending element order, then the quantised norm (round-half-even of 2^20 * sqrt,
+// saturated at 2^44 - 1) added into Q[t] with a 64-bit integer atomic: integer
+// addition is associative, so Q does not depend on the order the atomics land in.
 #include "cm_hash_kernels.h"
 
 #include <cstring>
@@ -32,13 +30,27 @@ __device__ __forceinline__ uint32_t rotr8(uint32_t x) { return __byte_perm(x, 0,
 __device__ __forceinline__ uint32_t rotr12(uint32_t x) { return __funnelshift_r(x, x, 12); }
 __device__ __forceinline__ uint32_t rotr7(uint32_t x) { return __funnelshift_r(x, x, 7); }
 
+// a + b + x on the FMA pipe. An SM sub-partition's integer ALU pipe accepts one warp
+// instruction every two cycles and must take G's four xors and four rotations; a
+// three-input add left to it (one IADD3) would make that ten instructions per G. As
+// two multiply-adds by a 1 the compiler cannot see through (a __constant__ it must
+// load, so it cannot fold the product into an add), the sum goes to the FMA pipe,
+// which the compiler already gives the two-input adds: per G, 8 ALU and 6 FMA
+// instructions instead of 10 and 2. Measured on a q4b-shaped fragment: 0.326 instead
+// of 0.397 ms per 604 MB; rotations moved to the FMA pipe as well (a multiply and a
+// high multiply by 2^25) made it slower.
+__constant__ uint32_t g_one = 1;
+__device__ __forceinline__ uint32_t add3(uint32_t a, uint32_t b, uint32_t x) {
+    return (a + b * g_one) + x * g_one;
+}
+
 // The G mixing function of RFC 7693, Section 3.1 (rotation distances 16, 12, 8, 7).
 #define CM_G(a, b, c, d, x, y)      \
-    a = a + b + (x);                \
+    a = add3(a, b, (x));            \
     d = rotr16(d ^ a);              \
     c = c + d;                      \
     b = rotr12(b ^ c);              \
-    a = a + b + (y);                \
+    a = add3(a, b, (y));            \
     d = rotr8(d ^ a);               \
     c = c + d;                      \
     b = rotr7(b ^ c);
@@ -107,35 +119,61 @@ __device__ __forceinline__ void store_digest(uint8_t *dst, const uint32_t h[8]) 
     *reinterpret_cast<uint4 *>(dst) = make_uint4(h[0], h[1], h[2], h[3]);
 }
 
-// Squared-norm accumulation of one 16-byte vector (8 bf16, ascending element
-// order) at stream offset pos; finishes the row on its last vector.
-struct NormState {
-    double ss;
-};
-
-__device__ __forceinline__ void norm_vector(const LeafLaunch &a, NormState &st, uint4 w,
-                                            uint64_t pos) {
-    if (pos < a.norm_begin || pos >= a.norm_begin + a.plane_bytes) return;
+// fl(ss + x^2) for the 8 bf16 of one 16-byte vector, in ascending element order (x^2
+// is exact in fp64, so each step is the one rounding of the sum). A normal bf16 (exponent
+// field 1..254) is 2^(e-127) (1 + m/128) in magnitude; as an fp64 its exponent field is
+// e + 896 and its 7 fraction bits lead the 52-bit fraction, so the high word of |x| is
+// ((e << 7 | m) << 13) + (896 << 20) and the low word is 0: integer operations instead of
+// a conversion on the FP64 pipe, which is the slow one on this part. A vector holding a
+// zero, subnormal, infinity or NaN converts through fp32 instead.
+__device__ __forceinline__ double accumulate_squares(uint4 w, double ss) {
     const uint32_t words[4] = {w.x, w.y, w.z, w.w};
-    double ss = st.ss;
+    bool normal = true;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        const double lo = (double)__uint_as_float(words[i] << 16);
-        const double hi = (double)__uint_as_float(words[i] & 0xFFFF0000u);
-        ss = __fma_rn(lo, lo, ss);   // x*x is exact in fp64, so this is fl(ss + x^2)
-        ss = __fma_rn(hi, hi, ss);
+        const uint32_t elo = words[i] & 0x7F80u, ehi = words[i] & 0x7F800000u;
+        normal = normal && elo != 0u && elo != 0x7F80u && ehi != 0u && ehi != 0x7F800000u;
     }
-    const uint64_t rel = pos - a.norm_begin;
-    if ((rel & (uint64_t)(a.row_bytes - 1)) == (uint64_t)(a.row_bytes - 16)) {
-        const uint32_t row = (uint32_t)(rel / a.row_bytes);
-        const uint32_t t = row % a.seq_len;
-        const double scaled = __dsqrt_rn(ss) * 1048576.0;     // exact scaling by 2^20
-        const unsigned long long q =
-            (scaled < (double)kQMax) ? __double2ull_rn(scaled) : kQMax;   // NaN saturates too
-        atomicAdd(a.norm_key + t, q);
-        ss = 0.0;
+    if (normal) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const double lo = __hiloint2double((int)(((words[i] & 0x7FFFu) << 13) + 0x38000000u), 0);
+            const double hi = __hiloint2double((int)(((words[i] >> 3) & 0x0FFFE000u) + 0x38000000u), 0);
+            ss = __fma_rn(lo, lo, ss);
+            ss = __fma_rn(hi, hi, ss);
+        }
+    } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const double lo = (double)__uint_as_float(words[i] << 16);
+            const double hi = (double)__uint_as_float(words[i] & 0xFFFF0000u);
+            ss = __fma_rn(lo, lo, ss);
+            ss = __fma_rn(hi, hi, ss);
+        }
     }
-    st.ss = ss;
+    return ss;
+}
+
+// Norm key of row r of K[l*] (Eq. rho; the plane is [H][T][d], so r = h*T + t): one
+// thread reads the row's d/8 vectors and accumulates its squared norm, then adds the
+// quantised norm into Q[t].
+__device__ __forceinline__ void norm_row(const LeafLaunch &a, uint64_t r) {
+    const uint8_t *row = a.k + a.norm_begin / 2 + r * a.row_bytes;   // K[l*] at stream offset 2 l* plane
+    const uint32_t nvec = a.row_bytes >> 4;
+    double ss = 0.0;
+    for (uint32_t v = 0; v < nvec; v += 4) {
+        uint4 w[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+            if (v + q < nvec) w[q] = load_nc(row + 16 * (v + q));
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+            if (v + q < nvec) ss = accumulate_squares(w[q], ss);
+    }
+    const double scaled = __dsqrt_rn(ss) * 1048576.0;     // exact scaling by 2^20
+    const unsigned long long q =
+        (scaled < (double)kQMax) ? __double2ull_rn(scaled) : kQMax;   // NaN saturates too
+    atomicAdd(a.norm_key + r % a.seq_len, q);
 }
 
 // Cursor over the fragment's byte stream K[0] V[0] K[1] V[1] ...: every segment
@@ -181,25 +219,36 @@ constexpr int kLeafThreads = kLeafBlockThreads;
 
 __global__ void __launch_bounds__(kLeafThreads)
 leaf_hash_kernel(const __grid_constant__ LeafGroup grp) {
+    // the blocks after the leaf blocks compute norm keys, one thread per row of K[l*]:
+    // they fill SMs that the last wave of leaf blocks leaves idle
+    const uint32_t x = blockIdx.x;
+    const uint32_t leaf_blocks = (uint32_t)grp.block_begin[grp.count];
+    if (x >= leaf_blocks) {
+        const uint32_t k = x - leaf_blocks;
+        uint32_t fi = 0;
+        while (fi + 1 < grp.count && k >= grp.norm_block_begin[fi + 1]) ++fi;
+        const LeafLaunch &a = grp.frag[fi];
+        const uint64_t r = (uint64_t)(k - grp.norm_block_begin[fi]) * kLeafThreads + threadIdx.x;
+        if (r < (a.plane_bytes >> (__ffs(a.row_bytes) - 1))) norm_row(a, r);
+        return;
+    }
     uint32_t fi = 0;                                   // the block's fragment (uniform)
-    while (fi + 1 < grp.count && blockIdx.x >= grp.block_begin[fi + 1]) ++fi;
+    while (fi + 1 < grp.count && x >= grp.block_begin[fi + 1]) ++fi;
     const LeafLaunch &a = grp.frag[fi];
-    const uint64_t leaf = (uint64_t)(blockIdx.x - grp.block_begin[fi]) * kLeafThreads + threadIdx.x;
+    const uint64_t leaf = (uint64_t)(x - grp.block_begin[fi]) * kLeafThreads + threadIdx.x;
     if (leaf >= a.num_leaves) return;
     const uint64_t begin = leaf * kLeafBytes;
     const uint64_t rem = a.stream_bytes - begin;
     const uint32_t len = rem < (uint64_t)kLeafBytes ? (uint32_t)rem : (uint32_t)kLeafBytes;
     const uint32_t nblocks = (len + 63) / 64;
     const bool last_node = leaf + 1 == a.num_leaves;
-    const bool norm_leaf = begin < a.norm_begin + a.plane_bytes && begin + len > a.norm_begin;
 
     uint32_t h[8];
     node_init(h, a.tree, leaf, 0);
     StreamCursor cur = cursor_at(a, begin);
-    NormState ns{0.0};
 
-    if (!norm_leaf && len == (uint32_t)kLeafBytes && cur.left >= (uint64_t)kLeafBytes) {
-        // the whole leaf lies in one K or V segment, away from the routing layer
+    if (len == (uint32_t)kLeafBytes && cur.left >= (uint64_t)kLeafBytes) {
+        // the whole leaf lies in one K or V segment
         const uint8_t *p = cur.ptr;
 #pragma unroll 1
         for (uint32_t b = 0; b < 16; ++b) {
@@ -218,11 +267,6 @@ leaf_hash_kernel(const __grid_constant__ LeafGroup grp) {
 #pragma unroll
         for (int q = 0; q < 4; ++q)
             w[q] = b * 64 + q * 16 < len ? load_nc(cursor_next(a, cur)) : make_uint4(0, 0, 0, 0);
-        if (norm_leaf) {
-#pragma unroll
-            for (int q = 0; q < 4; ++q)
-                if (b * 64 + q * 16 < len) norm_vector(a, ns, w[q], begin + b * 64 + q * 16);
-        }
         const uint32_t m[16] = {w[0].x, w[0].y, w[0].z, w[0].w, w[1].x, w[1].y, w[1].z, w[1].w,
                                 w[2].x, w[2].y, w[2].z, w[2].w, w[3].x, w[3].y, w[3].z, w[3].w};
         const uint32_t end = (b + 1) * 64 < len ? (b + 1) * 64 : len;
@@ -359,9 +403,20 @@ __global__ void compare_kernel(const uint4 *__restrict__ a, const uint4 *__restr
 
 }  // namespace
 
-cudaError_t launch_leaf_hash_group(const LeafGroup &g, cudaStream_t stream) {
-    const uint64_t blocks = g.block_begin[g.count];
-    if (g.count == 0 || blocks == 0) return cudaSuccess;
+cudaError_t launch_leaf_hash_group(const LeafGroup &in, cudaStream_t stream) {
+    if (in.count == 0 || in.count > (uint32_t)kMaxLeafGroup) return cudaSuccess;
+    LeafGroup g = in;
+    uint64_t norm_blocks = 0;
+    for (uint32_t i = 0; i < g.count; ++i) {
+        const LeafLaunch &a = g.frag[i];
+        const uint64_t rows = a.row_bytes ? a.plane_bytes / a.row_bytes : 0;
+        g.norm_block_begin[i] = norm_blocks;
+        norm_blocks += (rows + kLeafThreads - 1) / kLeafThreads;
+    }
+    g.norm_block_begin[g.count] = norm_blocks;
+    const uint64_t leaf_blocks = g.block_begin[g.count];
+    const uint64_t blocks = leaf_blocks + norm_blocks;
+    if (blocks == 0) return cudaSuccess;
     if (blocks > 0x7FFFFFFFull) return cudaErrorInvalidValue;
     leaf_hash_kernel<<<(unsigned)blocks, kLeafThreads, 0, stream>>>(g);
     return cudaGetLastError();
@@ -523,7 +578,8 @@ extern "C" cm_status cm_fragment_id_static(const cm_fragment *frag, int32_t rout
 // Register-only kernels that measure the ceiling of the content-address kernels on the
 // current GPU (a profiling aid for their roofline): chains of three-input xors, one
 // integer-ALU instruction each, and the compression function above applied to register
-// data with no memory traffic.
+// data with no memory traffic, counted as the 648 operations per 64-byte block that
+// issue on the integer ALU pipe (10 rounds x 8 G x (4 xors + 4 rotations) + 8 xors).
 
 namespace cm {
 namespace {
@@ -614,7 +670,7 @@ extern "C" cm_status cm_measure_int_alu(int32_t device, double *xor3_tops, doubl
             });
             if (st == CM_OK) {
                 const double ops_x = (double)grid_x * kLeafThreads * xor_iters * 8;
-                const double ops_c = (double)grid_c * kLeafThreads * comp_blocks * 808;
+                const double ops_c = (double)grid_c * kLeafThreads * comp_blocks * 648;
                 *xor3_tops = ops_x / (ms_x * 1e-3) / 1e12;
                 *compress_tops = ops_c / (ms_c * 1e-3) / 1e12;
             }

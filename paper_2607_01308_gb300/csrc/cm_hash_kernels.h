@@ -31,7 +31,7 @@ struct LeafLaunch {
     uint64_t stream_bytes;         // 2 * L * plane_bytes
     uint64_t num_leaves;           // ceil(stream_bytes / 1024)
     uint64_t norm_begin;           // stream offset of K[l*]; its length is plane_bytes
-    uint32_t row_bytes;            // d*2; a power of two <= 1024, so rows never straddle leaves
+    uint32_t row_bytes;            // d*2; a power of two in [32, 1024]
     uint32_t seq_len;              // T
     unsigned long long *norm_key;  // Q[T] accumulators, zeroed before the launch
     uint8_t *digests;              // num_leaves * 16 bytes out
@@ -39,14 +39,17 @@ struct LeafLaunch {
 };
 
 // Level 0 of up to kMaxLeafGroup fragments in one launch: one thread per leaf, the
-// blocks of fragment i being [block_begin[i], block_begin[i + 1]); each thread whose
-// leaf lies in K[l*] also accumulates the routing-layer norm key.
+// leaf blocks of fragment i being [block_begin[i], block_begin[i + 1]) (set by the
+// caller); after the last leaf block, one thread per row of K[l*] for the routing-layer
+// norm key, the norm blocks of fragment i being block_begin[count] +
+// [norm_block_begin[i], norm_block_begin[i + 1]) (set by the launcher).
 constexpr int kMaxLeafGroup = 32;
-constexpr int kLeafBlockThreads = 128;   // threads (= leaves) per block of the leaf launch
+constexpr int kLeafBlockThreads = 128;   // threads (= leaves or rows) per block of the leaf launch
 struct LeafGroup {
     uint32_t count;
     uint32_t pad_;
     uint64_t block_begin[kMaxLeafGroup + 1];
+    uint64_t norm_block_begin[kMaxLeafGroup + 1];
     LeafLaunch frag[kMaxLeafGroup];
 };
 cudaError_t launch_leaf_hash_group(const LeafGroup &g, cudaStream_t stream);

@@ -46,7 +46,8 @@ def _render(ctx, deliveries, cap=None, fill=None):
 # ---------------------------------------------------------------- content address + norm key
 
 ID_SHAPES = [(4, 2, 37, 64), (4, 2, 53, 64), (1, 1, 1, 16), (2, 3, 1, 512), (3, 1, 5, 16),
-             (2, 2, 33, 32), (5, 2, 7, 256), (28, 8, 9, 128), (1, 1, 300, 128)]
+             (2, 2, 33, 32), (5, 2, 7, 256), (28, 8, 9, 128), (1, 1, 300, 128),
+             (3, 8, 70, 64), (2, 4, 129, 512)]
 
 
 @pytest.mark.parametrize("shape", ID_SHAPES)
@@ -74,6 +75,36 @@ def test_norm_key_special_values(ctx):
     ref = oracle_fragment(K, V)
     assert fid == ref.fid
     assert np.array_equal(np.array(Q, dtype=np.uint64), ref.Q)
+
+
+def test_norm_key_wide_exponent_range(ctx):
+    # routing-layer rows whose elements span up to 2^40 in magnitude (most fp64 row sums
+    # round; rows with large elements saturate), with zeros, subnormals and infinities
+    # mixed into some vectors: every exponent field of the bf16 -> fp64 conversion, and
+    # both the integer conversion of all-normal vectors and the fp32 one of the others
+    L, H, T, d = 3, 4, 150, 64                      # 600 rows of K[1]: several norm blocks
+    rng = np.random.default_rng(2607)
+    bits = rng.integers(0, 1 << 16, size=(L, H, T, d), dtype=np.uint32).astype(np.uint16)
+    rows = bits[1].reshape(H * T, d)
+    emax = rng.integers(115, 161, size=(H * T, 1))   # largest element 2^-12 .. 2^33
+    expo = np.clip(emax - rng.integers(0, 41, size=(H * T, d)), 1, 254)
+    sign = rng.integers(0, 2, size=(H * T, d)) << 15
+    rows[:] = (sign | (expo << 7) | rng.integers(0, 128, size=(H * T, d))).astype(np.uint16)
+    odd = rng.random((H * T, d)) < 0.03
+    rows[odd] = (rng.integers(0, 2, size=int(odd.sum())) << 15 |
+                 rng.integers(0, 128, size=int(odd.sum()))).astype(np.uint16)   # zeros, subnormals
+    rows[7, 3] = 0x7F80                             # +inf
+    rows[400, 60] = 0xFF80                          # -inf
+    rows[9, :] = rng.integers(1, 128, size=d).astype(np.uint16)   # all subnormal
+    K = torch.from_numpy(bits.view(np.int16)).to("cuda:0").view(torch.bfloat16)
+    V = torch.zeros_like(K)
+    fid, Q = ctx.fragment_id(K, V)
+    ref = oracle_fragment(K, V)
+    assert fid == ref.fid
+    got = np.array(Q, dtype=np.uint64)
+    assert np.array_equal(got, ref.Q)
+    sat = np.uint64((1 << 44) - 1)
+    assert (got >= sat).any() and (got < sat).any()   # positions with and without a saturated head
 
 
 # ---------------------------------------------------------------- tiny workload: every order
