@@ -70,7 +70,7 @@ def parse_args():
                         "re-deliveries) instead of the single-merge benchmark")
     p.add_argument("--group", type=int, default=8,
                    help="serving sweep: requests per cm_ingest_many / cm_render_many call")
-    p.add_argument("--workload", default=WORKLOAD, choices=["q4b", "q4b_t512", "q17_n2", "tiny"],
+    p.add_argument("--workload", default=WORKLOAD, choices=["q4b", "q4b_t512", "q4b_t2048", "q17_n2", "tiny"],
                    help="single-request workload (q4b is the benchmark; the others are small "
                         "cases for profiling)")
     return p.parse_args()
@@ -81,6 +81,8 @@ WORKLOAD_TEXT = {
            "N=4 fragments x 4096 tokens (16384 merged tokens), bf16",
     "q4b_t512": "Qwen3-4B-shaped merge, short fragments: 36 layers, 8 KV heads, head_dim 128, "
                 "RoPE theta 1e6, N=4 fragments x 512 tokens, bf16",
+    "q4b_t2048": "Qwen3-4B-shaped merge, mid-length fragments: 36 layers, 8 KV heads, head_dim 128, "
+                 "RoPE theta 1e6, N=4 fragments x 2048 tokens, bf16",
     "q17_n2": "Qwen3-1.7B-shaped merge: 28 layers, 8 KV heads, head_dim 128, RoPE theta 1e6, "
               "N=2 fragments x 512 tokens, bf16",
     "tiny": "tiny merge: 4 layers, 2 KV heads, head_dim 64, fragments of 37 and 53 tokens, bf16",

@@ -341,7 +341,8 @@ cm_status cm_context_set_render_warps(cm_context *ctx, int32_t warps);
 typedef struct cm_kernel_times {
     double leaf_hash_ms;          /* content address, level 0 (one launch per up to 32 fragments) */
     int64_t leaf_hash_launches;
-    double inner_hash_ms;         /* content address, tree levels above the leaves */
+    double inner_hash_ms;         /* content address, tree levels above the leaves (level 1,
+                                     then the levels above it: two kernels per call) */
     int64_t inner_hash_launches;
     double render_ms;             /* render / BagMerge */
     int64_t render_launches;

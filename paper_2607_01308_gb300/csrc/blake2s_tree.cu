@@ -361,6 +361,48 @@ __device__ __forceinline__ uint32_t arrive_acq_rel(uint32_t *counter) {
     return old;
 }
 
+constexpr int kLevel1Threads = 128;
+
+// Level 1 of up to kMaxGroup fragments: one thread per node (node_begin: prefix sums of
+// the level-1 sizes), its children read straight into registers. Every lane of a warp
+// hashes a node, and with no shared memory many warps fit on an SM.
+__global__ void __launch_bounds__(kLevel1Threads)
+level1_kernel(const __grid_constant__ TreeTop t) {
+    const uint64_t g = (uint64_t)blockIdx.x * kLevel1Threads + threadIdx.x;
+    if (g >= t.node_begin[t.count]) return;
+    uint32_t fi = 0;
+    while (fi + 1 < t.count && g >= t.node_begin[fi + 1]) ++fi;
+    const TreeTopFragment &f = t.frag[fi];
+    const uint64_t j = g - t.node_begin[fi];
+    const uint64_t first = j * kFanout;
+    const uint64_t nc64 = f.size[0] - first;
+    const uint32_t nc = nc64 < (uint64_t)kFanout ? (uint32_t)nc64 : (uint32_t)kFanout;
+    const uint32_t len = nc * kDigestBytes;
+    const uint32_t nblocks = (len + 63) / 64;
+    const bool last_node = j + 1 == f.size[1];
+    const uint8_t *src = f.level[0] + first * kDigestBytes;
+    uint32_t h[8];
+    node_init(h, f.tree, j, 1);
+#pragma unroll 1
+    for (uint32_t b = 0; b < nblocks; ++b) {
+        uint4 w[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const uint32_t off = b * 64 + q * 16;
+            w[q] = off < len ? load_nc(src + off) : make_uint4(0, 0, 0, 0);
+        }
+        const uint32_t m[16] = {w[0].x, w[0].y, w[0].z, w[0].w, w[1].x, w[1].y, w[1].z, w[1].w,
+                                w[2].x, w[2].y, w[2].z, w[2].w, w[3].x, w[3].y, w[3].z, w[3].w};
+        const uint32_t end = (b + 1) * 64 < len ? (b + 1) * 64 : len;
+        compress(h, m, end, b + 1 == nblocks, last_node);
+    }
+    store_digest(f.level[1] + j * kDigestBytes, h);
+}
+
+// Levels kStart and up (node_begin: prefix sums of the level-kStart sizes, 0 for a
+// fragment without that level): one thread per level-kStart node hashes it; then,
+// level by level, the thread that completes a parent's last child hashes the parent.
+template <int kStart>
 __global__ void __launch_bounds__(kInnerThreads)
 tree_top_kernel(const __grid_constant__ TreeTop t) {
     __shared__ uint4 stage_all[kInnerThreads][16];
@@ -371,8 +413,8 @@ tree_top_kernel(const __grid_constant__ TreeTop t) {
     while (fi + 1 < t.count && g >= t.node_begin[fi + 1]) ++fi;
     const TreeTopFragment &f = t.frag[fi];
     uint64_t j = g - t.node_begin[fi];
-    uint32_t len = stage_children<false>(stage, f.level[0], f.size[0], j);
-    for (uint32_t k = 1;; ++k) {
+    uint32_t len = stage_children<false>(stage, f.level[kStart - 1], f.size[kStart - 1], j);
+    for (uint32_t k = kStart;; ++k) {
         hash_node_from(stage, len, f.level[k], j, f.size[k], k, f.tree);
         if (k + 1 >= f.levels) break;
         // this thread finished node j of level k; the one that finishes the last child of
@@ -441,11 +483,36 @@ cudaError_t launch_inner_hash(const uint8_t *children, uint64_t num_children, ui
     return cudaGetLastError();
 }
 
+int tree_top_kernels(const TreeTop &t) {
+    if (t.count == 0 || t.count > (uint32_t)kMaxGroup || t.node_begin[t.count] == 0) return 0;
+    if (t.node_begin[t.count] < kSplitLevel1Nodes) return 1;
+    for (uint32_t i = 0; i < t.count; ++i)
+        if (t.frag[i].levels >= 3) return 2;
+    return 1;
+}
+
 cudaError_t launch_tree_top(const TreeTop &t, cudaStream_t stream) {
-    const uint64_t total = t.node_begin[t.count];
-    if (total == 0) return cudaSuccess;
-    const uint64_t blocks = (total + kInnerThreads - 1) / kInnerThreads;
-    tree_top_kernel<<<(unsigned)blocks, kInnerThreads, 0, stream>>>(t);
+    if (t.count == 0 || t.count > (uint32_t)kMaxGroup) return cudaSuccess;
+    const uint64_t total1 = t.node_begin[t.count];
+    if (total1 == 0) return cudaSuccess;
+    if (total1 < kSplitLevel1Nodes) {
+        // one launch from level 1: the level-2 parents are hashed by the threads that
+        // finish their last child, with no second launch
+        tree_top_kernel<1><<<(unsigned)((total1 + kInnerThreads - 1) / kInnerThreads),
+                             kInnerThreads, 0, stream>>>(t);
+        return cudaGetLastError();
+    }
+    level1_kernel<<<(unsigned)((total1 + kLevel1Threads - 1) / kLevel1Threads), kLevel1Threads, 0,
+                    stream>>>(t);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    TreeTop u = t;   // the same fragments, counted by their level-2 nodes
+    for (uint32_t i = 0; i < u.count; ++i)
+        u.node_begin[i + 1] = u.node_begin[i] + (u.frag[i].levels >= 3 ? u.frag[i].size[2] : 0);
+    const uint64_t total2 = u.node_begin[u.count];
+    if (total2 == 0) return cudaSuccess;
+    tree_top_kernel<2><<<(unsigned)((total2 + kInnerThreads - 1) / kInnerThreads), kInnerThreads,
+                         0, stream>>>(u);
     return cudaGetLastError();
 }
 

@@ -64,10 +64,15 @@ cudaError_t launch_inner_hash(const uint8_t *children, uint64_t num_children, ui
 
 constexpr int kMaxGroup = 32;
 
-// Every tree level above the leaves, for up to kMaxGroup fragments, in one launch.
-// One thread per level-1 node hashes it; then, level by level, the thread that
-// completes a parent's last child (a per-node arrival counter, zeroed before the
-// launch) hashes that parent, up to the root. No thread ever waits for another.
+// Every tree level above the leaves, for up to kMaxGroup fragments. One thread per
+// level-s node hashes it; then, level by level, the thread that completes a parent's
+// last child (a per-node arrival counter, zeroed before the launch) hashes that parent,
+// up to the root. No thread ever waits for another. With fewer than kSplitLevel1Nodes
+// level-1 nodes in all, one launch with s = 1. With more, a first launch hashes level 1
+// with every lane of a warp busy and many warps per SM, and a second runs the scheme
+// above with s = 2 (in one launch, each warp would hash 32 level-1 nodes and then two
+// level-2 parents with two of its lanes). The caller sets node_begin from the level-1
+// sizes.
 constexpr int kMaxLevels = 12;
 struct TreeTopFragment {
     uint8_t *level[kMaxLevels];       // digests of level k; level[levels - 1] is the root
@@ -78,10 +83,12 @@ struct TreeTopFragment {
 };
 struct TreeTop {
     uint32_t count;
-    uint64_t node_begin[kMaxGroup + 1];   // prefix sum of the fragments' level-1 sizes
+    uint64_t node_begin[kMaxGroup + 1];   // prefix sum of the fragments' level-1 sizes (level 2 in the second launch)
     TreeTopFragment frag[kMaxGroup];
 };
+constexpr uint64_t kSplitLevel1Nodes = 32768;
 cudaError_t launch_tree_top(const TreeTop &t, cudaStream_t stream);
+int tree_top_kernels(const TreeTop &t);   // kernels launch_tree_top launches for t
 
 // *flag |= 1 if the `bytes` bytes at a and b differ (16-byte aligned, bytes % 16 == 0).
 cudaError_t launch_compare(const void *a, const void *b, uint64_t bytes, unsigned int *flag,

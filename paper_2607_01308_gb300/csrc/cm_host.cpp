@@ -135,6 +135,7 @@ struct cm_context {
     struct Pending {
         int kind;
         cudaEvent_t start, end;
+        int kernels;   // kernels launched between the two events
     };
     std::vector<Pending> pending;
     std::vector<cudaEvent_t> event_pool;
@@ -271,23 +272,25 @@ cudaEvent_t take_event(cm_context *ctx) {
     return e;
 }
 
-// Runs `launch` on `stream`; when timing is on, brackets it with two events.
+// Runs `launch` (which launches `kernels` kernels) on `stream`; when timing is on,
+// brackets it with two events.
 template <class F>
-cudaError_t timed_launch(cm_context *ctx, int kind, cudaStream_t stream, F &&launch) {
+cudaError_t timed_launch(cm_context *ctx, int kind, cudaStream_t stream, F &&launch,
+                         int kernels = 1) {
     if (!ctx->timing) return launch();
     cudaEvent_t a = take_event(ctx), b = take_event(ctx);
     if (!a || !b) return launch();
     cudaEventRecord(a, stream);
     const cudaError_t e = launch();
     cudaEventRecord(b, stream);
-    ctx->pending.push_back({kind, a, b});
+    ctx->pending.push_back({kind, a, b, kernels});
     return e;
 }
 
 // Id(C) and Q[t] of n fragments in one pass: the leaf-hash launches of all
-// fragments, then one grouped launch per tree level (up to kMaxGroup fragments
-// each), then a single copy of every root digest and norm key to the host and one
-// synchronisation. Caller holds ctx->mu and the device scope.
+// fragments (with their norm keys), then the tree levels above the leaves (level 1,
+// then the levels above it: two launches per kMaxGroup fragments), then a single copy
+// of every root digest and norm key to the host and one synchronisation. Caller holds ctx->mu and the device scope.
 //   device scratch: [roots n x 16][Q of fragment 0]...[Q of fragment n-1][levels...]
 cm_status fragments_digest(cm_context *ctx, const cm_fragment *const *frags, size_t n,
                            cudaStream_t stream, cm_id *ids, std::vector<uint64_t> *Qs) {
@@ -375,8 +378,9 @@ cm_status fragments_digest(cm_context *ctx, const cm_fragment *const *frags, siz
     std::memset(top.get(), 0, sizeof(cm::TreeTop));
     auto flush = [&]() -> cudaError_t {
         if (top->count == 0) return cudaSuccess;
-        const cudaError_t e =
-            timed_launch(ctx, kTimeInner, stream, [&] { return cm::launch_tree_top(*top, stream); });
+        const int kernels = cm::tree_top_kernels(*top);
+        const cudaError_t e = timed_launch(
+            ctx, kTimeInner, stream, [&] { return cm::launch_tree_top(*top, stream); }, kernels);
         std::memset(top.get(), 0, sizeof(cm::TreeTop));
         return e;
     };
@@ -1045,7 +1049,7 @@ cm_status cm_context_kernel_times(cm_context *ctx, cm_kernel_times *out, int32_t
             CM_CUDA_TRY(cudaEventSynchronize(pe.end), "timing event");
             CM_CUDA_TRY(cudaEventElapsedTime(&ms, pe.start, pe.end), "timing event");
             ctx->time_ms[pe.kind] += ms;
-            ctx->launches[pe.kind] += 1;
+            ctx->launches[pe.kind] += pe.kernels;
             ctx->event_pool.push_back(pe.start);
             ctx->event_pool.push_back(pe.end);
         }

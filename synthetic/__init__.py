@@ -18,6 +18,8 @@ Workloads (shapes of the paper's Qwen3-1.7B / Qwen3-4B caches, Section 5.8):
   q17_arity  L=28, H=8, d=128, N=5, T ~ U{256..2048}, 8 deliveries (3 duplicates)
   q4b        L=36, H=8, d=128, N=4 x T=4096, scale U(0.5,1.5)
   q4b_t512   the q4b shape with T=512 per fragment (302 MB of inputs): profiling case
+  q4b_t2048  the q4b shape with T=2048 per fragment (1.2 GB of inputs): profiling case
+             large enough for the two-kernel tree top (73,728 level-1 nodes)
   serve      q4b shape, 64 requests x N=3, T ~ U{512..4096}, each delivery
              re-sent with probability 0.1, shuffled per request
 
@@ -69,6 +71,7 @@ WORKLOADS = {
     "q17_arity": Workload("q17_arity", 28, 8, 128, 5, length_range=(256, 2048), num_dups=3),
     "q4b": Workload("q4b", 36, 8, 128, 4, lengths=(4096, 4096, 4096, 4096)),
     "q4b_t512": Workload("q4b_t512", 36, 8, 128, 4, lengths=(512, 512, 512, 512)),
+    "q4b_t2048": Workload("q4b_t2048", 36, 8, 128, 4, lengths=(2048, 2048, 2048, 2048)),
     "serve": Workload("serve", 36, 8, 128, 3, length_range=(512, 4096), num_requests=64,
                       dup_prob=0.1),
 }

@@ -72,7 +72,13 @@ def test_q4b_full_size_bench_configuration(ctx):
              for sp in specs]
     A, B = cm.FragmentSet(ctx), cm.FragmentSet(ctx)
     # the bench's launch configuration: one cm_ingest_many call feeds both replicas
+    cm.cm_context_kernel_times(ctx.handle, reset=True)
+    cm.cm_context_set_timing(ctx.handle, True)
     res = cm.ingest_many([(A, *frags[0]), (A, *frags[1]), (B, *frags[2]), (B, *frags[3])])
+    cm.cm_context_set_timing(ctx.handle, False)
+    t = cm.cm_context_kernel_times(ctx.handle, reset=True)
+    # 4 x 36,864 level-1 nodes: level 1 in its own kernel, then the levels above it
+    assert t["leaf_hash_launches"] == 1 and t["inner_hash_launches"] == 2
     ra, rb = res[:2], res[2:]
     A.union(B)
     total = sum(sp.seq_len for sp in specs)
@@ -88,6 +94,28 @@ def test_q4b_full_size_bench_configuration(ctx):
     _check_sampled_planes(frags, order, k_out, v_out, layers=[0, 18, 35], heads=[0, 7])
     A.close()
     B.close()
+
+
+def test_split_tree_top_with_roots_at_levels_one_and_two(ctx):
+    # one call whose level-1 nodes are enough for the two-kernel tree top, with a
+    # fragment whose root is level 1 and one whose root is level 2 beside a full one
+    w = synthetic.WORKLOADS["q4b"]
+    big = synthetic.make_fragment_torch(synthetic.fragment_specs(w)[0], w.num_layers,
+                                        w.num_kv_heads, w.head_dim, "cuda:0")
+    g = torch.Generator(device="cuda:0").manual_seed(1716)
+    small = [tuple(torch.randn((1, 1, T, 16), generator=g, device="cuda:0").to(torch.bfloat16)
+                   for _ in range(2)) for T in (3, 257)]          # 1 and 17 leaves
+    sets = [cm.FragmentSet(ctx) for _ in range(3)]
+    cm.cm_context_kernel_times(ctx.handle, reset=True)
+    cm.cm_context_set_timing(ctx.handle, True)
+    res = cm.ingest_many([(sets[0], *small[0]), (sets[1], *big), (sets[2], *small[1])])
+    cm.cm_context_set_timing(ctx.handle, False)
+    t = cm.cm_context_kernel_times(ctx.handle, reset=True)
+    assert t["inner_hash_launches"] == 2
+    want = [fragment_id(synthetic.to_bits(K), synthetic.to_bits(V)) for K, V in (small[0], big, small[1])]
+    assert [fid for fid, _ in res] == want
+    for S in sets:
+        S.close()
 
 
 @pytest.mark.parametrize("request_index", [0, 1])
@@ -218,7 +246,7 @@ def test_kernel_timing_counts_every_launch(ctx):
     cm.cm_context_set_timing(ctx.handle, False)
     t = cm.cm_context_kernel_times(ctx.handle, reset=True)
     assert t["leaf_hash_launches"] == 1 and t["leaf_hash_fragments"] == 3   # one grouped launch
-    assert t["inner_hash_launches"] == 1
+    assert t["inner_hash_launches"] == 1            # few level-1 nodes: one tree-top kernel
     assert t["render_launches"] == 1
     assert t["aux_launches"] == 1                  # the ingest's result readback
     assert t["leaf_hash_ms"] > 0 and t["render_ms"] > 0

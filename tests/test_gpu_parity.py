@@ -309,7 +309,34 @@ def test_union_algebra_and_render_invariance(ctx):
 
 # ---------------------------------------------------------------- launch-group boundaries
 
-def test_forty_fragments_span_two_render_and_two_tree_launches(ctx):
+def test_roots_at_level_one_and_two(ctx):
+    # 64 T bytes per fragment: T <= 256 gives at most 16 leaves, so level 1 is the root;
+    # T = 257 has 17 leaves and its root at level 2 (one tree-top kernel per call: few
+    # level-1 nodes)
+    L, H, d = 1, 1, 16
+    g = torch.Generator(device="cuda:0").manual_seed(16)
+    frags = [(torch.randn((L, H, T, d), generator=g, device="cuda:0").to(torch.bfloat16),
+              torch.randn((L, H, T, d), generator=g, device="cuda:0").to(torch.bfloat16))
+             for T in (1, 15, 16, 17, 255, 256)]
+    cm.cm_context_kernel_times(ctx.handle, reset=True)
+    cm.cm_context_set_timing(ctx.handle, True)
+    S = cm.FragmentSet(ctx)
+    res = S.ingest_batch(frags)
+    cm.cm_context_set_timing(ctx.handle, False)
+    t = cm.cm_context_kernel_times(ctx.handle, reset=True)
+    assert t["inner_hash_launches"] == 1
+    assert [r[0] for r in res] == [oracle_fragment(K, V).fid for K, V in frags]
+    K, V = (torch.randn((L, H, 257, d), generator=g, device="cuda:0").to(torch.bfloat16)
+            for _ in range(2))
+    cm.cm_context_set_timing(ctx.handle, True)
+    fid, _ = S.ingest(K, V)
+    cm.cm_context_set_timing(ctx.handle, False)
+    t = cm.cm_context_kernel_times(ctx.handle, reset=True)
+    assert t["inner_hash_launches"] == 1 and fid == oracle_fragment(K, V).fid
+    S.close()
+
+
+def test_forty_fragments_span_two_render_and_two_tree_top_calls(ctx):
     # more fragments than one render launch (32 slots) or one tree-top launch (32) holds
     L, H, d = 2, 1, 64
     g = torch.Generator(device="cuda:0").manual_seed(40)
@@ -328,6 +355,7 @@ def test_forty_fragments_span_two_render_and_two_tree_launches(ctx):
     n, order = S.render(k_out, v_out)
     cm.cm_context_set_timing(ctx.handle, False)
     t = cm.cm_context_kernel_times(ctx.handle, reset=True)
+    # two tree-top calls (32 + 8 fragments), one kernel each (few level-1 nodes)
     assert t["render_launches"] == 2 and t["inner_hash_launches"] == 2
     assert t["leaf_hash_launches"] == 2 and t["leaf_hash_fragments"] == 40
     ref_frags = [oracle_fragment(K, V) for K, V in frags]
