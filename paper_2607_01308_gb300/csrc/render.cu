@@ -390,7 +390,7 @@ __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const fl
         s[e] = __fadd_rn(t.z, t.w);
     }
     const uint4 *src = reinterpret_cast<const uint4 *>(buf);
-#pragma unroll 2
+#pragma unroll 1
     for (int q = lane; q < n_pairs; q += 32) {
         const int row = q >> p.log2_pairs_per_row;
         const int off = row * vecs_per_row + lane_v;
