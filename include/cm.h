@@ -153,9 +153,10 @@ cm_status cm_ingest(cm_set *set, const cm_fragment *frag, cm_stream_t stream, cm
                     int32_t *out_absorbed);
 
 /* Ingest of n deliveries in order (Algorithm 2, Ingest, applied n times): the same
- * result as n calls of cm_ingest, with one pass of GPU work for all of them (one
- * leaf-hash launch and one launch for the tree levels above the leaves per 32
- * fragments) and a single synchronisation of `stream`. A delivery whose id is
+ * result as n calls of cm_ingest, with one pass of GPU work for all of them (per 32
+ * fragments one leaf-hash launch, which also computes the norm keys, and one or two
+ * launches for the tree levels above the leaves) and a single synchronisation of
+ * `stream`. A delivery whose id is
  * already in the set, or equal to an earlier delivery of the same batch, is
  * absorbed. All fragments must have the set's shape (or one common shape if the
  * set is empty). Nothing is inserted if validation fails.
@@ -341,8 +342,9 @@ cm_status cm_context_set_render_warps(cm_context *ctx, int32_t warps);
 typedef struct cm_kernel_times {
     double leaf_hash_ms;          /* content address, level 0 (one launch per up to 32 fragments) */
     int64_t leaf_hash_launches;
-    double inner_hash_ms;         /* content address, tree levels above the leaves (level 1,
-                                     then the levels above it: two kernels per call) */
+    double inner_hash_ms;         /* content address, tree levels above the leaves (one
+                                     kernel per call, or two when the call has 32,768 or
+                                     more level-1 nodes: level 1, then the levels above) */
     int64_t inner_hash_launches;
     double render_ms;             /* render / BagMerge */
     int64_t render_launches;
