@@ -446,7 +446,8 @@ __global__ void compare_kernel(const uint4 *__restrict__ a, const uint4 *__restr
 }  // namespace
 
 cudaError_t launch_leaf_hash_group(const LeafGroup &in, cudaStream_t stream) {
-    if (in.count == 0 || in.count > (uint32_t)kMaxLeafGroup) return cudaSuccess;
+    if (in.count > (uint32_t)kMaxLeafGroup) return cudaErrorInvalidValue;
+    if (in.count == 0) return cudaSuccess;
     LeafGroup g = in;
     uint64_t norm_blocks = 0;
     for (uint32_t i = 0; i < g.count; ++i) {
@@ -492,7 +493,8 @@ int tree_top_kernels(const TreeTop &t) {
 }
 
 cudaError_t launch_tree_top(const TreeTop &t, cudaStream_t stream) {
-    if (t.count == 0 || t.count > (uint32_t)kMaxGroup) return cudaSuccess;
+    if (t.count > (uint32_t)kMaxGroup) return cudaErrorInvalidValue;
+    if (t.count == 0) return cudaSuccess;
     const uint64_t total1 = t.node_begin[t.count];
     if (total1 == 0) return cudaSuccess;
     if (total1 < kSplitLevel1Nodes) {
