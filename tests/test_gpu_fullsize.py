@@ -118,6 +118,41 @@ def test_split_tree_top_with_roots_at_levels_one_and_two(ctx):
         S.close()
 
 
+def test_redelivery_fast_path_at_full_size():
+    # two q4b fragments, each also delivered as a byte-identical clone in its own buffer,
+    # into one set with the re-delivery fast path on: the clones take their originals'
+    # ids without being hashed (full 604 MB byte comparisons), and the set and its render
+    # are the oracle's
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    w = synthetic.WORKLOADS["q4b"]
+    specs = synthetic.fragment_specs(w)[:2]
+    frags = [synthetic.make_fragment_torch(sp, w.num_layers, w.num_kv_heads, w.head_dim, "cuda:0")
+             for sp in specs]
+    clones = [(K.clone(), V.clone()) for K, V in frags]
+    c = cm.Context(0, THETA)
+    cm.cm_context_set_dedup_by_bytes(c.handle, True)
+    S = cm.FragmentSet(c)
+    cm.cm_context_kernel_times(c.handle, reset=True)
+    cm.cm_context_set_timing(c.handle, True)
+    res = S.ingest_batch([frags[0], clones[1], clones[0], frags[1]])
+    cm.cm_context_set_timing(c.handle, False)
+    t = cm.cm_context_kernel_times(c.handle, reset=True)
+    assert [a for _, a in res] == [False, False, True, True]
+    assert t["leaf_hash_fragments"] == 2           # the first delivery of each fragment only
+    keys = _oracle_keys(frags, w.num_layers // 2)
+    assert [fid for fid, _ in res] == [keys[0][0], keys[1][0], keys[0][0], keys[1][0]]
+    total = sum(sp.seq_len for sp in specs)
+    k_out, v_out = empty_out(w.num_layers, w.num_kv_heads, total, w.head_dim)
+    n, order_ids = S.render(k_out, v_out)
+    torch.cuda.synchronize()
+    order = _oracle_order(keys, [sp.seq_len for sp in specs])
+    assert n == total and order_ids == [keys[i][0] for i in order]
+    _check_sampled_planes(frags, order, k_out, v_out, layers=[0, 18, 35], heads=[2, 5])
+    S.close()
+    c.close()
+
+
 @pytest.mark.parametrize("request_index", [0, 1])
 def test_serving_requests_with_redelivery(ctx, request_index):
     w = synthetic.WORKLOADS["serve"]
