@@ -13,7 +13,8 @@ loudly if the library has not been built; nothing here computes on the CPU.
 from ._binding import (  # noqa: F401
     CMError, Status, cm_id, cm_fragment, lib, LIB_PATH, EXPORTED,
     cm_abi_version, cm_status_string, cm_last_error_message,
-    cm_context_create, cm_context_destroy, cm_context_check, cm_set_create, cm_set_destroy,
+    cm_context_create, cm_context_destroy, cm_context_check, cm_testing_bounds_violations,
+    cm_set_create, cm_set_destroy,
     cm_fragment_id, cm_fragment_id_static, cm_ingest, cm_ingest_batch, cm_ingest_many,
     cm_render_many, cm_render_job, cm_set_contains, cm_set_leq, ingest_many, render_many,
     cm_measure_int_alu, cm_context_set_render_warps, cm_context_set_dedup_by_bytes,

@@ -13,7 +13,9 @@ import os
 from typing import List, Optional, Sequence, Tuple
 
 PKG_DIR = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(PKG_DIR, "libcm.so")
+# CM_LIBRARY names another build of the same library (the bounds-checked testing build,
+# libcm_bounds.so); by default the in-tree libcm.so
+LIB_PATH = os.environ.get("CM_LIBRARY") or os.path.join(PKG_DIR, "libcm.so")
 
 if not os.path.exists(LIB_PATH):
     raise ImportError(f"{LIB_PATH} is not built: run `python -c \"import __graft_entry__ as g; "
@@ -117,6 +119,8 @@ _SIGS = {
     "cm_bagmerge": (_c.c_int, [_P, _c.POINTER(cm_fragment), _c.c_int32, _P, _P, _c.c_int64, _P,
                                _c.POINTER(_c.c_int64)]),
     "cm_testing_render_withheld_load": (_c.c_int, [_P, _P, _P, _c.c_int64, _P]),
+    "cm_testing_bounds_violations": (_c.c_int, [_c.c_int32, _c.POINTER(_c.c_uint64),
+                                                _c.POINTER(_c.c_int32)]),
     "cm_render_paged": (_c.c_int, [_P, _c.POINTER(cm_paged_cache), _P, _c.POINTER(_c.c_int64),
                                    _c.POINTER(cm_id)]),
     "cm_render_incremental": (_c.c_int, [_P, _P, _P, _c.c_int64, _c.POINTER(cm_id), _c.c_int64, _P,
@@ -177,6 +181,14 @@ def cm_context_destroy(ctx: Optional[int]) -> None:
 
 def cm_context_check(ctx: int, stream=None) -> None:
     _check(lib.cm_context_check(ctx, _stream_handle(stream)))
+
+
+def cm_testing_bounds_violations(device: int = 0) -> Tuple[int, bool]:
+    """(count, enabled): out-of-buffer accesses counted by a bounds-checked build since the
+    previous call (the device is synchronised), and whether this library is such a build."""
+    n, en = ctypes.c_uint64(), ctypes.c_int32()
+    _check(lib.cm_testing_bounds_violations(device, ctypes.byref(n), ctypes.byref(en)))
+    return n.value, bool(en.value)
 
 
 def cm_set_create(ctx: int) -> int:

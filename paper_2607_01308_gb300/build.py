@@ -8,6 +8,11 @@ Three translation units compiled in parallel, then one shared-library link:
   csrc/readback.cu       small device-to-host results written by the SMs (nvcc, sm_103a)
 The CUDA runtime is linked statically into libcm.so and only the cm_* symbols
 are exported (csrc/libcm.map).
+
+`--bounds` (build(bounds=True)) builds the same sources with -DCM_DEBUG_BOUNDS into
+libcm_bounds.so (objects in _build_bounds/): a testing build whose kernels check every
+global access against its buffer (csrc/cm_bounds.h). The binding loads it when the
+environment variable CM_LIBRARY names it.
 """
 from __future__ import annotations
 
@@ -22,6 +27,8 @@ CSRC = os.path.join(PKG_DIR, "csrc")
 INCLUDE = os.path.join(REPO_DIR, "include")
 BUILD_DIR = os.path.join(PKG_DIR, "_build")
 LIB_PATH = os.path.join(PKG_DIR, "libcm.so")
+BOUNDS_BUILD_DIR = os.path.join(PKG_DIR, "_build_bounds")
+BOUNDS_LIB_PATH = os.path.join(PKG_DIR, "libcm_bounds.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-std=c++17", "-O3", "-lineinfo", "-fmad=false", "-Xcompiler", "-fPIC",
@@ -52,38 +59,42 @@ def _run(cmd, verbose):
     return r.stdout
 
 
-def build(verbose: bool = False, ptxas_info: bool = False) -> str:
-    """Compile and link libcm.so; returns its path. Raises RuntimeError on failure."""
+def build(verbose: bool = False, ptxas_info: bool = False, bounds: bool = False) -> str:
+    """Compile and link libcm.so (libcm_bounds.so with bounds=True); returns its path.
+    Raises RuntimeError on failure."""
+    build_dir = BOUNDS_BUILD_DIR if bounds else BUILD_DIR
+    lib_path = BOUNDS_LIB_PATH if bounds else LIB_PATH
+    defs = ["-DCM_DEBUG_BOUNDS"] if bounds else []
     cuda = _cuda_home()
     nvcc = os.path.join(cuda, "bin", "nvcc")
     if not os.path.exists(nvcc):
         nvcc = shutil.which("nvcc") or "nvcc"
     cxx = os.environ.get("CXX", shutil.which("g++") or "g++")
-    os.makedirs(BUILD_DIR, exist_ok=True)
+    os.makedirs(build_dir, exist_ok=True)
     cuda_inc = os.path.join(cuda, "include")
     jobs = []
     for src in CUDA_SOURCES:
-        obj = os.path.join(BUILD_DIR, src + ".o")
+        obj = os.path.join(build_dir, src + ".o")
         extra = ["-Xptxas", "-v"] if ptxas_info else []
-        jobs.append([nvcc] + ARCH + NVCC_FLAGS + extra + ["-c", os.path.join(CSRC, src), "-o", obj])
+        jobs.append([nvcc] + ARCH + NVCC_FLAGS + defs + extra + ["-c", os.path.join(CSRC, src), "-o", obj])
     for src in CXX_SOURCES:
-        obj = os.path.join(BUILD_DIR, src + ".o")
-        jobs.append([cxx] + CXX_FLAGS + ["-I" + cuda_inc, "-c", os.path.join(CSRC, src), "-o", obj])
+        obj = os.path.join(build_dir, src + ".o")
+        jobs.append([cxx] + CXX_FLAGS + defs + ["-I" + cuda_inc, "-c", os.path.join(CSRC, src), "-o", obj])
     with ThreadPoolExecutor(max_workers=len(jobs)) as ex:
         logs = list(ex.map(lambda c: _run(c, verbose), jobs))
     if ptxas_info:
         for log in logs:
             print(log)
-    objs = [os.path.join(BUILD_DIR, s + ".o") for s in CUDA_SOURCES + CXX_SOURCES]
-    tmp = LIB_PATH + ".tmp"
+    objs = [os.path.join(build_dir, s + ".o") for s in CUDA_SOURCES + CXX_SOURCES]
+    tmp = lib_path + ".tmp"
     link = ["-shared", "-Xcompiler", "-fPIC", "-cudart", "static",
             "-Xlinker", "--version-script=" + os.path.join(CSRC, "libcm.map"),
             "-Xlinker", "-Bsymbolic"]
     _run([nvcc] + ARCH + link + ["-o", tmp] + objs, verbose)
-    os.replace(tmp, LIB_PATH)
-    return LIB_PATH
+    os.replace(tmp, lib_path)
+    return lib_path
 
 
 if __name__ == "__main__":
     import sys
-    print(build(verbose=True, ptxas_info="--ptxas" in sys.argv))
+    print(build(verbose=True, ptxas_info="--ptxas" in sys.argv, bounds="--bounds" in sys.argv))

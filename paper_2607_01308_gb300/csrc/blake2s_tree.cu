@@ -12,6 +12,7 @@
 // ascending element order, then the quantised norm (round-half-even of 2^20 * sqrt,
 // saturated at 2^44 - 1) added into Q[t] with a 64-bit integer atomic: integer
 // addition is associative, so Q does not depend on the order the atomics land in.
+#include "cm_bounds.h"
 #include "cm_hash_kernels.h"
 
 #include <cstring>
@@ -119,6 +120,23 @@ __device__ __forceinline__ void store_digest(uint8_t *dst, const uint32_t h[8]) 
     *reinterpret_cast<uint4 *>(dst) = make_uint4(h[0], h[1], h[2], h[3]);
 }
 
+// Bounds-checked builds: [p, p + n) lies inside the fragment's K or V array (each
+// stream_bytes / 2 long); otherwise a violation is counted.
+__device__ __forceinline__ bool in_fragment(const LeafLaunch &a, const uint8_t *p, uint64_t n) {
+#ifdef CM_DEBUG_BOUNDS
+    const uint64_t half = a.stream_bytes / 2, x = reinterpret_cast<uint64_t>(p);
+    const uint64_t k = reinterpret_cast<uint64_t>(a.k), v = reinterpret_cast<uint64_t>(a.v);
+    if (n <= half && ((x >= k && x - k <= half - n) || (x >= v && x - v <= half - n))) return true;
+    bounds_fail();
+    return false;
+#else
+    (void)a;
+    (void)p;
+    (void)n;
+    return true;
+#endif
+}
+
 // fl(ss + x^2) for the 8 bf16 of one 16-byte vector, in ascending element order (x^2
 // is exact in fp64, so each step is the one rounding of the sum). A normal bf16 (exponent
 // field 1..254) is 2^(e-127) (1 + m/128) in magnitude; as an fp64 its exponent field is
@@ -165,7 +183,10 @@ __device__ __forceinline__ void norm_row(const LeafLaunch &a, uint64_t r) {
         uint4 w[4];
 #pragma unroll
         for (int q = 0; q < 4; ++q)
-            if (v + q < nvec) w[q] = load_nc(row + 16 * (v + q));
+            if (v + q < nvec)
+                w[q] = CM_IN_BOUNDS(row + 16 * (v + q), 16, a.k + a.norm_begin / 2, a.plane_bytes)
+                           ? load_nc(row + 16 * (v + q))
+                           : make_uint4(0, 0, 0, 0);
 #pragma unroll
         for (int q = 0; q < 4; ++q)
             if (v + q < nvec) ss = accumulate_squares(w[q], ss);
@@ -173,7 +194,8 @@ __device__ __forceinline__ void norm_row(const LeafLaunch &a, uint64_t r) {
     const double scaled = __dsqrt_rn(ss) * 1048576.0;     // exact scaling by 2^20
     const unsigned long long q =
         (scaled < (double)kQMax) ? __double2ull_rn(scaled) : kQMax;   // NaN saturates too
-    atomicAdd(a.norm_key + r % a.seq_len, q);
+    const uint64_t t = r % a.seq_len;
+    if (CM_IN_BOUNDS(a.norm_key + t, 8, a.norm_key, (uint64_t)a.seq_len * 8)) atomicAdd(a.norm_key + t, q);
 }
 
 // Cursor over the fragment's byte stream K[0] V[0] K[1] V[1] ...: every segment
@@ -250,6 +272,7 @@ leaf_hash_kernel(const __grid_constant__ LeafGroup grp) {
     if (len == (uint32_t)kLeafBytes && cur.left >= (uint64_t)kLeafBytes) {
         // the whole leaf lies in one K or V segment
         const uint8_t *p = cur.ptr;
+        if (!in_fragment(a, p, kLeafBytes)) return;
 #pragma unroll 1
         for (uint32_t b = 0; b < 16; ++b) {
             const uint4 w0 = load_nc(p + 64 * b), w1 = load_nc(p + 64 * b + 16),
@@ -258,21 +281,30 @@ leaf_hash_kernel(const __grid_constant__ LeafGroup grp) {
                                     w2.x, w2.y, w2.z, w2.w, w3.x, w3.y, w3.z, w3.w};
             compress(h, m, (b + 1) * 64, b == 15, last_node);
         }
-        store_digest(a.digests + leaf * kDigestBytes, h);
+        if (CM_IN_BOUNDS(a.digests + leaf * kDigestBytes, kDigestBytes, a.digests,
+                         a.num_leaves * kDigestBytes))
+            store_digest(a.digests + leaf * kDigestBytes, h);
         return;
     }
 
     for (uint32_t b = 0; b < nblocks; ++b) {
         uint4 w[4];
 #pragma unroll
-        for (int q = 0; q < 4; ++q)
-            w[q] = b * 64 + q * 16 < len ? load_nc(cursor_next(a, cur)) : make_uint4(0, 0, 0, 0);
+        for (int q = 0; q < 4; ++q) {
+            w[q] = make_uint4(0, 0, 0, 0);
+            if (b * 64 + q * 16 < len) {
+                const uint8_t *ptr = cursor_next(a, cur);
+                if (in_fragment(a, ptr, 16)) w[q] = load_nc(ptr);
+            }
+        }
         const uint32_t m[16] = {w[0].x, w[0].y, w[0].z, w[0].w, w[1].x, w[1].y, w[1].z, w[1].w,
                                 w[2].x, w[2].y, w[2].z, w[2].w, w[3].x, w[3].y, w[3].z, w[3].w};
         const uint32_t end = (b + 1) * 64 < len ? (b + 1) * 64 : len;
         compress(h, m, end, b + 1 == nblocks, last_node);
     }
-    store_digest(a.digests + leaf * kDigestBytes, h);
+    if (CM_IN_BOUNDS(a.digests + leaf * kDigestBytes, kDigestBytes, a.digests,
+                     a.num_leaves * kDigestBytes))
+        store_digest(a.digests + leaf * kDigestBytes, h);
 }
 
 constexpr int kInnerThreads = 32;
@@ -298,14 +330,17 @@ inner_hash_kernel(const uint8_t *__restrict__ children, uint64_t num_children,
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
             const uint32_t off = b * 64 + q * 16;
-            w[q] = off < len ? load_nc(src + off) : make_uint4(0, 0, 0, 0);
+            w[q] = off < len && CM_IN_BOUNDS(src + off, 16, children, num_children * kDigestBytes)
+                       ? load_nc(src + off)
+                       : make_uint4(0, 0, 0, 0);
         }
         const uint32_t m[16] = {w[0].x, w[0].y, w[0].z, w[0].w, w[1].x, w[1].y, w[1].z, w[1].w,
                                 w[2].x, w[2].y, w[2].z, w[2].w, w[3].x, w[3].y, w[3].z, w[3].w};
         const uint32_t end = (b + 1) * 64 < len ? (b + 1) * 64 : len;
         compress(h, m, end, b + 1 == nblocks, last_node);
     }
-    store_digest(out + j * kDigestBytes, h);
+    if (CM_IN_BOUNDS(out + j * kDigestBytes, kDigestBytes, out, num_nodes * kDigestBytes))
+        store_digest(out + j * kDigestBytes, h);
 }
 
 // Node j of a tree level over the digests at `children` (num_children of them): its
@@ -329,7 +364,8 @@ __device__ __forceinline__ void hash_node_from(uint4 *stage, uint32_t len, uint8
         const uint32_t end = (b + 1) * 64 < len ? (b + 1) * 64 : len;
         compress(h, m, end, b + 1 == nblocks, last_node);
     }
-    store_digest(out + j * kDigestBytes, h);
+    if (CM_IN_BOUNDS(out + j * kDigestBytes, kDigestBytes, out, num_nodes * kDigestBytes))
+        store_digest(out + j * kDigestBytes, h);
 }
 
 // Loads node j's children (zero-padded to 256 bytes) into `stage`; returns their length.
@@ -347,7 +383,8 @@ __device__ __forceinline__ uint32_t stage_children(uint4 *stage, const uint8_t *
     uint4 w[16];
 #pragma unroll
     for (int q = 0; q < 16; ++q) {
-        const bool in = (uint32_t)(q * 16) < len;
+        const bool in = (uint32_t)(q * 16) < len &&
+                        CM_IN_BOUNDS(src + q, 16, children, num_children * kDigestBytes);
         w[q] = in ? (kCoherent ? __ldcg(src + q) : __ldg(src + q)) : make_uint4(0, 0, 0, 0);
     }
 #pragma unroll
@@ -389,14 +426,17 @@ level1_kernel(const __grid_constant__ TreeTop t) {
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
             const uint32_t off = b * 64 + q * 16;
-            w[q] = off < len ? load_nc(src + off) : make_uint4(0, 0, 0, 0);
+            w[q] = off < len && CM_IN_BOUNDS(src + off, 16, f.level[0], f.size[0] * kDigestBytes)
+                       ? load_nc(src + off)
+                       : make_uint4(0, 0, 0, 0);
         }
         const uint32_t m[16] = {w[0].x, w[0].y, w[0].z, w[0].w, w[1].x, w[1].y, w[1].z, w[1].w,
                                 w[2].x, w[2].y, w[2].z, w[2].w, w[3].x, w[3].y, w[3].z, w[3].w};
         const uint32_t end = (b + 1) * 64 < len ? (b + 1) * 64 : len;
         compress(h, m, end, b + 1 == nblocks, last_node);
     }
-    store_digest(f.level[1] + j * kDigestBytes, h);
+    if (CM_IN_BOUNDS(f.level[1] + j * kDigestBytes, kDigestBytes, f.level[1], f.size[1] * kDigestBytes))
+        store_digest(f.level[1] + j * kDigestBytes, h);
 }
 
 // Levels kStart and up (node_begin: prefix sums of the level-kStart sizes, 0 for a
@@ -425,6 +465,8 @@ tree_top_kernel(const __grid_constant__ TreeTop t) {
         const uint32_t siblings = left < (uint64_t)kFanout ? (uint32_t)left : (uint32_t)kFanout;
         // one acquire-release add: it publishes this node's digest and, for the thread
         // that counts the last sibling, makes every sibling's digest visible
+        if (!CM_IN_BOUNDS(f.arrivals[k + 1] + parent, 4, f.arrivals[k + 1], f.size[k + 1] * 4))
+            return;
         const uint32_t done = arrive_acq_rel(f.arrivals[k + 1] + parent) + 1;
         if (done != siblings) return;
         j = parent;
@@ -444,6 +486,8 @@ __global__ void compare_kernel(const uint4 *__restrict__ a, const uint4 *__restr
 }
 
 }  // namespace
+
+CM_DEFINE_BOUNDS_READER(take_hash_bounds_violations)
 
 cudaError_t launch_leaf_hash_group(const LeafGroup &in, cudaStream_t stream) {
     if (in.count > (uint32_t)kMaxLeafGroup) return cudaErrorInvalidValue;

@@ -94,6 +94,10 @@ int tree_top_kernels(const TreeTop &t);   // kernels launch_tree_top launches fo
 cudaError_t launch_compare(const void *a, const void *b, uint64_t bytes, unsigned int *flag,
                            cudaStream_t stream);
 
+// Bounds-checked builds: reads and zeroes the content-address kernels' violation count on
+// the current device (0 in other builds).
+cudaError_t take_hash_bounds_violations(unsigned int *out);
+
 // Host-core helpers used by the allocation-free entry point in blake2s_tree.cu.
 TreeParams make_tree_params(int32_t L, int32_t H, int32_t d, int32_t T);
 cm_status check_fragment(const cm_fragment *f);

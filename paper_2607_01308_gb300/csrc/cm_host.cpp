@@ -536,6 +536,7 @@ cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t 
             p->k_pool = paged->k_pool;
             p->v_pool = paged->v_pool;
             p->block_table = paged->block_table;
+            p->table_entries = paged->table_entries;
             p->block_size = paged->block_size;
             p->log2_block_size = is_pow2(paged->block_size)
                                      ? (int32_t)__builtin_ctzll((unsigned long long)paged->block_size)
@@ -1281,6 +1282,25 @@ cm_status cm_render_paged(const cm_set *set, const cm_paged_cache *out, cm_strea
 cm_status cm_testing_render_withheld_load(const cm_set *set, void *k_out, void *v_out,
                                           int64_t capacity_tokens, cm_stream_t stream) {
     return render_set(set, k_out, v_out, capacity_tokens, stream, nullptr, nullptr, 1);
+}
+
+cm_status cm_testing_bounds_violations(int32_t device, uint64_t *out_count, int32_t *out_enabled) {
+    return guarded([&]() -> cm_status {
+        if (!out_count || !out_enabled) return fail(CM_ERR_INVALID_ARG, "out_count or out_enabled is NULL");
+        DeviceScope scope(device);
+        if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
+        CM_CUDA_TRY(cudaDeviceSynchronize(), "device synchronisation");
+        unsigned int render = 0, hash = 0;
+        CM_CUDA_TRY(cm::take_render_bounds_violations(&render), "render violation count");
+        CM_CUDA_TRY(cm::take_hash_bounds_violations(&hash), "content-address violation count");
+        *out_count = (uint64_t)render + hash;
+#ifdef CM_DEBUG_BOUNDS
+        *out_enabled = 1;
+#else
+        *out_enabled = 0;
+#endif
+        return CM_OK;
+    });
 }
 
 cm_status cm_context_check(cm_context *ctx, cm_stream_t stream) {

@@ -53,6 +53,7 @@ struct RenderParams {
     int64_t block_size;
     int32_t log2_block_size;    // >= 0 when block_size is a power of two, else -1
     int32_t pad3_;
+    int64_t table_entries;      // entries of block_table (bounds-checked builds check reads)
     int64_t stride_block, stride_layer, stride_head, stride_token;
     RenderSlot slot[kMaxSlots];
     double cs[2 * kMaxTablePairs];   // (cos a, sin a) of a = s * theta^(-2j/d), interleaved
@@ -62,5 +63,9 @@ struct RenderParams {
 // other streams) per SM; render_prepare() once per device before the first launch.
 cudaError_t launch_render(const RenderParams &p, int grid, int warps, cudaStream_t stream);
 cudaError_t render_prepare();
+
+// Bounds-checked builds: reads and zeroes the render kernels' violation count on the
+// current device (0 in other builds).
+cudaError_t take_render_bounds_violations(unsigned int *out);
 
 }  // namespace cm

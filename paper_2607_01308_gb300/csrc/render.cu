@@ -28,6 +28,7 @@
 // cannot certify are recomputed in fp64 with the operation sequence of the
 // definition and rounded directly to bf16 (fp64 throughput is very low on this part,
 // so it must stay rare). The output is bit-exact either way.
+#include "cm_bounds.h"
 #include "cm_render_kernels.h"
 
 namespace cm {
@@ -247,6 +248,12 @@ struct Item {
     int32_t rows;
     int32_t rotate;      // 1: K of a slot at a nonzero offset
     int32_t cs_index;    // first (cos, sin) of this slot
+#ifdef CM_DEBUG_BOUNDS
+    const uint8_t *src_base;   // the slot's K or V fragment
+    uint64_t src_size;
+    const uint8_t *dst_base;   // the slot's K or V output (paged: the pool, whose size the
+    uint64_t dst_size;         // library is not told: only the lower end is checked)
+#endif
 };
 
 // Item g: pair g / 2 of its slot (row chunk c of (layer, head) plane lh), K if g is
@@ -256,7 +263,6 @@ __device__ __forceinline__ Item item_of(const RenderParams &p, uint32_t g) {
     while (si + 1 < p.num_slots && g >= p.slot[si + 1].chunk_begin) ++si;
     const RenderSlot &S = p.slot[si];
     const uint32_t local = g - S.chunk_begin;
-    const uint32_t lh_planes = (uint32_t)p.num_layers * (uint32_t)p.num_heads;
     const bool is_v = (local & 1u) != 0;             // K and V items alternate
     const uint32_t pair = local >> 1;
     const uint32_t lhp = pair / S.chunks_per_plane;
@@ -282,7 +288,38 @@ __device__ __forceinline__ Item item_of(const RenderParams &p, uint32_t g) {
     it.rows = rows;
     it.rotate = (!is_v && S.rotate) ? 1 : 0;
     it.cs_index = S.table_base;
+#ifdef CM_DEBUG_BOUNDS
+    const uint64_t lh_planes = (uint64_t)p.num_layers * (uint64_t)p.num_heads;
+    it.src_base = static_cast<const uint8_t *>(is_v ? S.v : S.k);
+    it.src_size = (uint64_t)lh_planes * (uint64_t)S.seq_len * (uint64_t)row_bytes;
+    if (p.paged) {
+        it.dst_base = static_cast<const uint8_t *>(is_v ? p.v_pool : p.k_pool);
+        it.dst_size = ~0ull - reinterpret_cast<uint64_t>(it.dst_base);
+    } else {
+        it.dst_base = static_cast<const uint8_t *>(is_v ? S.v_out : S.k_out);
+        it.dst_size = (uint64_t)lh_planes * (uint64_t)S.capacity * (uint64_t)row_bytes;
+    }
+#endif
     return it;
+}
+
+// Physical block of logical block b of a paged output (in bounds-checked builds: an index
+// outside the table or a negative entry counts a violation and reads as block 0).
+__device__ __forceinline__ int64_t table_entry(const RenderParams &p, int64_t b) {
+#ifdef CM_DEBUG_BOUNDS
+    if (b < 0 || !CM_IN_BOUNDS(p.block_table + b, 4, p.block_table, (uint64_t)p.table_entries * 4)) {
+        if (b < 0) bounds_fail();
+        return 0;
+    }
+    const int64_t blk = __ldg(p.block_table + b);
+    if (blk < 0) {
+        bounds_fail();
+        return 0;
+    }
+    return blk;
+#else
+    return __ldg(p.block_table + b);
+#endif
 }
 
 // Paged outputs: where the rows of one item go. When the block size is a power of two
@@ -308,10 +345,10 @@ __device__ __forceinline__ PagedRows paged_rows(const RenderParams &p, const Ite
         const int64_t b0 = it.pos0 >> p.log2_block_size;
         const int64_t o0 = it.pos0 & (p.block_size - 1);
         const int64_t k = p.block_size - o0;                 // rows left in block b0
-        pr.a = it.dst + (int64_t)__ldg(p.block_table + b0) * p.stride_block * 2 + o0 * pr.stride;
+        pr.a = it.dst + table_entry(p, b0) * p.stride_block * 2 + o0 * pr.stride;
         if (k < it.rows) {
             pr.split = (int)k;
-            pr.b = it.dst + (int64_t)__ldg(p.block_table + b0 + 1) * p.stride_block * 2 - k * pr.stride;
+            pr.b = it.dst + table_entry(p, b0 + 1) * p.stride_block * 2 - k * pr.stride;
         }
     }
     return pr;
@@ -336,7 +373,7 @@ __device__ __forceinline__ uint4 *row_dst(const RenderParams &p, const Item &it,
         b = pos / p.block_size;
         o = pos - b * p.block_size;
     }
-    const int64_t blk = __ldg(p.block_table + b);
+    const int64_t blk = table_entry(p, b);
     return reinterpret_cast<uint4 *>(it.dst + (blk * p.stride_block + o * p.stride_token) * 2);
 }
 
@@ -357,14 +394,18 @@ __device__ __forceinline__ void copy_from_smem(const RenderParams &p, const Item
         uint4 *dst = reinterpret_cast<uint4 *>(it.dst);
 #pragma unroll
         for (int u = 0; u < kU; ++u)
-            if (lane + 32 * u < n_vec) st_stream(dst + lane + 32 * u, r[u]);
+            if (lane + 32 * u < n_vec && CM_IN_BOUNDS(dst + lane + 32 * u, 16, it.dst_base, it.dst_size))
+                st_stream(dst + lane + 32 * u, r[u]);
     } else {
         const int log2_vpr = p.log2_pairs_per_row + 1;     // vectors per row = d / 8
         const int col_mask = (1 << log2_vpr) - 1;
 #pragma unroll
         for (int u = 0; u < kU; ++u) {
             const int v = lane + 32 * u;
-            if (v < n_vec) st_stream(row_dst<true>(p, it, v >> log2_vpr, pr) + (v & col_mask), r[u]);
+            if (v < n_vec) {
+                uint4 *q = row_dst<true>(p, it, v >> log2_vpr, pr) + (v & col_mask);
+                if (CM_IN_BOUNDS(q, 16, it.dst_base, it.dst_size)) st_stream(q, r[u]);
+            }
         }
     }
 }
@@ -404,8 +445,8 @@ __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const fl
         rotate_word(a.w, b.w, c[6], s[6], c[7], s[7], ao.w, bo.w, b3);
         if ((b0 | b1 | b2 | b3) != 0u) fixup_pair(p, tab, cs_index, a, b, b0, b1, b2, b3, ao, bo);
         uint4 *d = row_dst<kPaged>(p, it, row, pr) + lane_v;
-        st_stream(d, ao);
-        st_stream(d + half_vecs, bo);
+        if (CM_IN_BOUNDS(d, 16, it.dst_base, it.dst_size)) st_stream(d, ao);
+        if (CM_IN_BOUNDS(d + half_vecs, 16, it.dst_base, it.dst_size)) st_stream(d + half_vecs, bo);
     }
 }
 
@@ -462,9 +503,12 @@ render_kernel(const __grid_constant__ RenderParams p) {
         const uint32_t s = j % kStages;
         const Item it = item_of(p, 2 * (first + (j >> 1) * stride) + (j & 1));
         items[warp][s] = it;
-        mbar_arrive_expect_tx(&full[warp][s], it.bytes);
+        // bounds-checked builds: a source outside the slot's fragment is not copied (the
+        // stage keeps stale bytes, the barrier completes without them)
+        const bool src_ok = CM_IN_BOUNDS(it.src, it.bytes, it.src_base, it.src_size);
+        mbar_arrive_expect_tx(&full[warp][s], src_ok ? it.bytes : 0u);
         if (j == 0 && p.withhold_warp == first + 1) return;   // injected: the wait runs out
-        bulk_load(wbuf + (size_t)s * kItemBytes, it.src, it.bytes, &full[warp][s]);
+        if (src_ok) bulk_load(wbuf + (size_t)s * kItemBytes, it.src, it.bytes, &full[warp][s]);
     };
 
     uint32_t produced = 0;
@@ -515,6 +559,8 @@ cudaError_t launch_width(const RenderParams &p, int grid, cudaStream_t stream) {
 }
 
 }  // namespace
+
+CM_DEFINE_BOUNDS_READER(take_render_bounds_violations)
 
 cudaError_t render_prepare() {
     cudaError_t e = set_smem_attribute<false, 16>();

@@ -81,3 +81,18 @@ def test_null_and_range_arguments_rejected_without_cuda(cm):
     # destroying NULL handles is a no-op
     assert lib.cm_set_destroy(None) == cm.Status.OK
     assert lib.cm_context_destroy(None) == cm.Status.OK
+
+
+def test_bounds_checked_build_compiles_and_exports_every_declared_call():
+    # the testing build (build.py --bounds) is the same library with checked accesses
+    import shutil
+    import subprocess
+    nm = shutil.which("nm")
+    if nm is None:
+        pytest.skip("nm is not available")
+    from paper_2607_01308_gb300 import build as cm_build
+    path = cm_build.build(bounds=True)
+    out = subprocess.run([nm, "-D", "--defined-only", path], stdout=subprocess.PIPE, text=True,
+                         check=True).stdout
+    exported = set(re.findall(r"\b(cm_[a-z_]+)\b", out))
+    assert set(_declared_functions()) <= exported
