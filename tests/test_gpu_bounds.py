@@ -33,3 +33,13 @@ def test_bounds_checked_build_sees_no_access_outside_its_buffers():
     assert res["violations"] == 0
     assert res["negative_table_entry_violations"] > 0
     assert res["violations_after"] == 0
+
+
+def test_normal_build_reports_no_checks():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2607_01308_gb300 as cm
+    if os.environ.get("CM_LIBRARY"):
+        pytest.skip("another build of the library is loaded")
+    count, enabled = cm.cm_testing_bounds_violations(0)
+    assert not enabled and count == 0
