@@ -199,11 +199,11 @@ def sm_max_mhz():
 
 # ---------------------------------------------------------------- CPU oracle (baseline leg)
 
-def oracle_sample_seconds(layers=1, w=None):
+def oracle_sample_parts(layers=1, w=None):
     """The oracle as it stands on a bounded sample of the workload: the first `layers`
-    layers of each of the 4 fragments (T = 4096). Returns the seconds of one full merge
-    estimated from it: the content address and the render cost the same per layer, so
-    their sample times are scaled by num_layers / layers; the routing-layer norm key
+    layers of each of the 4 fragments (T = 4096). Returns (seconds of the per-layer work,
+    seconds of the norm key): the content address and the render cost the same per layer,
+    so a full merge takes num_layers / layers times the first; the routing-layer norm key
     covers one layer of each fragment in a full merge as in the sample, so its time is
     taken as it is."""
     import numpy as np
@@ -236,6 +236,16 @@ def oracle_sample_seconds(layers=1, w=None):
     K_out, V_out, _ = oracle.render(S, synthetic.ROPE_THETA)
     t_layers += time.perf_counter() - t0
     assert K_out.shape[2] == sum(s.seq_len for s in specs)
+    return t_layers, t_norm
+
+
+def oracle_sample_seconds(layers=1, w=None):
+    """(estimated seconds of one full merge, seconds the sample took): the per-layer work
+    (content address, union and render) scaled by num_layers / layers, the norm key as it
+    is (see oracle_sample_parts)."""
+    import synthetic
+    w = w or synthetic.WORKLOADS[WORKLOAD]
+    t_layers, t_norm = oracle_sample_parts(layers, w)
     return t_layers * w.num_layers / layers + t_norm, t_layers + t_norm
 
 
@@ -266,6 +276,47 @@ def cpu_baseline_entry(layers=24):
                       f"({dt:.2f} s); content address and render scaled by {w.num_layers}/{layers}, "
                       f"the routing-layer norm key (one layer per fragment either way) unscaled; "
                       f"single thread (numpy fp64 + hashlib)",
+            "seconds_per_merge": per_merge}
+
+
+def _oracle_worker(layers: int):
+    """One process of the multi-core estimate: the oracle's compute seconds on a sample of
+    `layers` layers of the headline merge (fragment generation not included), split into
+    the per-layer work and the routing-layer norm key."""
+    import synthetic
+    return oracle_sample_parts(layers, synthetic.WORKLOADS[WORKLOAD])
+
+
+def _oracle_ready(_):
+    import numpy  # noqa: F401
+    import oracle  # noqa: F401
+    import synthetic  # noqa: F401
+    return os.getpid()
+
+
+def cpu_baseline_multicore(layers_per_core=2):
+    """The oracle split by layer over every host core (SURVEY's optional second row): one
+    process per core runs the single-thread sample on its own `layers_per_core` layers at
+    the same time; the slowest process's compute time, scaled to the merge's layer count,
+    estimates a merge on all cores (the upper levels of the hash tree, which span layers,
+    are counted per sample as in the single-core estimate)."""
+    import multiprocessing as mp
+    import synthetic
+    w = synthetic.WORKLOADS[WORKLOAD]
+    cores = os.cpu_count() or 1
+    pool_ctx = mp.get_context("spawn")     # this process already holds a CUDA context
+    with pool_ctx.Pool(cores) as pool:
+        pool.map(_oracle_ready, range(cores))
+        parts = pool.map(_oracle_worker, [layers_per_core] * cores)
+    t_layers = max(p[0] for p in parts)
+    t_norm = max(p[1] for p in parts)
+    per_merge = t_layers * w.num_layers / (cores * layers_per_core) + t_norm
+    return {"value": 1.0 / per_merge, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "estimate": True,
+            "sample": f"{cores} processes, each the single-thread sample on {layers_per_core} "
+                      f"layers at once (slowest per-layer work {t_layers:.2f} s, scaled by "
+                      f"{w.num_layers}/({cores} x {layers_per_core}); norm key {t_norm:.2f} s, "
+                      f"unscaled)",
             "seconds_per_merge": per_merge}
 
 
@@ -833,6 +884,7 @@ def main():
         }
         if world == 1 and not args.no_cpu_baseline and args.workload == WORKLOAD:
             line["cpu_baseline"] = cpu_baseline_entry()
+            line["cpu_baseline"]["all_cores"] = cpu_baseline_multicore()
         print(json.dumps(line), flush=True)
     ctx.close()
     if world > 1:
