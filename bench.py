@@ -98,8 +98,20 @@ def workload_config(w):
         "head_dim": w.head_dim, "fragments": len(specs), "seq_lens": [s.seq_len for s in specs],
         "merged_tokens": sum(s.seq_len for s in specs), "routing_layer": w.num_layers // 2,
         "replicas_per_merge": 2,
-        "l2": "no flush: every step streams 2.4 GB of fragments and 2.4 GB of output (> 129 MB L2)",
+        "l2": l2_note(sum(s.seq_len for s in specs) * w.bytes_per_token),
     }
+
+
+def l2_note(fragment_bytes: int) -> str:
+    """How a step stands against L2 reuse between steps: the hash and the render each read
+    every fragment once and the render writes as many bytes."""
+    mb = fragment_bytes / 1e6
+    note = (f"no flush: every step reads {mb:.1f} MB of fragments twice (hash, render) and "
+            f"writes {mb:.1f} MB of merged cache, {3 * mb:.1f} MB per step against a 129 MB L2")
+    if fragment_bytes < 129e6:
+        note += ("; the fragments alone fit in L2, so part of a step's reads may hit it: a "
+                 "profiling case, not a headline configuration")
+    return note
 
 
 # ---------------------------------------------------------------- measured peaks, clocks, profiles
