@@ -62,9 +62,9 @@ def parse_args():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--e2e-steps", type=int, default=None)
     p.add_argument("--redeliver", type=int, default=0, metavar="R",
-                   help="re-delivery sweep: every fragment of the Qwen3-4B-shaped merge arrives R "
-                        "times as separate copies; merges/s with the byte-comparison fast path "
-                        "off and on")
+                   help="re-delivery sweep: every fragment of the workload (--workload, default the "
+                        "Qwen3-4B-shaped merge) arrives R times as separate copies; merges/s with the "
+                        "byte-comparison fast path off and on")
     p.add_argument("--serve", action="store_true",
                    help="run the serving sweep (64 requests of 3 Qwen3-4B-shaped fragments with "
                         "re-deliveries) instead of the single-merge benchmark")
@@ -385,8 +385,8 @@ def whole_job_rate(world: int, steps_per_rank: int, max_elapsed_ms: float) -> fl
 # ---------------------------------------------------------------- serving sweep
 
 def run_redeliver(args):
-    """Re-delivery (the fault model of Section 5.9): one replica receives each of the 4
-    Qwen3-4B-shaped fragments R times, every delivery its own byte-identical copy, in a
+    """Re-delivery (the fault model of Section 5.9): one replica receives each fragment of
+    the workload (default: the 4 Qwen3-4B-shaped fragments) R times, every delivery its own byte-identical copy, in a
     shuffled order, with one cm_ingest_batch call, then renders the set. Timed with the
     re-delivery fast path (cm_context_set_dedup_by_bytes) off and on; the rendered bytes
     are compared between the two."""
@@ -395,7 +395,7 @@ def run_redeliver(args):
     import paper_2607_01308_gb300 as cm
     import synthetic
     R = args.redeliver
-    w = synthetic.WORKLOADS[WORKLOAD]
+    w = synthetic.WORKLOADS[args.workload]
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     specs = synthetic.fragment_specs(w)
@@ -420,7 +420,7 @@ def run_redeliver(args):
 
     line = {"mode": "re-delivery sweep", "metric": METRIC, "unit": UNIT, "n_gpus": 1,
             "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": WORKLOAD_TEXT[WORKLOAD], "redeliveries": R,
+            "config": {"workload": WORKLOAD_TEXT[args.workload], "redeliveries": R,
                        "deliveries": len(fd), "distinct": len(frags)}}
     for name, on, (k_out, v_out) in (("fast_path_off", False, outs[:2]), ("fast_path_on", True, outs[2:])):
         cm.cm_context_set_dedup_by_bytes(ctx.handle, on)
