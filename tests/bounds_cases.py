@@ -176,6 +176,20 @@ def main():
     S.close()
     cases += 2
 
+    # several sets in shared render launches (per-slot outputs of different capacities)
+    sa, sb = cm.FragmentSet(ctx), cm.FragmentSet(ctx)
+    fa, fb2 = frags_of(51, 2, 2, 64, (30, 17)), frags_of(52, 2, 2, 64, (9, 40, 2))
+    cm.ingest_many([(sa, *f) for f in fa] + [(sb, *f) for f in fb2])
+    outs = [empty_out(2, 2, sa.seq_len() + 3, 64), empty_out(2, 2, sb.seq_len(), 64)]
+    ns = cm.render_many([(sa, *outs[0]), (sb, *outs[1])])
+    torch.cuda.synchronize()
+    for S, f, (k, v), n in ((sa, fa, outs[0], ns[0]), (sb, fb2, outs[1], ns[1])):
+        kr, vr, _ = check_render(ctx, f, cap_extra=0)
+        assert n == kr.shape[2]
+        assert torch.equal(k[:, :, :n], kr) and torch.equal(v[:, :, :n], vr)
+        S.close()
+    cases += 1
+
     clean, _ = cm.cm_testing_bounds_violations(0)
 
     # positive control: a negative block-table entry must be counted
