@@ -75,3 +75,46 @@ def test_random_merge_matches_oracle(ctx, seed):
     assert assert_k_parity(synthetic.to_bits(k[:, :, :n]), K_ref) == 0
     assert (k.view(torch.int16)[:, :, n:] == 0x2468).all() and (v.view(torch.int16)[:, :, n:] == 0x2468).all()
     S.close()
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_random_paged_render_matches_contiguous(ctx, seed):
+    frags, deliveries, _ = _case(100 + seed)
+    L, H, _, d = frags[0][0].shape
+    rng = np.random.default_rng(3000 + seed)
+    bs = int(rng.choice((1, 3, 8, 16, 17, 64, 128)))
+    layout = "per_layer" if rng.random() < 0.5 else "block_major"
+    S = cm.FragmentSet(ctx)
+    S.ingest_batch([frags[i] for i in deliveries])
+    total = S.seq_len()
+    k, v = empty_out(L, H, total, d)
+    n, order = S.render(k, v)
+    nb = -(-total // bs)
+    num_blocks = nb + int(rng.integers(1, 5))
+    table = torch.from_numpy(rng.permutation(num_blocks)[:nb].astype(np.int32)).to("cuda:0")
+    if layout == "per_layer":          # [L][num_blocks][bs][H][d]
+        shape = (L, num_blocks, bs, H, d)
+        strides = dict(stride_layer=num_blocks * bs * H * d, stride_block=bs * H * d,
+                       stride_token=H * d, stride_head=d)
+    else:                              # [num_blocks][L][H][bs][d]
+        shape = (num_blocks, L, H, bs, d)
+        strides = dict(stride_block=L * H * bs * d, stride_layer=H * bs * d,
+                       stride_head=bs * d, stride_token=d)
+    kp = torch.full(shape, 0x1357, dtype=torch.int16, device="cuda:0").view(torch.bfloat16)
+    vp = torch.full(shape, 0x1357, dtype=torch.int16, device="cuda:0").view(torch.bfloat16)
+    cache = cm.cm_paged_cache(kp.data_ptr(), vp.data_ptr(), table.data_ptr(), nb, bs, **strides)
+    n2, order2 = cm.cm_render_paged(S.handle, cache)
+    torch.cuda.synchronize()
+    assert n2 == n and order2 == order
+    pos = torch.arange(total, device="cuda:0")
+    blk = table.long()[pos // bs]
+    off = pos % bs
+    if layout == "per_layer":
+        kg, vg = kp[:, blk, off].permute(0, 2, 1, 3), vp[:, blk, off].permute(0, 2, 1, 3)
+    else:
+        kg, vg = kp[blk, :, :, off].permute(1, 2, 0, 3), vp[blk, :, :, off].permute(1, 2, 0, 3)
+    assert torch.equal(kg, k) and torch.equal(vg, v)
+    spare = [b for b in range(num_blocks) if b not in set(table.tolist())]
+    untouched = kp.view(torch.int16)[:, spare] if layout == "per_layer" else kp.view(torch.int16)[spare]
+    assert (untouched == 0x1357).all()
+    S.close()
