@@ -118,3 +118,59 @@ def test_random_paged_render_matches_contiguous(ctx, seed):
     untouched = kp.view(torch.int16)[:, spare] if layout == "per_layer" else kp.view(torch.int16)[spare]
     assert (untouched == 0x1357).all()
     S.close()
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_random_grouped_calls_match_separate_calls(ctx, seed):
+    # deliveries spread over several sets in one cm_ingest_many, then one cm_render_many:
+    # every set's ids, order and bytes equal its own cm_ingest_batch + cm_render
+    rng = np.random.default_rng(4000 + seed)
+    frags, _, _ = _case(200 + seed)
+    L, H, _, d = frags[0][0].shape
+    n_sets = int(rng.integers(1, 5))
+    plan = [(int(rng.integers(0, n_sets)), int(rng.integers(0, len(frags))))
+            for _ in range(int(rng.integers(1, 9)))]
+    sets = [cm.FragmentSet(ctx) for _ in range(n_sets)]
+    res = cm.ingest_many([(sets[s], *frags[f]) for s, f in plan])
+    outs = [empty_out(L, H, max(S.seq_len(), 1) + int(rng.integers(0, 9)), d) for S in sets]
+    lens = cm.render_many([(S, k, v) for S, (k, v) in zip(sets, outs)])
+    torch.cuda.synchronize()
+    for si, S in enumerate(sets):
+        mine = [f for s, f in plan if s == si]
+        T = cm.FragmentSet(ctx)
+        ref = T.ingest_batch([frags[f] for f in mine])
+        assert [r for (s, _), r in zip(plan, res) if s == si] == ref
+        k, v = empty_out(L, H, max(T.seq_len(), 1), d)
+        n, _ = T.render(k, v)
+        torch.cuda.synchronize()
+        assert lens[si] == n
+        assert torch.equal(outs[si][0][:, :, :n], k[:, :, :n]) and torch.equal(outs[si][1][:, :, :n], v[:, :, :n])
+        T.close()
+    for S in sets:
+        S.close()
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_random_incremental_render_matches_full_render(ctx, seed):
+    # fragments arrive in two waves; the second render reuses the first's canonical prefix
+    rng = np.random.default_rng(5000 + seed)
+    frags, _, _ = _case(300 + seed)
+    L, H, _, d = frags[0][0].shape
+    cut = int(rng.integers(0, len(frags) + 1))
+    total = sum(K.shape[2] for K, _ in frags)
+    S = cm.FragmentSet(ctx)
+    k, v = empty_out(L, H, total, d)
+    S.ingest_batch(frags[:cut])
+    _, order = S.render(k, v) if cut else (0, [])
+    S.ingest_batch(frags[cut:])
+    n, order2, reused = S.render_incremental(k, v, order)
+    torch.cuda.synchronize()
+    T = cm.FragmentSet(ctx)
+    T.ingest_batch(frags)
+    kf, vf = empty_out(L, H, total, d)
+    nf, orderf = T.render(kf, vf)
+    torch.cuda.synchronize()
+    assert n == nf == total and order2 == orderf and 0 <= reused <= total
+    assert torch.equal(k, kf) and torch.equal(v, vf)
+    S.close()
+    T.close()
