@@ -190,6 +190,20 @@ def main():
         S.close()
     cases += 1
 
+    # seeded random merges over the accepted shape space, and paged renders of random
+    # block sizes (the generator of test_gpu_random.py)
+    from test_gpu_random import _case
+    for seed in range(10):
+        frags, deliveries, _ = _case(700 + seed)
+        check_render(ctx, [frags[i] for i in sorted(set(deliveries))], cap_extra=int(seed % 4))
+        cases += 1
+    for seed, bs in zip(range(6), (1, 3, 8, 17, 64, 128)):
+        frags, _, _ = _case(800 + seed)
+        kc2, vc2, _ = check_render(ctx, frags, cap_extra=0)
+        kg, vg = paged_render(ctx, frags, bs)
+        assert torch.equal(kg, kc2) and torch.equal(vg, vc2)
+        cases += 1
+
     clean, _ = cm.cm_testing_bounds_violations(0)
 
     # positive control: a negative block-table entry must be counted
