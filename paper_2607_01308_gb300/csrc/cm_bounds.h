@@ -1,10 +1,10 @@
 // Bounds-checked builds (compiled with -DCM_DEBUG_BOUNDS: build.py --bounds), a testing
 // aid standing in for a device memory checker. Every global access of the kernels that
 // carry these checks is tested against the buffer it belongs to; an access outside it is
-// counted in the translation unit's violation counter and not made (a load reads the
-// buffer's first bytes instead, a store is dropped), so a wrong index shows up as a count
-// instead of a fault. Without the macro the checks compile to nothing. Not part of the
-// public ABI.
+// counted in the translation unit's violation counter and not made (a load is skipped or
+// reads zeros, a store is dropped, a TMA copy is not issued), so a wrong index shows up as
+// a count instead of a fault. Without the macro the checks compile to nothing. Not part of
+// the public ABI.
 #pragma once
 
 #include <cstdint>
