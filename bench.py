@@ -307,7 +307,7 @@ def _oracle_ready(_):
 
 
 def cpu_baseline_multicore(layers_per_core=2):
-    """The oracle split by layer over every host core (SURVEY's optional second row): one
+    """The oracle split by layer over every host core (a secondary CPU figure): one
     process per core runs the single-thread sample on its own `layers_per_core` layers at
     the same time; the slowest process's compute time, scaled to the merge's layer count,
     estimates a merge on all cores (the upper levels of the hash tree, which span layers,
