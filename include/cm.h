@@ -159,7 +159,10 @@ cm_status cm_ingest(cm_set *set, const cm_fragment *frag, cm_stream_t stream, cm
  * `stream`. A delivery whose id is
  * already in the set, or equal to an earlier delivery of the same batch, is
  * absorbed. All fragments must have the set's shape (or one common shape if the
- * set is empty). Nothing is inserted if validation fails.
+ * set is empty). Nothing is inserted if validation fails. A delivery that fails the
+ * byte check of verify_bytes_on_hit returns CM_ERR_COLLISION with the deliveries before
+ * it inserted and it and the later ones not processed, as n calls of cm_ingest that
+ * stop at the failing one.
  *   frags         HOST array of n descriptors (n >= 0)
  *   out_ids       nullable HOST array of n ids
  *   out_absorbed  nullable HOST array of n flags */
@@ -173,7 +176,9 @@ cm_status cm_ingest_batch(cm_set *set, const cm_fragment *frags, int32_t n, cm_s
  * single synchronisation of `stream`. All sets must come from one context
  * (CM_ERR_INVALID_ARG); each delivery must have its set's shape, where a set that is
  * empty takes the shape of its first delivery (CM_ERR_SHAPE_MISMATCH). Different sets
- * may have different shapes. Nothing is inserted if validation fails.
+ * may have different shapes. Nothing is inserted if validation fails; on
+ * CM_ERR_COLLISION the deliveries before the failing one are inserted (as in
+ * cm_ingest_batch).
  *   sets          HOST array of n set pointers
  *   frags         HOST array of n descriptors (n >= 0)
  *   out_ids       nullable HOST array of n ids

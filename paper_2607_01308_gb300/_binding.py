@@ -422,12 +422,14 @@ class FragmentSet:
         self.ctx = ctx
         self.handle = cm_set_create(ctx.handle)
         self._keep = {}
+        self._held = []   # tensors of failed batch calls, some of which the set may hold
 
     def close(self):
         if self.handle:
             cm_set_destroy(self.handle)
             self.handle = None
             self._keep.clear()
+            self._held.clear()
 
     def __del__(self):
         try:
@@ -437,7 +439,14 @@ class FragmentSet:
 
     def ingest_batch(self, pairs, stream=None) -> List[Tuple[bytes, bool]]:
         """Ingest [(K, V), ...] in order with one synchronisation."""
-        res = cm_ingest_batch(self.handle, [fragment_from_tensors(K, V) for K, V in pairs], stream)
+        pairs = list(pairs)
+        try:
+            res = cm_ingest_batch(self.handle, [fragment_from_tensors(K, V) for K, V in pairs],
+                                  stream)
+        except CMError:
+            # the deliveries before a failing one (CM_ERR_COLLISION) are in the set
+            self._held.extend(pairs)
+            raise
         for (fid, absorbed), kv in zip(res, pairs):
             if not absorbed:
                 self._keep.setdefault(fid, kv)
@@ -453,6 +462,7 @@ class FragmentSet:
         cm_union(self.handle, other.handle)
         for fid, kv in other._keep.items():
             self._keep.setdefault(fid, kv)
+        self._held.extend(other._held)
 
     def __len__(self) -> int:
         return cm_set_size(self.handle)
@@ -485,8 +495,15 @@ class FragmentSet:
 def ingest_many(deliveries, stream=None) -> List[Tuple[bytes, bool]]:
     """Ingest [(FragmentSet, K, V), ...] in order, one GPU pass and one synchronisation
     for all of them; deliveries may go to different sets."""
-    res = cm_ingest_many([S.handle for S, _, _ in deliveries],
-                         [fragment_from_tensors(K, V) for _, K, V in deliveries], stream)
+    deliveries = list(deliveries)
+    try:
+        res = cm_ingest_many([S.handle for S, _, _ in deliveries],
+                             [fragment_from_tensors(K, V) for _, K, V in deliveries], stream)
+    except CMError:
+        # the deliveries before a failing one (CM_ERR_COLLISION) are in their sets
+        for S, K, V in deliveries:
+            S._held.append((K, V))
+        raise
     for (fid, absorbed), (S, K, V) in zip(res, deliveries):
         if not absorbed:
             S._keep.setdefault(fid, (K, V))

@@ -273,6 +273,45 @@ def test_verify_bytes_on_hit_accepts_true_duplicates(ctx):
     c.close()
 
 
+def test_verify_bytes_on_hit_reports_a_collision(ctx):
+    # an id hit whose bytes differ, made by breaking the borrow contract on purpose: the
+    # set's record is changed in place after its ingest, then the original bytes arrive
+    # again and hash to the stored id
+    c = cm.Context(0, THETA, verify_bytes_on_hit=True)
+    g = torch.Generator(device="cuda:0").manual_seed(3)
+    mk = lambda T: (torch.randn((2, 2, T, 64), generator=g, device="cuda:0").to(torch.bfloat16),
+                    torch.randn((2, 2, T, 64), generator=g, device="cuda:0").to(torch.bfloat16))
+    (K, V), B, C = mk(9), mk(5), mk(7)
+    K0, V0 = K.clone(), V.clone()
+    S = cm.FragmentSet(c)
+    fid, _ = S.ingest(K, V)
+    V.view(torch.int16)[1, 1, 8, 63] ^= 1
+    with pytest.raises(cm.CMError) as e:
+        S.ingest(K0, V0)
+    assert e.value.status == cm.Status.ERR_COLLISION
+    assert len(S) == 1
+    # in a batch the deliveries before the colliding one are inserted, the later ones
+    # are not processed (as n single calls that stop at the failing one)
+    with pytest.raises(cm.CMError) as e:
+        S.ingest_batch([B, (K0, V0), C])
+    assert e.value.status == cm.Status.ERR_COLLISION
+    assert len(S) == 2 and S.ids() == sorted([fid, oracle_fragment(*B).fid])
+    assert any(kv[0] is B[0] for kv in S._held)     # the binding keeps B's tensors alive
+    # with the record's bytes restored the same delivery is absorbed again
+    V.copy_(V0)
+    assert S.ingest(K0, V0) == (fid, True)
+    # without verification an id hit is absorbed on the id alone
+    c2 = cm.Context(0, THETA)
+    S2 = cm.FragmentSet(c2)
+    S2.ingest(K, V)
+    V.view(torch.int16)[1, 1, 8, 63] ^= 1
+    assert S2.ingest(K0, V0) == (fid, True)
+    S2.close()
+    c2.close()
+    S.close()
+    c.close()
+
+
 # ---------------------------------------------------------------- union on the GPU-built sets
 
 def test_union_algebra_and_render_invariance(ctx):
