@@ -323,8 +323,10 @@ def cpu_baseline_multicore(layers_per_core=2):
     t_layers = max(p[0] for p in parts)
     t_norm = max(p[1] for p in parts)
     per_merge = t_layers * w.num_layers / (cores * layers_per_core) + t_norm
+    merged = sum(s.seq_len for s in synthetic.fragment_specs(w))
     return {"value": 1.0 / per_merge, "unit": UNIT, "cores": cores, "kind": "oracle",
             "estimate": True,
+            "render_bytes_gbs": 2 * merged * w.bytes_per_token / per_merge / 1e9,
             "sample": f"{cores} processes, each the single-thread sample on {layers_per_core} "
                       f"layers at once (slowest per-layer work {t_layers:.2f} s, scaled by "
                       f"{w.num_layers}/({cores} x {layers_per_core}); norm key {t_norm:.2f} s, "
