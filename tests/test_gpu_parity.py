@@ -452,6 +452,34 @@ def test_long_fragment_and_large_offsets(ctx):
     S.close()
 
 
+@pytest.mark.parametrize("L,H,d,lengths", [
+    (1, 1, 16, (262145, 3, 1000)),      # 2^18 + 1 tokens: offsets past 262,144, 16,385 leaves
+    (1, 64, 512, (37, 5)),              # many heads, 1 KiB rows (4 rows per work item)
+    (80, 1, 16, (9, 70)),               # many layers (routing layer 40)
+    (3, 8, 128, (1, 1, 1)),             # single-token fragments only (T* = 1)
+])
+def test_shape_extremes_match_oracle(ctx, L, H, d, lengths):
+    g = torch.Generator(device="cuda:0").manual_seed(L * 1000 + H * 10 + d)
+    # decreasing K scales: the first (longest) fragment leads the canonical order, so the
+    # others are rotated by offsets of its length
+    frags = [((torch.randn((L, H, T, d), generator=g, device="cuda:0") * (0.5 + len(lengths) - i))
+              .to(torch.bfloat16),
+              torch.randn((L, H, T, d), generator=g, device="cuda:0").to(torch.bfloat16))
+             for i, T in enumerate(lengths)]
+    S = cm.FragmentSet(ctx)
+    res = S.ingest_batch(frags)
+    refs = [oracle_fragment(K, V) for K, V in frags]
+    assert [r[0] for r in res] == [f.fid for f in refs]
+    k_out, v_out = empty_out(L, H, S.seq_len(), d)
+    n, order = S.render(k_out, v_out)
+    torch.cuda.synchronize()
+    K_ref, V_ref, o_order = oracle.render(oracle.from_deliveries(refs), THETA)
+    assert n == sum(lengths) and order == [f.fid for f in o_order] and order[0] == refs[0].fid
+    assert np.array_equal(synthetic.to_bits(v_out), V_ref)
+    assert assert_k_parity(synthetic.to_bits(k_out), K_ref) == 0
+    S.close()
+
+
 # ---------------------------------------------------------------- rotation stress
 
 @pytest.mark.parametrize("theta", [1.0e4, 1.0e6, 5.0e5, 1.0e40])
