@@ -480,6 +480,37 @@ def test_shape_extremes_match_oracle(ctx, L, H, d, lengths):
     S.close()
 
 
+@pytest.mark.parametrize("rl", [-1, 0, 2, 5])
+def test_explicit_routing_layer(rl):
+    # the routing layer l* picks whose norms order the set (Eq. rho); A's keys are large in
+    # layers 0-2, B's in layers 3-5, C's in none, so A leads for l* < 3 and B for l* >= 3
+    # (the default floor(6 / 2) = 3 included)
+    L, H, d = 6, 2, 64
+    c = cm.Context(0, THETA, routing_layer=rl)
+    g = torch.Generator(device="cuda:0").manual_seed(50 + rl)
+    lo = torch.tensor([3.0, 3.0, 3.0, 0.5, 0.5, 0.5], device="cuda:0").view(L, 1, 1, 1)
+    scales = (lo, lo.flip(0), torch.ones_like(lo))
+    frags = [((torch.randn((L, H, T, d), generator=g, device="cuda:0") * sc).to(torch.bfloat16),
+              torch.randn((L, H, T, d), generator=g, device="cuda:0").to(torch.bfloat16))
+             for sc, T in zip(scales, (40, 27, 61))]
+    refs = [oracle_fragment(K, V, routing_layer=rl) for K, V in frags]
+    for (K, V), ref in zip(frags, refs):
+        fid, q = c.fragment_id(K, V)
+        assert fid == ref.fid and np.array_equal(np.array(q, dtype=np.uint64), ref.Q)
+    S = cm.FragmentSet(c)
+    S.ingest_batch(frags[::-1])
+    k_out, v_out = empty_out(L, H, S.seq_len(), d)
+    n, order = S.render(k_out, v_out)
+    torch.cuda.synchronize()
+    K_ref, V_ref, o_order = oracle.render(oracle.from_deliveries(refs), THETA)
+    assert order == [f.fid for f in o_order]
+    assert order[0] == refs[0 if 0 <= rl < 3 else 1].fid
+    assert np.array_equal(synthetic.to_bits(v_out), V_ref)
+    assert assert_k_parity(synthetic.to_bits(k_out), K_ref) == 0
+    S.close()
+    c.close()
+
+
 # ---------------------------------------------------------------- rotation stress
 
 @pytest.mark.parametrize("theta", [1.0e4, 1.0e6, 5.0e5, 1.0e40])
