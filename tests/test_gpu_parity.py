@@ -511,6 +511,43 @@ def test_explicit_routing_layer(rl):
     c.close()
 
 
+def test_exact_ties_order_by_id():
+    # A, B and C tie exactly on S (Eq. rho over the last T* = 20 rows of K[l*]): A and B
+    # share K and differ in V, C is 10 rows longer with the same last 20 rows at l*. D has
+    # larger keys. Expected: D, then the tied three by descending id (big-endian), under
+    # every delivery order, as the oracle orders them.
+    L, H, d, rl = 4, 2, 64, 2
+    g = torch.Generator(device="cuda:0").manual_seed(77)
+    rnd = lambda T, sc=1.0: (torch.randn((L, H, T, d), generator=g, device="cuda:0") * sc).to(torch.bfloat16)
+    K0 = rnd(20)
+    A = (K0, rnd(20))
+    B = (K0.clone(), rnd(20))
+    KC = rnd(30)
+    KC[rl, :, 10:] = K0[rl]
+    C = (KC, rnd(30))
+    D = (rnd(25, 4.0), rnd(25))
+    frags = [A, B, C, D]
+    refs = [oracle_fragment(K, V) for K, V in frags]
+    assert len({f.fid for f in refs}) == 4
+    tail = [int(f.Q[-20:].astype(object).sum()) for f in refs]
+    assert tail[0] == tail[1] == tail[2] < tail[3]
+    K_ref, V_ref, o_order = oracle.render(oracle.from_deliveries(refs), THETA)
+    want = [refs[3].fid] + sorted((f.fid for f in refs[:3]), reverse=True)
+    assert [f.fid for f in o_order] == want
+    c = cm.Context(0, THETA)
+    for perm in itertools.permutations(range(4)):
+        S = cm.FragmentSet(c)
+        S.ingest_batch([frags[i] for i in perm])
+        k_out, v_out = empty_out(L, H, S.seq_len(), d)
+        n, order = S.render(k_out, v_out)
+        torch.cuda.synchronize()
+        assert order == want
+        assert np.array_equal(synthetic.to_bits(v_out), V_ref)
+        assert assert_k_parity(synthetic.to_bits(k_out), K_ref) == 0
+        S.close()
+    c.close()
+
+
 # ---------------------------------------------------------------- rotation stress
 
 @pytest.mark.parametrize("theta", [1.0e4, 1.0e6, 5.0e5, 1.0e40])
