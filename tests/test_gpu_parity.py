@@ -548,6 +548,37 @@ def test_exact_ties_order_by_id():
     c.close()
 
 
+def test_rendered_cache_as_a_fragment_is_the_foil(ctx):
+    # Section 4.4's foil: a rendered cache M = render({A, B}) delivered again as a fragment
+    # is a new element; render({M, B}) differs from render({A, B}). The GPU's M hashes to
+    # the oracle's id of the oracle's M, and the second merge equals the oracle's.
+    L, H, d = 3, 2, 64
+    g = torch.Generator(device="cuda:0").manual_seed(88)
+    rnd = lambda T, sc: (torch.randn((L, H, T, d), generator=g, device="cuda:0") * sc).to(torch.bfloat16)
+    A, B = (rnd(23, 2.0), rnd(23, 1.0)), (rnd(17, 0.7), rnd(17, 1.0))
+    S = cm.FragmentSet(ctx)
+    S.ingest_batch([A, B])
+    Mk, Mv = empty_out(L, H, 40, d)
+    S.render(Mk, Mv)
+    torch.cuda.synchronize()
+    refs = [oracle_fragment(K, V) for K, V in (A, B)]
+    K1, V1, _ = oracle.render(oracle.from_deliveries(refs), THETA)
+    m_ref = oracle.make_fragment(K1, V1)
+    T2 = cm.FragmentSet(ctx)
+    res = T2.ingest_batch([(Mk, Mv), B])
+    assert res[0] == (m_ref.fid, False) and res[0][0] not in S.ids()
+    k2, v2 = empty_out(L, H, 57, d)
+    n, order = T2.render(k2, v2)
+    torch.cuda.synchronize()
+    K2, V2, o2 = oracle.render(oracle.from_deliveries([m_ref, refs[1]]), THETA)
+    assert n == 57 and order == [f.fid for f in o2]
+    assert np.array_equal(synthetic.to_bits(v2), V2)
+    assert assert_k_parity(synthetic.to_bits(k2), K2) == 0
+    assert K2.shape != K1.shape
+    S.close()
+    T2.close()
+
+
 # ---------------------------------------------------------------- rotation stress
 
 @pytest.mark.parametrize("theta", [1.0e4, 1.0e6, 5.0e5, 1.0e40])
