@@ -13,6 +13,7 @@ import pytest
 import torch
 
 import oracle
+from oracle.bf16 import is_nan_bits
 import synthetic
 from parity_util import THETA, assert_k_parity, empty_out, gpu_fragments, oracle_fragment
 
@@ -166,6 +167,48 @@ def test_rotation_of_special_values_matches_oracle(ctx):
     ref = oracle.rotate_k(bits, 1000, THETA)
     got = synthetic.to_bits(k_out)[:, :, 1000:]
     assert assert_k_parity(got, ref) == 0
+
+
+# numpy warns when it widens a signalling NaN payload; the oracle's result is still NaN
+@pytest.mark.filterwarnings("ignore:invalid value encountered in cast:RuntimeWarning")
+def test_nan_and_inf_inputs_hash_as_bytes_and_propagate():
+    # NaN and inf are bytes to the content address and IEEE values to the rotation: ids
+    # equal the oracle's, V and the first slot's K (byte copies) keep every NaN payload,
+    # and the rotated K is NaN exactly where the oracle's is (within 1 ulp elsewhere). The
+    # routing layer 1 holds no NaN, so the norm keys stay finite and order the two.
+    L, H, d = 3, 2, 64
+    rng = np.random.default_rng(21)
+    specials = np.array([0x7FC1, 0xFFA0, 0x7F81, 0xFFFF, 0x7F80, 0xFF80], dtype=np.uint16)
+    frags, bits = [], []
+    for T, sc in ((20, 2.0), (33, 0.5)):
+        K = (rng.standard_normal((L, H, T, d)) * sc).astype(np.float32)
+        V = rng.standard_normal((L, H, T, d)).astype(np.float32)
+        kb = (K.view(np.uint32) >> 16).astype(np.uint16)
+        vb = (V.view(np.uint32) >> 16).astype(np.uint16)
+        for arr in (kb, vb):
+            for layer in (0, 2):
+                idx = rng.integers(0, arr[layer].size, size=12)
+                arr[layer].reshape(-1)[idx] = rng.choice(specials, size=12)
+        bits.append((kb, vb))
+        frags.append(tuple(torch.from_numpy(a.view(np.int16)).to("cuda:0").view(torch.bfloat16)
+                           for a in (kb, vb)))
+    refs = [oracle.make_fragment(kb, vb) for kb, vb in bits]
+    c = cm.Context(0, THETA)
+    S = cm.FragmentSet(c)
+    res = S.ingest_batch(frags)
+    assert [r[0] for r in res] == [f.fid for f in refs]
+    k_out, v_out = empty_out(L, H, S.seq_len(), d)
+    n, order = S.render(k_out, v_out)
+    torch.cuda.synchronize()
+    K_ref, V_ref, o_order = oracle.render(oracle.from_deliveries(refs), THETA)
+    assert order == [f.fid for f in o_order] and order[0] == refs[0].fid
+    kg, vg = synthetic.to_bits(k_out), synthetic.to_bits(v_out)
+    assert np.array_equal(vg, V_ref) and np.array_equal(vg[:, :, :20], bits[0][1])
+    assert np.array_equal(kg[:, :, :20], bits[0][0])        # slot 0: bytes, payloads kept
+    assert is_nan_bits(kg[:, :, 20:]).any()
+    assert assert_k_parity(kg, K_ref) == 0
+    S.close()
+    c.close()
 
 
 # ---------------------------------------------------------------- layout, capacity, canaries
