@@ -138,3 +138,41 @@ def test_fast_path_with_verify_on_hit():
     assert res2 == [(res[0][0], True)]
     S.close()
     ctx.close()
+
+
+@pytest.mark.parametrize("seed", range(10))
+def test_random_redeliveries_equal_the_path_off(ctxs, seed):
+    # seeded random merges (the generator of test_gpu_random.py) with every delivery a
+    # separate buffer, re-sent copies in random order and, in every other case, a one-bit
+    # near-duplicate of one fragment; spread over one or two ingest calls, then a union
+    from test_gpu_random import _case
+    off, on = ctxs
+    rng = np.random.default_rng(6000 + seed)
+    frags, deliveries, _ = _case(400 + seed)
+    msgs = [_clone(frags[i]) for i in deliveries]
+    if seed % 2:
+        K, V = _clone(frags[int(rng.integers(0, len(frags)))])
+        K.view(torch.int16).view(-1)[int(rng.integers(0, K.numel()))] ^= 1
+        msgs.insert(int(rng.integers(0, len(msgs) + 1)), (K, V))
+    cut = int(rng.integers(0, len(msgs) + 1))
+    L, H, _, d = frags[0][0].shape
+    results = []
+    for c in (off, on):
+        A, B = cm.FragmentSet(c), cm.FragmentSet(c)
+        res = A.ingest_batch(msgs[:cut]) + B.ingest_batch(msgs[cut:])
+        B.ingest_batch(msgs[:cut])                 # B re-receives A's deliveries
+        A.union(B)
+        k, v = empty_out(L, H, A.seq_len(), d)
+        n, order = A.render(k, v)
+        torch.cuda.synchronize()
+        results.append((res, sorted(A.ids()), n, order, synthetic.to_bits(k), synthetic.to_bits(v)))
+        A.close()
+        B.close()
+    (r0, ids0, n0, o0, k0, v0), (r1, ids1, n1, o1, k1, v1) = results
+    assert r0 == r1 and ids0 == ids1 and n0 == n1 and o0 == o1
+    assert np.array_equal(k0, k1) and np.array_equal(v0, v1)
+    refs = [oracle_fragment(K, V) for K, V in msgs]
+    assert [fid for fid, _ in r0] == [f.fid for f in refs]
+    K_ref, V_ref, o_ref = oracle.render(oracle.from_deliveries(refs), THETA)
+    assert o0 == [f.fid for f in o_ref] and np.array_equal(v0, V_ref)
+    assert assert_k_parity(k0, K_ref) == 0
