@@ -68,6 +68,9 @@ def parse_args():
     p.add_argument("--serve", action="store_true",
                    help="run the serving sweep (64 requests of 3 Qwen3-4B-shaped fragments with "
                         "re-deliveries) instead of the single-merge benchmark")
+    p.add_argument("--paged-layouts", action="store_true",
+                   help="render the workload's merge back to back into a contiguous output and "
+                        "into paged pools of two layouts and two block sizes; one JSON line of times")
     p.add_argument("--group", type=int, default=8,
                    help="serving sweep: requests per cm_ingest_many / cm_render_many call")
     p.add_argument("--workload", default=WORKLOAD, choices=["q4b", "q4b_t512", "q4b_t2048", "q17_n2", "tiny"],
@@ -386,6 +389,77 @@ def whole_job_rate(world: int, steps_per_rank: int, max_elapsed_ms: float) -> fl
 
 # ---------------------------------------------------------------- serving sweep
 
+def run_paged_layouts(args):
+    """The merge of the workload rendered back to back (5 warm-up renders, the median of 20
+    timed by CUDA events) into a contiguous output, into per-layer pools
+    [L][blocks][bs][H][d] (each item's rows land in 256-byte runs for the Qwen3 shapes) and
+    into block-major pools [blocks][L][H][bs][d] (one contiguous run per item when bs is a
+    multiple of the item's rows), bs 16 and 64, through a shuffled block table."""
+    import numpy as np
+    import torch
+    import paper_2607_01308_gb300 as cm
+    import synthetic
+    w = synthetic.WORKLOADS[args.workload]
+    L, H, d = w.num_layers, w.num_kv_heads, w.head_dim
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream(dev)
+    frags = [synthetic.make_fragment_torch(sp, L, H, d, dev) for sp in synthetic.fragment_specs(w)]
+    ctx = cm.Context(0, 1e6)
+    S = cm.FragmentSet(ctx)
+    S.ingest_batch(frags)
+    total = S.seq_len()
+    moved = 2 * sum(K.numel() * 2 + V.numel() * 2 for K, V in frags)
+
+    def median_ms(fn, reps=20, warm=5):
+        for _ in range(warm):
+            fn()
+        ts = []
+        for _ in range(reps):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            torch.cuda.synchronize(dev)
+            ts.append(a.elapsed_time(b))
+        return sorted(ts)[len(ts) // 2]
+
+    out = {}
+    k = torch.empty((L, H, total, d), dtype=torch.bfloat16, device=dev)
+    v = torch.empty_like(k)
+    out["contiguous"] = median_ms(lambda: S.render(k, v, stream))
+    ref_k = k.clone()
+    del v
+    for bs in (16, 64):
+        nb = -(-total // bs)
+        table = torch.from_numpy(np.random.default_rng(bs).permutation(nb).astype(np.int32)).to(dev)
+        for layout in ("per_layer", "block_major"):
+            if layout == "per_layer":
+                shape = (L, nb, bs, H, d)
+                st = dict(stride_layer=nb * bs * H * d, stride_block=bs * H * d,
+                          stride_token=H * d, stride_head=d)
+            else:
+                shape = (nb, L, H, bs, d)
+                st = dict(stride_block=L * H * bs * d, stride_layer=H * bs * d,
+                          stride_head=bs * d, stride_token=d)
+            kp = torch.empty(shape, dtype=torch.bfloat16, device=dev)
+            vp = torch.empty_like(kp)
+            cache = cm.cm_paged_cache(kp.data_ptr(), vp.data_ptr(), table.data_ptr(), nb, bs, **st)
+            out[f"{layout}_bs{bs}"] = median_ms(lambda: cm.cm_render_paged(S.handle, cache, stream))
+            # the pools hold the contiguous render's K (a spot check of the first layer)
+            pos = torch.arange(total, device=dev)
+            blk, off = table.long()[pos // bs], pos % bs
+            got = kp[0, blk, off].permute(1, 0, 2) if layout == "per_layer" else kp[blk, 0, :, off].permute(1, 0, 2)
+            assert torch.equal(got, ref_k[0]), layout
+            del kp, vp
+    S.close()
+    ctx.close()
+    print(json.dumps({"workload": WORKLOAD_TEXT.get(args.workload, args.workload),
+                      "bytes_per_render": moved,
+                      "ms": out, "gbs": {k_: moved / ms / 1e6 for k_, ms in out.items()}}))
+    return 0
+
+
 def run_redeliver(args):
     """Re-delivery (the fault model of Section 5.9): one replica receives each fragment of
     the workload (default: the 4 Qwen3-4B-shaped fragments) R times, every delivery its own byte-identical copy, in a
@@ -612,6 +686,8 @@ def main():
         return run_reference(args)
     if args.redeliver:
         return run_redeliver(args)
+    if args.paged_layouts:
+        return run_paged_layouts(args)
     if args.serve:
         return run_serve(args)
 
