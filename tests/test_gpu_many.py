@@ -291,3 +291,48 @@ def test_eight_warp_render_writes_the_same_bytes(ctx):
     assert torch.equal(bag[0][0].view(torch.int16), bag[1][0].view(torch.int16))
     assert torch.equal(bag[0][1].view(torch.int16), bag[1][1].view(torch.int16))
     ctx8.close()
+
+
+def test_overlapped_groups_match_the_oracle():
+    # the serving loop's overlap: group g renders (8-warp CTAs) on the compute stream while
+    # group g + 1 is hashed on a second stream; every request's cache equals the oracle's
+    c = cm.Context(0, THETA)
+    cm.cm_context_set_render_warps(c.handle, 8)
+    L, H, d = 8, 4, 128
+    rng = np.random.default_rng(31)
+    reqs = []
+    for r in range(9):
+        frags = _fragments(700 + r, [int(t) for t in rng.integers(150, 600, size=3)], L, H, d)
+        deliveries = frags + ([frags[int(rng.integers(0, 3))]] if r % 2 else [])
+        reqs.append((frags, deliveries))
+    outs = [empty_out(L, H, sum(K.shape[2] for K, _ in f), d, fill=CANARY) for f, _ in reqs]
+    stream = torch.cuda.current_stream()
+    s_hash = torch.cuda.Stream()
+    groups = [list(range(g0, g0 + 3)) for g0 in range(0, 9, 3)]
+
+    def ingest(group):
+        sets = [cm.FragmentSet(c) for _ in group]
+        cm.ingest_many([(S, K, V) for S, r in zip(sets, group) for K, V in reqs[r][1]], s_hash)
+        return sets
+
+    s_hash.wait_stream(stream)
+    sets = ingest(groups[0])
+    lens, held = [], []
+    for gi, group in enumerate(groups):
+        stream.wait_stream(s_hash)
+        lens += cm.render_many([(S, *outs[r]) for S, r in zip(sets, group)], stream)
+        held += sets
+        if gi + 1 < len(groups):
+            sets = ingest(groups[gi + 1])
+    stream.wait_stream(s_hash)
+    torch.cuda.synchronize()
+    for r, (frags, _) in enumerate(reqs):
+        refs = [oracle_fragment(K, V) for K, V in frags]
+        K_ref, V_ref, _ = oracle.render(oracle.from_deliveries(refs), THETA)
+        k, v = outs[r]
+        assert lens[r] == K_ref.shape[2]
+        assert np.array_equal(synthetic.to_bits(v), V_ref)
+        assert assert_k_parity(synthetic.to_bits(k), K_ref) == 0
+    for S in held:
+        S.close()
+    c.close()
