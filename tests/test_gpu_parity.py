@@ -694,3 +694,39 @@ def test_two_threads_share_a_context(ctx):
             assert ids == ref.ids()
             assert np.array_equal(vb, V_ref)
             assert assert_k_parity(kb, K_ref) == 0
+
+
+# ---------------------------------------------------------------- resources
+
+def test_contexts_release_device_memory():
+    # contexts created, used (scratch grown by a batch, timing events, the re-delivery fast
+    # path, a render) and destroyed 20 times: the device's free memory returns to where it
+    # was after the first cycle (every tensor here is allocated before the baseline)
+    L, H, d = 4, 4, 128
+    g = torch.Generator(device="cuda:0").manual_seed(99)
+    frags = [((torch.randn((L, H, T, d), generator=g, device="cuda:0")).to(torch.bfloat16),
+              torch.randn((L, H, T, d), generator=g, device="cuda:0").to(torch.bfloat16))
+             for T in (3000, 1700, 900)]
+    copy = (frags[0][0].clone(), frags[0][1].clone())
+    k, v = empty_out(L, H, 5600, d)
+
+    def cycle():
+        c = cm.Context(0, THETA)
+        cm.cm_context_set_timing(c.handle, True)
+        cm.cm_context_set_dedup_by_bytes(c.handle, True)
+        S = cm.FragmentSet(c)
+        S.ingest_batch(frags + [copy])
+        n, _ = S.render(k, v)
+        cm.cm_context_kernel_times(c.handle, reset=True)
+        S.close()
+        c.close()
+        return n
+
+    assert cycle() == 5600
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    for _ in range(20):
+        cycle()
+    torch.cuda.synchronize()
+    free1 = torch.cuda.mem_get_info()[0]
+    assert free0 - free1 < (4 << 20), (free0, free1)
