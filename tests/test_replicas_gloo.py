@@ -49,3 +49,18 @@ def test_single_process_identity():
     import bench
     assert bench.max_over_ranks(3.5, torch.device("cpu")) == 3.5
     assert bench.whole_job_rate(1, 10, 100.0) == pytest.approx(100.0)
+
+
+def test_reference_arm_runs_on_rank_zero_only():
+    # under torchrun every rank starts bench.py --impl reference; ranks other than 0 exit 0
+    # at once, without work or output (rank 0 alone times the oracle and prints the line)
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = dict(os.environ, RANK="1", LOCAL_RANK="1", WORLD_SIZE="2",
+               MASTER_ADDR="127.0.0.1", MASTER_PORT=str(_free_port()))
+    r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--gpus", "2",
+                        "--steps", "1", "--warmup", "3"],
+                       cwd=root, env=env, capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0, r.stderr
+    assert r.stdout.strip() == ""
