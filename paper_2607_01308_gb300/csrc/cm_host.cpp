@@ -474,7 +474,10 @@ struct Slot {
 cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t L, int32_t H,
                        int32_t d, cudaStream_t stream, uint32_t withhold_warp = 0,
                        const cm_paged_cache *paged = nullptr) {
-    const int rows_per_chunk = cm::kChunkBytes / (2 * d);
+    // the failure-injection hook withholds a TMA copy, so it runs the half-SM kernel (the
+    // only one that waits)
+    const int warps = withhold_warp ? 8 : ctx->render_warps;
+    const int rows_per_chunk = (int)cm::render_item_bytes(warps) / (2 * d);
     const int half = d / 2;
     const int max_group = std::min<int>(cm::kMaxSlots, cm::kMaxTablePairs / half);
     const uint64_t planes = 2ull * L * H;
@@ -546,9 +549,9 @@ cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t 
             p->stride_head = paged->stride_head;
             p->stride_token = paged->stride_token;
         }
-        const int grid = (int)std::max<uint64_t>(1, std::min<uint64_t>(chunk, ctx->num_sms));
+        const int grid = cm::render_grid(chunk, ctx->num_sms, warps);
         CM_CUDA_TRY(timed_launch(ctx, kTimeRender, stream,
-                                 [&] { return cm::launch_render(*p, grid, ctx->render_warps, stream); }),
+                                 [&] { return cm::launch_render(*p, grid, warps, stream); }),
                     "render launch");
     }
     return CM_OK;

@@ -14,7 +14,6 @@ namespace cm {
 // ---------------------------------------------------------------- render
 constexpr int kMaxSlots = 32;          // fragments per render launch
 constexpr int kMaxTablePairs = 1792;   // sum over slots of head_dim / 2
-constexpr int kChunkBytes = 4096;      // bytes of one source plane handled per work item
 
 struct RenderSlot {
     const void *k;              // source K [L][H][T][d], device
@@ -38,7 +37,7 @@ struct RenderParams {
     int32_t num_heads;
     int32_t head_dim;
     int32_t num_slots;
-    int32_t rows_per_chunk;     // kChunkBytes / (2 d)
+    int32_t rows_per_chunk;     // render_item_bytes(warps) / (2 d)
     int32_t log2_pairs_per_row; // log2(d / 16)
     uint32_t total_chunks;
     uint32_t pad_;
@@ -59,10 +58,16 @@ struct RenderParams {
     double cs[2 * kMaxTablePairs];   // (cos a, sin a) of a = s * theta^(-2j/d), interleaved
 };
 
-// One CTA of `warps` warps (16, or 8 to leave half of each SM's registers to kernels of
-// other streams) per SM; render_prepare() once per device before the first launch.
+// warps = 16: the full-SM render (all of each SM's warp slots it needs, no shared-memory
+// staging); warps = 8: the half-SM render (one 8-warp CTA per SM, leaving half of each
+// SM's registers to kernels of other streams). A launch group's work items are row
+// chunks of render_item_bytes(warps) bytes of one source plane; render_grid gives the
+// launch's CTA count for `chunks` items. render_prepare() once per device before the
+// first launch.
 cudaError_t launch_render(const RenderParams &p, int grid, int warps, cudaStream_t stream);
 cudaError_t render_prepare();
+uint32_t render_item_bytes(int warps);
+int render_grid(uint64_t chunks, int num_sms, int warps);
 
 // Bounds-checked builds: reads and zeroes the render kernels' violation count on the
 // current device (0 in other builds).

@@ -10,11 +10,17 @@
 // turned by one constant angle a_j = s * theta^(-2j/d) per frequency j (the delta
 // formula of Section 2.3), pairing element j with element j + d/2.
 //
-// Work item: up to 4 KiB of rows of one source plane. A persistent grid of one CTA
-// per SM walks the items, every warp with its own pipeline of 1-D TMA bulk copies
-// through shared memory (see render_kernel). For a rotated K item a lane takes
-// vector v of a row's first half and vector v of its second half: 8 (x, y) pairs
-// that share the lane's 8 (cos, sin) values for the whole item.
+// Two kernels move the items. The full-SM render (render_reg_kernel, the default) has
+// every warp take one (K, V) pair of 1 KiB items at a time: its lanes load both items
+// as 16-byte vectors straight into registers, rotate the K rows, and store both with
+// streaming stores; 24 warps per SM keep about 48 KiB of loads in flight, where HBM
+// serves this mix of reads and writes best (more bytes in flight made the same copy
+// slower). The half-SM render (render_kernel, cm_context_set_render_warps(8)) runs one
+// 8-warp CTA per SM that leaves half of the register file to kernels of other
+// streams; its warps keep three 4 KiB items in flight each as 1-D TMA bulk copies
+// into shared memory, which needs fewer warps for the same bytes in flight. For a
+// rotated K item a lane takes vector v of a row's first half and vector v of its
+// second half: 8 (x, y) pairs that share the lane's 8 (cos, sin) values.
 //
 // Rounding. The result must equal round-to-nearest-even-bf16 of
 // fl64(fl64(x c) - fl64(y s)) (and fl64(fl64(y c) + fl64(x s))), c and s the fp64
@@ -30,6 +36,8 @@
 // so it must stay rare). The output is bit-exact either way.
 #include "cm_bounds.h"
 #include "cm_render_kernels.h"
+
+#include <algorithm>
 
 namespace cm {
 namespace {
@@ -237,7 +245,6 @@ constexpr size_t kTableBytes = sizeof(float4) * kMaxTablePairs;
 // Dynamic shared memory of a CTA of kW warps: the warps' stages, then the (cos, sin) table.
 template <int kW>
 constexpr size_t dyn_smem() { return (size_t)kW * kStages * kItemBytes + kTableBytes; }
-static_assert(kChunkBytes == (int)kItemBytes, "host and kernel disagree on the work item size");
 
 // One work item: up to kItemBytes of one source plane and where it goes.
 struct Item {
@@ -457,9 +464,9 @@ __device__ __forceinline__ float2 split16(double c) {
     return make_float2(c1, __double2float_rn(c - (double)c1));
 }
 
-// Persistent kernel, one CTA of kW warps per SM (16: the whole register file at 128
-// registers a thread; 8: half of it, leaving room for kernels of another stream on
-// the same SMs); every warp runs its own
+// Half-SM render: a persistent kernel with one CTA of kW = 8 warps per SM (half of the
+// register file, leaving room for kernels of other streams on the same SMs); every
+// warp runs its own
 // pipeline over its own items, with no block-wide barrier after set-up. Items come
 // in (K, V) pairs of the same (slot, layer, head, row chunk); a warp takes pairs
 // warp id + m * total warps and does the K item, then the V item, so rotation work
@@ -549,13 +556,242 @@ cudaError_t set_smem_attribute() {
                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn_smem<kW>());
 }
 
-template <int kW>
-cudaError_t launch_width(const RenderParams &p, int grid, cudaStream_t stream) {
-    if (p.paged)
-        render_kernel<true, kW><<<grid, kW * 32, dyn_smem<kW>(), stream>>>(p);
-    else
-        render_kernel<false, kW><<<grid, kW * 32, dyn_smem<kW>(), stream>>>(p);
-    return cudaGetLastError();
+// ---------------------------------------------------------------- full-SM render
+
+constexpr int kRegThreads = 256;           // 8 warps per CTA
+constexpr int kRegBlocksPerSm = 3;         // 24 warps per SM
+constexpr uint32_t kRegItemBytes = 1024;   // one work item: 2 vectors per lane
+constexpr int kRegVecs = kRegItemBytes / 16 / 32;
+
+// A (K, V) item pair: the same rows of one (slot, layer, head) plane of K and of V.
+struct Pair {
+    const uint8_t *ks, *vs;   // sources
+    uint8_t *kd, *vd;         // contiguous: first output row; paged: pool + (layer, head) offset
+    int64_t pos0;             // output position of the first row
+    int32_t rows;
+    int32_t rotate;
+    int32_t cs_index;
+#ifdef CM_DEBUG_BOUNDS
+    const uint8_t *ks_base, *vs_base, *kd_base, *vd_base;
+    uint64_t src_size, dst_size;
+#endif
+};
+
+// The pairs pr = first, first + stride, ... of a warp. Pair pr of a launch is pair
+// pr - chunk_begin / 2 of its slot: row chunk c of (layer, head) plane lhp. Along the
+// stride, (plane, chunk) advance by additions; only entering a slot costs a search
+// and a division.
+struct PairWalk {
+    uint32_t pr, npairs, stride;
+    int si;
+    uint32_t lhp, c, st_l, st_c;
+
+    __device__ __forceinline__ void enter(const RenderParams &p) {
+        si = 0;
+        while (si + 1 < p.num_slots && 2 * pr >= p.slot[si + 1].chunk_begin) ++si;
+        const RenderSlot &S = p.slot[si];
+        const uint32_t local = pr - (S.chunk_begin >> 1);
+        lhp = local / S.chunks_per_plane;
+        c = local - lhp * S.chunks_per_plane;
+        st_l = stride / S.chunks_per_plane;
+        st_c = stride - st_l * S.chunks_per_plane;
+    }
+    __device__ __forceinline__ bool next(const RenderParams &p) {
+        pr += stride;
+        if (pr >= npairs) return false;
+        const uint32_t cpp = p.slot[si].chunks_per_plane;
+        c += st_c;
+        lhp += st_l;
+        if (c >= cpp) {
+            c -= cpp;
+            ++lhp;
+        }
+        if (lhp >= (uint32_t)(p.num_layers * p.num_heads)) enter(p);
+        return true;
+    }
+};
+
+__device__ __forceinline__ Pair pair_of(const RenderParams &p, const PairWalk &w) {
+    const RenderSlot &S = p.slot[w.si];
+    const int64_t row_bytes = (int64_t)p.head_dim * 2;
+    const int64_t row0 = (int64_t)w.c * p.rows_per_chunk;
+    const int64_t left = S.seq_len - row0;
+    Pair q;
+    q.rows = left < p.rows_per_chunk ? (int)left : p.rows_per_chunk;
+    const int64_t so = ((int64_t)w.lhp * S.seq_len + row0) * row_bytes;
+    q.ks = static_cast<const uint8_t *>(S.k) + so;
+    q.vs = static_cast<const uint8_t *>(S.v) + so;
+    if (p.paged) {
+        const uint32_t l32 = w.lhp / (uint32_t)p.num_heads;
+        const int64_t l = l32, h = (int64_t)(w.lhp - l32 * (uint32_t)p.num_heads);
+        const int64_t o = (l * p.stride_layer + h * p.stride_head) * 2;
+        q.kd = static_cast<uint8_t *>(p.k_pool) + o;
+        q.vd = static_cast<uint8_t *>(p.v_pool) + o;
+    } else {
+        const int64_t o = ((int64_t)w.lhp * S.capacity + S.offset + row0) * row_bytes;
+        q.kd = static_cast<uint8_t *>(S.k_out) + o;
+        q.vd = static_cast<uint8_t *>(S.v_out) + o;
+    }
+    q.pos0 = S.offset + row0;
+    q.rotate = S.rotate;
+    q.cs_index = S.table_base;
+#ifdef CM_DEBUG_BOUNDS
+    const uint64_t lh_planes = (uint64_t)p.num_layers * (uint64_t)p.num_heads;
+    q.ks_base = static_cast<const uint8_t *>(S.k);
+    q.vs_base = static_cast<const uint8_t *>(S.v);
+    q.src_size = lh_planes * (uint64_t)S.seq_len * (uint64_t)row_bytes;
+    if (p.paged) {
+        q.kd_base = static_cast<const uint8_t *>(p.k_pool);
+        q.vd_base = static_cast<const uint8_t *>(p.v_pool);
+        q.dst_size = ~0ull - reinterpret_cast<uint64_t>(q.kd_base > q.vd_base ? q.kd_base : q.vd_base);
+    } else {
+        q.kd_base = static_cast<const uint8_t *>(S.k_out);
+        q.vd_base = static_cast<const uint8_t *>(S.v_out);
+        q.dst_size = lh_planes * (uint64_t)S.capacity * (uint64_t)row_bytes;
+    }
+#endif
+    return q;
+}
+
+// The K or V half of a pair as an Item (for the placement helpers).
+__device__ __forceinline__ Item half_item(const Pair &q, bool v) {
+    Item it;
+    it.src = v ? q.vs : q.ks;
+    it.dst = v ? q.vd : q.kd;
+    it.pos0 = q.pos0;
+    it.rows = q.rows;
+    it.bytes = 0;
+    it.rotate = v ? 0 : q.rotate;
+    it.cs_index = q.cs_index;
+#ifdef CM_DEBUG_BOUNDS
+    it.src_base = v ? q.vs_base : q.ks_base;
+    it.src_size = q.src_size;
+    it.dst_base = v ? q.vd_base : q.kd_base;
+    it.dst_size = q.dst_size;
+#endif
+    return it;
+}
+
+// Stores vector v (0 <= v < rows * d / 8) of a copied item.
+template <bool kPaged>
+__device__ __forceinline__ void store_vec(const RenderParams &p, const Item &it, const PagedRows &pr,
+                                          int v, const uint4 &x) {
+    const int log2_vpr = p.log2_pairs_per_row + 1;   // vectors per row = d / 8
+    uint4 *d = row_dst<kPaged>(p, it, v >> log2_vpr, pr) + (v & ((1 << log2_vpr) - 1));
+    if (CM_IN_BOUNDS(d, 16, it.dst_base, it.dst_size)) st_stream(d, x);
+}
+
+// Full-SM render: persistent, kRegBlocksPerSm CTAs of 8 warps per SM, no shared-memory
+// staging and no waits. Per pair, each lane loads its 2 vectors of the K item (for a
+// rotated item: vector v of the first and of the second half of one row, v = lane mod
+// (d/16)) and its 2 vectors of the V item, then stores V, then rotates (slots at a
+// nonzero offset) and stores K. The lane's 8 (cos, sin) values are reloaded only when
+// the slot changes.
+template <bool kPaged>
+__global__ void __launch_bounds__(kRegThreads, kRegBlocksPerSm)
+render_reg_kernel(const __grid_constant__ RenderParams p) {
+    __shared__ float4 tab[kMaxTablePairs];   // (c1, c2, s1, s2) for the second level
+    __shared__ float2 cs32[kMaxTablePairs];  // (c32, s32) = (fl(c1 + c2), fl(s1 + s2))
+    const int half = p.head_dim >> 1;
+    const int n_table = p.num_slots * half;
+    for (int i = threadIdx.x; i < n_table; i += kRegThreads) {
+        const float2 cc = split16(p.cs[2 * i]), ss = split16(p.cs[2 * i + 1]);
+        tab[i] = make_float4(cc.x, cc.y, ss.x, ss.y);
+        cs32[i] = make_float2(__fadd_rn(cc.x, cc.y), __fadd_rn(ss.x, ss.y));
+    }
+    __syncthreads();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    PairWalk w;
+    w.pr = blockIdx.x * (kRegThreads / 32) + warp;
+    w.stride = gridDim.x * (kRegThreads / 32);
+    w.npairs = p.total_chunks / 2;
+    if (w.pr >= w.npairs) return;
+    w.enter(p);
+    const int half_vecs = p.head_dim >> 4;
+    const int vecs_per_row = p.head_dim >> 3;
+    const int log2_hv = p.log2_pairs_per_row;
+    const int lane_v = lane & (half_vecs - 1);
+    int cur = -1;
+    float c[8], s[8];
+    do {
+        const Pair q = pair_of(p, w);
+        const int n_vec = q.rows * vecs_per_row;
+        const int n_pairs = q.rows * half_vecs;
+        const uint4 *ks = reinterpret_cast<const uint4 *>(q.ks);
+        const uint4 *vs = reinterpret_cast<const uint4 *>(q.vs);
+        uint4 rk[kRegVecs], rv[kRegVecs];
+        if (q.rotate) {
+#pragma unroll
+            for (int k = 0; k < kRegVecs / 2; ++k) {
+                const int qq = lane + 32 * k;
+                const int off = (qq >> log2_hv) * vecs_per_row + lane_v;
+                rk[2 * k] = rk[2 * k + 1] = make_uint4(0, 0, 0, 0);
+                if (qq < n_pairs && CM_IN_BOUNDS(ks + off, 16, q.ks_base, q.src_size) &&
+                    CM_IN_BOUNDS(ks + off + half_vecs, 16, q.ks_base, q.src_size)) {
+                    rk[2 * k] = __ldcs(ks + off);
+                    rk[2 * k + 1] = __ldcs(ks + off + half_vecs);
+                }
+            }
+        } else {
+#pragma unroll
+            for (int u = 0; u < kRegVecs; ++u) {
+                const int v = lane + 32 * u;
+                rk[u] = make_uint4(0, 0, 0, 0);
+                if (v < n_vec && CM_IN_BOUNDS(ks + v, 16, q.ks_base, q.src_size)) rk[u] = __ldcs(ks + v);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kRegVecs; ++u) {
+            const int v = lane + 32 * u;
+            rv[u] = make_uint4(0, 0, 0, 0);
+            if (v < n_vec && CM_IN_BOUNDS(vs + v, 16, q.vs_base, q.src_size)) rv[u] = __ldcs(vs + v);
+        }
+        const Item vi = half_item(q, true);
+        PagedRows pv{};
+        if (kPaged) pv = paged_rows(p, vi);
+#pragma unroll
+        for (int u = 0; u < kRegVecs; ++u)
+            if (lane + 32 * u < n_vec) store_vec<kPaged>(p, vi, pv, lane + 32 * u, rv[u]);
+        const Item ki = half_item(q, false);
+        PagedRows pk{};
+        if (kPaged) pk = paged_rows(p, ki);
+        if (q.rotate) {
+            if (q.cs_index != cur) {
+                cur = q.cs_index;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const float2 t = cs32[cur + 8 * lane_v + e];
+                    c[e] = t.x;
+                    s[e] = t.y;
+                }
+            }
+#pragma unroll
+            for (int k = 0; k < kRegVecs / 2; ++k) {
+                const int qq = lane + 32 * k;
+                if (qq < n_pairs) {
+                    // copies, not references into rk: the non-inlined fixup must not
+                    // force the register arrays into local memory
+                    const uint4 a = rk[2 * k], b = rk[2 * k + 1];
+                    uint4 ao, bo;
+                    uint32_t b0, b1, b2, b3;
+                    rotate_word(a.x, b.x, c[0], s[0], c[1], s[1], ao.x, bo.x, b0);
+                    rotate_word(a.y, b.y, c[2], s[2], c[3], s[3], ao.y, bo.y, b1);
+                    rotate_word(a.z, b.z, c[4], s[4], c[5], s[5], ao.z, bo.z, b2);
+                    rotate_word(a.w, b.w, c[6], s[6], c[7], s[7], ao.w, bo.w, b3);
+                    if ((b0 | b1 | b2 | b3) != 0u)
+                        fixup_pair(p, tab, cur + 8 * lane_v, a, b, b0, b1, b2, b3, ao, bo);
+                    uint4 *d = row_dst<kPaged>(p, ki, qq >> log2_hv, pk) + lane_v;
+                    if (CM_IN_BOUNDS(d, 16, ki.dst_base, ki.dst_size)) st_stream(d, ao);
+                    if (CM_IN_BOUNDS(d + half_vecs, 16, ki.dst_base, ki.dst_size))
+                        st_stream(d + half_vecs, bo);
+                }
+            }
+        } else {
+#pragma unroll
+            for (int u = 0; u < kRegVecs; ++u)
+                if (lane + 32 * u < n_vec) store_vec<kPaged>(p, ki, pk, lane + 32 * u, rk[u]);
+        }
+    } while (w.next(p));
 }
 
 }  // namespace
@@ -563,16 +799,33 @@ cudaError_t launch_width(const RenderParams &p, int grid, cudaStream_t stream) {
 CM_DEFINE_BOUNDS_READER(take_render_bounds_violations)
 
 cudaError_t render_prepare() {
-    cudaError_t e = set_smem_attribute<false, 16>();
-    if (e == cudaSuccess) e = set_smem_attribute<true, 16>();
-    if (e == cudaSuccess) e = set_smem_attribute<false, 8>();
+    cudaError_t e = set_smem_attribute<false, 8>();
     if (e == cudaSuccess) e = set_smem_attribute<true, 8>();
     return e;
 }
 
+uint32_t render_item_bytes(int warps) { return warps == 8 ? kItemBytes : kRegItemBytes; }
+
+int render_grid(uint64_t chunks, int num_sms, int warps) {
+    if (warps == 8) return (int)std::max<uint64_t>(1, std::min<uint64_t>(chunks, (uint64_t)num_sms));
+    const uint64_t ctas = (chunks / 2 + kRegThreads / 32 - 1) / (kRegThreads / 32);
+    return (int)std::max<uint64_t>(1, std::min<uint64_t>(ctas, (uint64_t)kRegBlocksPerSm * num_sms));
+}
+
 cudaError_t launch_render(const RenderParams &p, int grid, int warps, cudaStream_t stream) {
     if (p.total_chunks == 0) return cudaSuccess;
-    return warps == 8 ? launch_width<8>(p, grid, stream) : launch_width<16>(p, grid, stream);
+    if (warps == 8) {
+        if (p.paged)
+            render_kernel<true, 8><<<grid, 8 * 32, dyn_smem<8>(), stream>>>(p);
+        else
+            render_kernel<false, 8><<<grid, 8 * 32, dyn_smem<8>(), stream>>>(p);
+    } else {
+        if (p.paged)
+            render_reg_kernel<true><<<grid, kRegThreads, 0, stream>>>(p);
+        else
+            render_reg_kernel<false><<<grid, kRegThreads, 0, stream>>>(p);
+    }
+    return cudaGetLastError();
 }
 
 }  // namespace cm

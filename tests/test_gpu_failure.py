@@ -1,8 +1,9 @@
-"""Failure detection on the GPU without a fault: every wait of the render kernel
-on its own TMA copies is bounded (about one second); when one runs out, the warp
-records the failure in the context and returns. A test-only hook withholds one
-copy so that the wait runs out; the host must read CM_ERR_TIMEOUT and the context
-must stay usable. Re-delivery (the paper's fault model, Section 5.9) is covered by
+"""Failure detection on the GPU without a fault: every wait of the half-SM render
+kernel on its own TMA copies is bounded (about one second); when one runs out, the
+warp records the failure in the context and returns. A test-only hook withholds one
+copy so that the wait runs out (the hook always runs that kernel: the full-SM render
+loads into registers and has no waits); the host must read CM_ERR_TIMEOUT and the
+context must stay usable, with either render width set. Re-delivery (the paper's fault model, Section 5.9) is covered by
 the absorption tests."""
 import numpy as np
 import pytest
