@@ -37,6 +37,7 @@ if ROOT not in sys.path:
 METRIC = "cm_render merged-cache GB/s and % of HBM peak; merges/sec (ingest+union+render)"
 UNIT = "merges/s"
 WORKLOAD = "q4b"
+ROPE_THETA = 1.0e6
 BASE_SEED_REDELIVER = 42 + 997   # delivery order of the re-delivery sweep
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
@@ -47,10 +48,10 @@ FALLBACK_HBM_GBS = 6800.0
 # the maximum SM clock.
 HASH_ALU_OPS_PER_BYTE = 648.0 / 64.0
 ALU_OPS_PER_CLK_PER_SM = 64
-NUM_SMS = 152
 CLOCK_FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
                 "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
-                "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+                "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap,"
+                "clocks.mem")
 
 
 def parse_args():
@@ -60,6 +61,8 @@ def parse_args():
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-extra", action="store_true",
+                   help="skip the Qwen3-1.7B-shaped merge and the 16-request serving measurement")
     p.add_argument("--e2e-steps", type=int, default=None)
     p.add_argument("--redeliver", type=int, default=0, metavar="R",
                    help="re-delivery sweep: every fragment of the workload (--workload, default the "
@@ -160,11 +163,14 @@ class ClockSampler:
         rows = [r for r in csv.reader(io.StringIO(getattr(self, "out", ""))) if len(r) >= 9]
         if not rows:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
-        sm = sorted(float(r[1]) for r in rows if r[1].strip().replace(".", "").isdigit())
-        mx = [float(r[2]) for r in rows if r[2].strip().replace(".", "").isdigit()]
+        num = lambda x: x.strip().replace(".", "").isdigit()
+        sm = sorted(float(r[1]) for r in rows if num(r[1]))
+        mx = [float(r[2]) for r in rows if num(r[2])]
+        mem = sorted(float(r[9]) for r in rows if len(r) > 9 and num(r[9]))
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         reasons = sorted({names[i] for r in rows for i in range(4) if "Active" == r[5 + i].strip()})
         return {"sm_mhz": sm[len(sm) // 2] if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "mem_mhz": mem[len(mem) // 2] if mem else None,
                 "reasons": reasons, "samples": len(rows)}
 
 
@@ -214,54 +220,34 @@ def sm_max_mhz():
 
 # ---------------------------------------------------------------- CPU oracle (baseline leg)
 
-def oracle_sample_parts(layers=1, w=None):
-    """The oracle as it stands on a bounded sample of the workload: the first `layers`
-    layers of each of the 4 fragments (T = 4096). Returns (seconds of the per-layer work,
-    seconds of the norm key): the content address and the render cost the same per layer,
-    so a full merge takes num_layers / layers times the first; the routing-layer norm key
-    covers one layer of each fragment in a full merge as in the sample, so its time is
-    taken as it is."""
-    import numpy as np
-    import oracle
+def oracle_fragments(w):
+    """The workload's fragments as the oracle takes them (numpy uint16 bits, made on the CPU)."""
     import synthetic
+    return [synthetic.make_fragment_bits(s, w.num_layers, w.num_kv_heads, w.head_dim)
+            for s in synthetic.fragment_specs(w)]
+
+
+def oracle_merge_seconds(frags, w) -> float:
+    """One whole merge by the oracle as it stands, as the GPU step does it: replica A ingests
+    the first half of the fragments, replica B the rest (content address and routing-layer
+    norm key per fragment), A := A u B, render A. Returns the wall time of that work
+    (fragment generation excluded)."""
+    import oracle
     from oracle.content_address import fragment_id
     from oracle.norm import norm_key
-    w = w or synthetic.WORKLOADS[WORKLOAD]
-    specs = synthetic.fragment_specs(w)
-    frags = [synthetic.make_fragment_bits(s, layers, w.num_kv_heads, w.head_dim) for s in specs]
-    t_layers = t_norm = 0.0
-    A = oracle.FragmentSet()
-    B = oracle.FragmentSet()
+    t0 = time.perf_counter()
+    A, B = oracle.FragmentSet(), oracle.FragmentSet()
+    half = (len(frags) + 1) // 2
     for i, (K, V) in enumerate(frags):
-        t0 = time.perf_counter()
-        fid = fragment_id(K, V)
-        t1 = time.perf_counter()
-        Q = norm_key(K, layers // 2)
-        t2 = time.perf_counter()
-        f = oracle.Fragment(K, V, fid, Q)
-        if i < 2:
+        f = oracle.Fragment(K, V, fragment_id(K, V), norm_key(K, w.num_layers // 2))
+        if i < half:
             A = oracle.ingest(A, f)
         else:
             B = oracle.ingest(B, f)
-        t3 = time.perf_counter()
-        t_layers += (t1 - t0) + (t3 - t2)
-        t_norm += t2 - t1
-    t0 = time.perf_counter()
-    S = oracle.union(A, B)
-    K_out, V_out, _ = oracle.render(S, synthetic.ROPE_THETA)
-    t_layers += time.perf_counter() - t0
-    assert K_out.shape[2] == sum(s.seq_len for s in specs)
-    return t_layers, t_norm
-
-
-def oracle_sample_seconds(layers=1, w=None):
-    """(estimated seconds of one full merge, seconds the sample took): the per-layer work
-    (content address, union and render) scaled by num_layers / layers, the norm key as it
-    is (see oracle_sample_parts)."""
-    import synthetic
-    w = w or synthetic.WORKLOADS[WORKLOAD]
-    t_layers, t_norm = oracle_sample_parts(layers, w)
-    return t_layers * w.num_layers / layers + t_norm, t_layers + t_norm
+    K_out, V_out, _ = oracle.render(oracle.union(A, B), ROPE_THETA)
+    dt = time.perf_counter() - t0
+    assert K_out.shape[2] == sum(K.shape[2] for K, _ in frags)
+    return dt
 
 
 def host_cpu():
@@ -278,91 +264,90 @@ def host_cpu():
     return {"model": model, "os_cpu_count": os.cpu_count()}
 
 
-def cpu_baseline_entry(layers=24):
-    import synthetic
-    w = synthetic.WORKLOADS[WORKLOAD]
-    per_merge, dt = oracle_sample_seconds(layers, w)
-    merged = sum(s.seq_len for s in synthetic.fragment_specs(w))
-    return {"value": 1.0 / per_merge, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "render_bytes_gbs": 2 * merged * w.bytes_per_token / per_merge / 1e9,
+def cpu_baseline_entry(w):
+    """The oracle on one host core: one whole merge of the workload, measured (no scaling)."""
+    frags = oracle_fragments(w)
+    dt = oracle_merge_seconds(frags, w)
+    merged = sum(K.shape[2] for K, _ in frags)
+    return {"value": 1.0 / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "render_bytes_gbs": 2 * merged * w.bytes_per_token / dt / 1e9,
             "host": host_cpu(),
-            "sample": f"one merge restricted to the first {layers} of {w.num_layers} layers "
-                      f"(4 fragments x 4096 tokens; ingest + union + render), timed once "
-                      f"({dt:.2f} s); content address and render scaled by {w.num_layers}/{layers}, "
-                      f"the routing-layer norm key (one layer per fragment either way) unscaled; "
+            "sample": f"one whole merge of the workload ({len(frags)} fragments: 2 replicas ingest, "
+                      f"union, render), timed once ({dt:.2f} s, fragment generation excluded); "
                       f"single thread (numpy fp64 + hashlib)",
-            "seconds_per_merge": per_merge}
+            "seconds_per_merge": dt}
 
 
-def _oracle_worker(layers: int):
-    """One process of the multi-core estimate: the oracle's compute seconds on a sample of
-    `layers` layers of the headline merge (fragment generation not included), split into
-    the per-layer work and the routing-layer norm key."""
+_WORKER_FRAGS = None
+
+
+def _oracle_worker_init(workload: str):
+    """Each oracle process of the reference arm makes the workload's fragments once."""
+    global _WORKER_FRAGS
+    os.environ["OMP_NUM_THREADS"] = "1"
     import synthetic
-    return oracle_sample_parts(layers, synthetic.WORKLOADS[WORKLOAD])
+    _WORKER_FRAGS = (workload, oracle_fragments(synthetic.WORKLOADS[workload]))
 
 
-def _oracle_ready(_):
-    import numpy  # noqa: F401
-    import oracle  # noqa: F401
-    import synthetic  # noqa: F401
-    return os.getpid()
-
-
-def cpu_baseline_multicore(layers_per_core=2):
-    """The oracle split by layer over every host core (a secondary CPU figure): one
-    process per core runs the single-thread sample on its own `layers_per_core` layers at
-    the same time; the slowest process's compute time, scaled to the merge's layer count,
-    estimates a merge on all cores (the upper levels of the hash tree, which span layers,
-    are counted per sample as in the single-core estimate)."""
-    import multiprocessing as mp
+def _oracle_worker_merge(_):
     import synthetic
-    w = synthetic.WORKLOADS[WORKLOAD]
+    name, frags = _WORKER_FRAGS
+    return oracle_merge_seconds(frags, synthetic.WORKLOADS[name])
+
+
+def reference_processes(w) -> int:
+    """Oracle processes that fit this host: one per core, each allowed 6 times the
+    workload's fragment bytes of memory (a whole merge of the 2.4 GB Qwen3-4B-shaped
+    workload peaks near 10 GB), at least 1."""
+    import synthetic
     cores = os.cpu_count() or 1
-    pool_ctx = mp.get_context("spawn")     # this process already holds a CUDA context
-    with pool_ctx.Pool(cores) as pool:
-        pool.map(_oracle_ready, range(cores))
-        parts = pool.map(_oracle_worker, [layers_per_core] * cores)
-    t_layers = max(p[0] for p in parts)
-    t_norm = max(p[1] for p in parts)
-    per_merge = t_layers * w.num_layers / (cores * layers_per_core) + t_norm
-    merged = sum(s.seq_len for s in synthetic.fragment_specs(w))
-    return {"value": 1.0 / per_merge, "unit": UNIT, "cores": cores, "kind": "oracle",
-            "estimate": True,
-            "render_bytes_gbs": 2 * merged * w.bytes_per_token / per_merge / 1e9,
-            "sample": f"{cores} processes, each the single-thread sample on {layers_per_core} "
-                      f"layers at once (slowest per-layer work {t_layers:.2f} s, scaled by "
-                      f"{w.num_layers}/({cores} x {layers_per_core}); norm key {t_norm:.2f} s, "
-                      f"unscaled)",
-            "seconds_per_merge": per_merge}
+    avail = None
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    avail = int(line.split()[1]) * 1024
+    except OSError:
+        pass
+    frag_bytes = sum(s.seq_len for s in synthetic.fragment_specs(w)) * w.bytes_per_token
+    per = max(8e9, 6.0 * frag_bytes)
+    fit = int(avail // per) if avail else 1
+    return max(1, min(cores, fit))
 
 
 def run_reference(args):
+    """The oracle as it stands, each step one whole merge of the workload, the steps run
+    by a pool of single-thread processes on the host's cores (one merge per process at a
+    time): W warm-up merges, then K timed merges; value = K / the wall time of the K."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
     os.environ.setdefault("OMP_NUM_THREADS", "1")
+    import multiprocessing as mp
     import synthetic
     w = synthetic.WORKLOADS[WORKLOAD]
-    layers = 1
-    for _ in range(args.warmup):
-        oracle_sample_seconds(layers, w)
-    total = 0.0
-    for _ in range(args.steps):
-        total += oracle_sample_seconds(layers, w)[0]
-    value = args.steps / total
+    procs = reference_processes(w)
+    with mp.get_context("spawn").Pool(procs, initializer=_oracle_worker_init,
+                                      initargs=(WORKLOAD,)) as pool:
+        if args.warmup:
+            pool.map(_oracle_worker_merge, range(args.warmup), chunksize=1)
+        t0 = time.perf_counter()
+        per = pool.map(_oracle_worker_merge, range(args.steps), chunksize=1)
+        wall = time.perf_counter() - t0
+    value = args.steps / wall
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": 1000.0 * total / args.steps, "higher_is_better": True,
+        "ms_per_step": 1000.0 * wall / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "u16 bits / f64", "data": "synthetic",
         "config": workload_config(w),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": procs, "kind": "oracle",
                          "host": host_cpu(),
-                         "sample": f"each step: one merge restricted to the first {layers} of "
-                                   f"{w.num_layers} layers; content address and render scaled by "
-                                   f"{w.num_layers}, the routing-layer norm key unscaled; single "
-                                   f"thread"},
+                         "seconds_per_merge_per_process": sum(per) / len(per),
+                         "sample": f"each step one whole merge of the workload (2 replicas "
+                                   f"ingest, union, render), measured; {procs} single-thread "
+                                   f"processes run the steps side by side, value = steps / wall "
+                                   f"time of the timed steps ({wall:.1f} s)"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -530,42 +515,44 @@ def run_redeliver(args):
     return 0
 
 
-def run_serve(args):
-    """64 independent merge requests on the Qwen3-4B shape: each delivers its 3 fragments
-    (lengths U{512..4096}, each re-sent with probability 0.1, in shuffled order) into a fresh
-    set, which is then rendered. Every delivery is its own device buffer. Timed four ways:
-    one request at a time (a batched ingest and a render per request); `--group` requests at
-    a time (one cm_ingest_many and one cm_render_many per group, each request rendering into
-    its own output buffer); grouped with each group's render (8-warp CTAs) running while
-    the next group hashes on a second stream; and that with the re-delivery fast path on
-    (the line's value)."""
-    import torch
+def serve_requests(w, dev, n_requests):
+    """The first n_requests requests of the serving workload: each delivers its 3 fragments
+    (lengths U{512..4096}, each re-sent with probability 0.1, in shuffled order); every
+    delivery is its own device buffer. Returns [(descriptors, tensors, merged tokens)]."""
     import paper_2607_01308_gb300 as cm
     import synthetic
-    w = synthetic.WORKLOADS["serve"]
-    dev = torch.device("cuda", 0)
-    torch.cuda.set_device(dev)
     reqs = []
-    for r in range(w.num_requests):
+    for r in range(n_requests):
         specs = synthetic.fragment_specs(w, r)
         frags = [synthetic.make_fragment_torch(sp, w.num_layers, w.num_kv_heads, w.head_dim, dev)
                  for sp in specs]
-        sched = synthetic.delivery_schedule(w, r)
         seen, msgs = set(), []
-        for i in sched:
+        for i in synthetic.delivery_schedule(w, r):
             K, V = frags[i]
             msgs.append((K, V) if i not in seen else (K.clone(), V.clone()))
             seen.add(i)
         reqs.append(([cm.fragment_from_tensors(K, V) for K, V in msgs], msgs,
                      sum(sp.seq_len for sp in specs)))
+    return reqs
+
+
+def serve_modes(ctx, reqs, w, dev, G, modes):
+    """Times the requests (after one untimed pass) in each of `modes`:
+      per_request         a batched ingest and a render per request
+      grouped             G requests per cm_ingest_many and per cm_render_many
+      grouped_overlapped  grouped, each group's render (8-warp CTAs) running while the
+                          next group hashes on a second stream
+      grouped_overlapped_dedup  that with the re-delivery fast path on
+    Returns {mode: summary}."""
+    import torch
+    import paper_2607_01308_gb300 as cm
     cap = max(t for _, _, t in reqs)
-    G = max(1, args.group)
+    G = max(1, G)
     outs = []
     for _ in range(G):
         k_out = torch.empty((w.num_layers, w.num_kv_heads, cap, w.head_dim), dtype=torch.bfloat16,
                             device=dev)
         outs.append((k_out, torch.empty_like(k_out)))
-    ctx = cm.Context(0, synthetic.ROPE_THETA)
     stream = torch.cuda.current_stream(dev)
 
     def one(req):
@@ -590,9 +577,6 @@ def run_serve(args):
         for s in sets:
             cm.cm_set_destroy(s)
 
-    def grouped(group):
-        render_group(ingest_group(group, stream), stream)
-
     s_hash = torch.cuda.Stream(dev)
 
     def overlapped(rs):
@@ -608,13 +592,21 @@ def run_serve(args):
                 sets = ingest_group(groups[gi + 1], s_hash)
         stream.wait_stream(s_hash)
 
+    def per_request(rs):
+        for req in rs:
+            one(req)
+
+    def per_group(rs):
+        for g0 in range(0, len(rs), G):
+            render_group(ingest_group(rs[g0:g0 + G], stream), stream)
+
     def timed(run_all):
         run_all(reqs)                           # warm-up: grows the scratch to its steady size
         torch.cuda.synchronize(dev)
         cm.cm_context_kernel_times(ctx.handle, reset=True)
         cm.cm_context_set_timing(ctx.handle, True)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        with ClockSampler(0) as clocks:
+        with ClockSampler(dev.index or 0) as clocks:
             e0.record(stream)
             run_all(reqs)
             e1.record(stream)
@@ -622,14 +614,6 @@ def run_serve(args):
         cm.cm_context_set_timing(ctx.handle, False)
         kt = cm.cm_context_kernel_times(ctx.handle, reset=True)
         return e0.elapsed_time(e1), kt, clocks.summary()
-
-    def per_request(rs):
-        for req in rs:
-            one(req)
-
-    def per_group(rs):
-        for g0 in range(0, len(rs), G):
-            grouped(rs[g0:g0 + G])
 
     render_bytes = sum(2 * t * w.bytes_per_token for _, _, t in reqs)
     peak, _ = hbm_peak()
@@ -640,45 +624,188 @@ def run_serve(args):
                 "render_gbs": render_gbs, "render_frac_of_measured_hbm": render_gbs / peak,
                 "render_ms_per_request": kt["render_ms"] / len(reqs),
                 "hash_ms_per_request": (kt["leaf_hash_ms"] + kt["inner_hash_ms"]) / len(reqs),
-                "kernel_launches": kt["leaf_hash_launches"] + kt["inner_hash_launches"] + kt["aux_launches"]
-                + kt["render_launches"]}
+                "kernel_launches": kt["leaf_hash_launches"] + kt["inner_hash_launches"] +
+                kt["aux_launches"] + kt["render_launches"]}
 
-    ms1, kt1, clocks1 = timed(per_request)
-    msg, ktg, clocksg = timed(per_group)
-    cm.cm_context_set_render_warps(ctx.handle, 8)
-    mso, kto, clockso = timed(overlapped)
-    cm.cm_context_set_dedup_by_bytes(ctx.handle, True)
-    msd, ktd, clocksd = timed(overlapped)
-    cm.cm_context_set_dedup_by_bytes(ctx.handle, False)
-    cm.cm_context_set_render_warps(ctx.handle, 16)
-    single = summary(ms1, kt1)
-    group = summary(msg, ktg)
-    ovl = summary(mso, kto)
-    ovl_dedup = summary(msd, ktd)
+    out = {}
+    for mode in modes:
+        overlap = mode.startswith("grouped_overlapped")
+        if overlap:
+            cm.cm_context_set_render_warps(ctx.handle, 8)
+        cm.cm_context_set_dedup_by_bytes(ctx.handle, mode.endswith("_dedup"))
+        run = {"per_request": per_request, "grouped": per_group}.get(mode, overlapped)
+        ms, kt, clocks = timed(run)
+        out[mode] = dict(summary(ms, kt), clocks=clocks)
+        cm.cm_context_set_dedup_by_bytes(ctx.handle, False)
+        cm.cm_context_set_render_warps(ctx.handle, 16)
+    return out
+
+
+def run_serve(args):
+    """64 independent merge requests on the Qwen3-4B shape, timed four ways (serve_modes);
+    the line's value is grouped_overlapped_dedup."""
+    import torch
+    import paper_2607_01308_gb300 as cm
+    import synthetic
+    w = synthetic.WORKLOADS["serve"]
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    reqs = serve_requests(w, dev, w.num_requests)
+    ctx = cm.Context(0, synthetic.ROPE_THETA)
+    modes = serve_modes(ctx, reqs, w, dev, args.group,
+                        ["per_request", "grouped", "grouped_overlapped", "grouped_overlapped_dedup"])
     line = {
-        "mode": "serving sweep", "metric": METRIC, "value": ovl_dedup["value"], "unit": UNIT,
-        "n_gpus": 1, "requests": len(reqs), "higher_is_better": True, "dtype": "bf16",
+        "mode": "serving sweep", "metric": METRIC, "value": modes["grouped_overlapped_dedup"]["value"],
+        "unit": UNIT, "n_gpus": 1, "requests": len(reqs), "higher_is_better": True, "dtype": "bf16",
         "data": "synthetic",
         "config": {"workload": "serving sweep on the Qwen3-4B shape: 64 requests x 3 fragments, "
                                "T ~ U{512..4096}, each delivery re-sent with p = 0.1",
                    "deliveries": sum(len(fd) for fd, _, _ in reqs),
                    "merged_tokens": sum(t for _, _, t in reqs),
-                   "group": G},
-        "grouped_overlapped": dict(ovl, clocks=clockso,
-                                   note="8-warp render CTAs; group g renders while group g+1 "
-                                        "hashes on a second stream, so the kernel times overlap"),
-        "grouped_overlapped_dedup": dict(ovl_dedup, clocks=clocksd,
-                                         note="as grouped_overlapped, with the re-delivery fast "
-                                              "path on (re-sent copies are compared, not hashed)"),
-        "grouped": dict(group, clocks=clocksg),
-        "per_request": dict(single, clocks=clocks1),
+                   "group": args.group},
     }
+    line.update(modes)
+    line["grouped_overlapped"]["note"] = ("8-warp render CTAs; group g renders while group g+1 "
+                                          "hashes on a second stream, so the kernel times overlap")
+    line["grouped_overlapped_dedup"]["note"] = ("as grouped_overlapped, with the re-delivery fast "
+                                                "path on (re-sent copies are compared, not hashed)")
     print(json.dumps(line), flush=True)
     ctx.close()
     return 0
 
 
 # ---------------------------------------------------------------- GPU arm
+
+# BLAKE2s work per 64-byte block of the content address: 10 rounds x 8 G, each G 6 additions,
+# 4 xors and 4 rotations, then 16 xors of the finalisation: 1136 two-input integer operations,
+# of which the 648 xors and rotations (three-input xors counted once) must issue on the
+# integer ALU pipe.
+HASH_INT_OPS_PER_BLOCK = 10 * 8 * (6 + 4 + 4) + 16
+
+
+def grouped_ms(fn, stream, groups=6, per=10):
+    """Median per-call device time of `fn` called back to back: `groups` groups of `per`
+    calls, each group bracketed by CUDA events on `stream` (the host enqueues ahead of the
+    GPU, so launch latency is hidden), after 3 warm-up calls."""
+    import torch
+    for _ in range(3):
+        fn()
+    torch.cuda.synchronize()
+    ts = []
+    for _ in range(groups):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(per):
+            fn()
+        b.record(stream)
+        b.synchronize()
+        ts.append(a.elapsed_time(b) / per)
+    ts.sort()
+    return ts[len(ts) // 2], ts
+
+
+def box_copy(dev, nbytes):
+    """This GPU's own copy rate on `nbytes` bytes: torch copy_ (a device-to-device
+    cudaMemcpyAsync), 3 warm-up copies, then 20 timed by CUDA events; read + write bytes."""
+    import torch
+    src = torch.empty(nbytes // 2, dtype=torch.bfloat16, device=dev)
+    dst = torch.empty_like(src)
+    src.fill_(1.0)
+    st = torch.cuda.current_stream(dev)
+    for _ in range(3):
+        dst.copy_(src)
+    ts = []
+    for _ in range(20):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(st)
+        dst.copy_(src)
+        b.record(st)
+        b.synchronize()
+        ts.append(a.elapsed_time(b))
+    ts.sort()
+    del src, dst
+    return {"bytes_moved": 2 * nbytes, "best_ms": ts[0], "median_ms": ts[len(ts) // 2],
+            "best_gbs": 2 * nbytes / (ts[0] * 1e-3) / 1e9,
+            "median_gbs": 2 * nbytes / (ts[len(ts) // 2] * 1e-3) / 1e9,
+            "how": "torch copy_ (device-to-device cudaMemcpyAsync) of the workload's fragment "
+                   "bytes, 20 copies timed by CUDA events after 3 warm-up copies"}
+
+
+def merge_fn(cm, ctx, fdesc, k_out, v_out, total_T, stream):
+    """One whole merge: replica A ingests the first half of the deliveries, replica B the
+    rest (one cm_ingest_many call: one GPU pass, one synchronisation), A := A u B, render A."""
+    def one_merge(timers=None, inputs=None, out=None):
+        k_dst, v_dst = out or (k_out, v_out)
+        a = cm.cm_set_create(ctx.handle)
+        b = cm.cm_set_create(ctx.handle)
+        fd = inputs or fdesc
+        half = (len(fd) + 1) // 2
+        if timers is not None:
+            timers["ingest"][0].record(stream)
+        cm.cm_ingest_many([a] * half + [b] * (len(fd) - half), fd, stream)
+        if timers is not None:
+            timers["ingest"][1].record(stream)
+        cm.cm_union(a, b)   # replica exchange: A := A u B
+        if timers is not None:
+            timers["render"][0].record(stream)
+        n, _ = cm.cm_render(a, k_dst.data_ptr(), v_dst.data_ptr(), total_T, stream,
+                            want_order=False)
+        if timers is not None:
+            timers["render"][1].record(stream)
+        cm.cm_set_destroy(b)
+        cm.cm_set_destroy(a)
+        return n
+    return one_merge
+
+
+def small_merge_entry(cm, dev, name, merges=200):
+    """A whole-merge measurement of a small workload (same step as the headline one), with
+    the render's in-step and back-to-back device times."""
+    import torch
+    import synthetic
+    w = synthetic.WORKLOADS[name]
+    L, H, d = w.num_layers, w.num_kv_heads, w.head_dim
+    frags = [synthetic.make_fragment_torch(s, L, H, d, dev) for s in synthetic.fragment_specs(w)]
+    T = sum(K.shape[2] for K, _ in frags)
+    k_out = torch.empty((L, H, T, d), dtype=torch.bfloat16, device=dev)
+    v_out = torch.empty_like(k_out)
+    ctx = cm.Context(dev.index or 0, synthetic.ROPE_THETA)
+    stream = torch.cuda.current_stream(dev)
+    fdesc = [cm.fragment_from_tensors(K, V) for K, V in frags]
+    one = merge_fn(cm, ctx, fdesc, k_out, v_out, T, stream)
+    for _ in range(10):
+        one()
+    torch.cuda.synchronize(dev)
+    cm.cm_context_kernel_times(ctx.handle, reset=True)
+    cm.cm_context_set_timing(ctx.handle, True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(merges):
+        one()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    cm.cm_context_set_timing(ctx.handle, False)
+    kt = cm.cm_context_kernel_times(ctx.handle, reset=True)
+    ms = e0.elapsed_time(e1) / merges
+    S = cm.FragmentSet(ctx)
+    S.ingest_batch(frags)
+    b2b, _ = grouped_ms(lambda: S.render(k_out, v_out, stream), stream, groups=10, per=20)
+    S.close()
+    ctx.close()
+    moved = 2 * T * w.bytes_per_token
+    return {"workload": WORKLOAD_TEXT[name], "value": 1000.0 / ms, "unit": UNIT,
+            "ms_per_merge": ms, "merges": merges,
+            "kernel_ms_per_merge": {"leaf_hash": kt["leaf_hash_ms"] / merges,
+                                    "inner_hash": kt["inner_hash_ms"] / merges,
+                                    "render": kt["render_ms"] / merges},
+            "launches_per_merge": (kt["leaf_hash_launches"] + kt["inner_hash_launches"] +
+                                   kt["render_launches"] + kt["aux_launches"]) / merges,
+            "render_us_in_step": 1000.0 * kt["render_ms"] / merges,
+            "render_us_back_to_back": 1000.0 * b2b,
+            "render_gbs_back_to_back": moved / (b2b * 1e-3) / 1e9,
+            "render_bytes": moved,
+            "render_bar_us": moved / (0.7 * NOMINAL_HBM_GBS * 1e9) * 1e6}
+
 
 def main():
     args = parse_args()
@@ -704,6 +831,7 @@ def main():
         dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
+    num_sms = torch.cuda.get_device_properties(dev).multi_processor_count
 
     w = synthetic.WORKLOADS[args.workload]
     L, H, d = w.num_layers, w.num_kv_heads, w.head_dim
@@ -716,33 +844,9 @@ def main():
     stream = torch.cuda.current_stream(dev)
     fdesc = [cm.fragment_from_tensors(K, V) for K, V in frags]
     render_bytes = 2 * total_T * w.bytes_per_token          # read + write of all K and V
-    hash_bytes = sum(s.seq_len for s in specs) * w.bytes_per_token
-
+    hash_bytes = total_T * w.bytes_per_token
+    one_merge = merge_fn(cm, ctx, fdesc, k_out, v_out, total_T, stream)
     ev = lambda: torch.cuda.Event(enable_timing=True)
-
-    def one_merge(timers=None, inputs=None, out=None):
-        k_dst, v_dst = out or (k_out, v_out)
-        a = cm.cm_set_create(ctx.handle)
-        b = cm.cm_set_create(ctx.handle)
-        fd = inputs or fdesc
-        half = (len(fd) + 1) // 2
-        if timers is not None:
-            timers["ingest"][0].record(stream)
-        # replica A takes the first half of the deliveries, replica B the rest: one
-        # cm_ingest_many call, so one GPU pass and one synchronisation for both
-        cm.cm_ingest_many([a] * half + [b] * (len(fd) - half), fd, stream)
-        if timers is not None:
-            timers["ingest"][1].record(stream)
-        cm.cm_union(a, b)   # replica exchange: A := A u B
-        if timers is not None:
-            timers["render"][0].record(stream)
-        n, _ = cm.cm_render(a, k_dst.data_ptr(), v_dst.data_ptr(), total_T, stream,
-                            want_order=False)
-        if timers is not None:
-            timers["render"][1].record(stream)
-        cm.cm_set_destroy(b)
-        cm.cm_set_destroy(a)
-        return n
 
     for _ in range(args.warmup):
         one_merge()
@@ -750,6 +854,7 @@ def main():
     # register-only integer-ALU rates of this GPU (the ceiling of the content address)
     xor3_tops, compress_tops = cm.cm_measure_int_alu(local_rank)
 
+    # the timed steps: exactly args.steps merges
     step_timers = [{"ingest": (ev(), ev()), "render": (ev(), ev())} for _ in range(args.steps)]
     start, end = ev(), ev()
     if world > 1:
@@ -772,6 +877,26 @@ def main():
     ingest_ms = sum(t["ingest"][0].elapsed_time(t["ingest"][1]) for t in step_timers) / args.steps
     elapsed_ms = max_over_ranks(elapsed_ms, dev)
 
+    # the same step loop again for at least 0.5 s (reported apart: a short timed region
+    # cannot separate the box from the kernels)
+    sustained_steps = max(args.steps, int(500.0 / max(elapsed_ms / args.steps, 1e-3)) + 1)
+    s0, s1 = ev(), ev()
+    torch.cuda.synchronize(dev)
+    with ClockSampler(local_rank) as sclocks:
+        s0.record(stream)
+        for _ in range(sustained_steps):
+            one_merge()
+        s1.record(stream)
+        torch.cuda.synchronize(dev)
+    sustained_ms = max_over_ranks(s0.elapsed_time(s1), dev)
+
+    # the render alone, back to back (device time per launch, launch latency hidden)
+    S = cm.FragmentSet(ctx)
+    S.ingest_batch(frags)
+    render_b2b_ms, render_b2b_all = grouped_ms(lambda: S.render(k_out, v_out, stream), stream)
+    # this GPU's own copy rate on the same bytes
+    copy = box_copy(dev, hash_bytes)
+
     # paged render of the same merge into per-layer block pools [L][blocks][16][H][d] through a
     # shuffled block table (timed apart from the steps, same algorithmic bytes)
     paged_ms = None
@@ -785,19 +910,9 @@ def main():
         cache = cm.cm_paged_cache(pool_k.data_ptr(), pool_v.data_ptr(), table.data_ptr(), nblk, bs,
                                   stride_block=bs * H * d, stride_layer=nblk * bs * H * d,
                                   stride_head=d, stride_token=H * d)
-        ps = cm.cm_set_create(ctx.handle)
-        cm.cm_ingest_batch(ps, fdesc, stream)
-        for _ in range(3):
-            cm.cm_render_paged(ps, cache, stream)
-        pe = [(ev(), ev()) for _ in range(10)]
-        for a_, b_ in pe:
-            a_.record(stream)
-            cm.cm_render_paged(ps, cache, stream)
-            b_.record(stream)
-        torch.cuda.synchronize(dev)
-        paged_ms = sum(a_.elapsed_time(b_) for a_, b_ in pe) / len(pe)
-        cm.cm_set_destroy(ps)
+        paged_ms, _ = grouped_ms(lambda: cm.cm_render_paged(S.handle, cache, stream), stream)
         del pool_k, pool_v
+    S.close()
 
     # end to end through the C ABI with host buffers: every step copies its inputs in from
     # pinned host memory and the whole merged cache out to pinned host memory
@@ -889,6 +1004,24 @@ def main():
                        dev_out[(e2e_steps - 1) % 2][0][:, :, -8:].view(torch.int16))
     serial_step()
     e2e_serial_ms = timed_e2e(lambda: [serial_step() for _ in range(e2e_steps)])
+    del dev_in, dev_desc, dev_out, host_in, host_out
+
+    # the other workloads of the benchmark, measured on rank 0 of a single-GPU run: the
+    # Qwen3-1.7B-shaped 2 x 512-token merge, and the first 16 requests of the serving sweep
+    extra = {}
+    if rank == 0 and world == 1 and args.workload == WORKLOAD and not args.no_extra:
+        extra["q17_n2"] = small_merge_entry(cm, dev, "q17_n2")
+        wserve = synthetic.WORKLOADS["serve"]
+        reqs = serve_requests(wserve, dev, 16)
+        sctx = cm.Context(local_rank, synthetic.ROPE_THETA)
+        modes = serve_modes(sctx, reqs, wserve, dev, 8, ["grouped", "grouped_overlapped_dedup"])
+        sctx.close()
+        extra["serve16"] = {"workload": "the first 16 requests of the serving sweep on the Qwen3-4B "
+                                        "shape (3 fragments each, T ~ U{512..4096}, re-sent with "
+                                        "p = 0.1), 8 requests per call",
+                            "value": modes["grouped_overlapped_dedup"]["value"], "unit": UNIT,
+                            "requests": len(reqs), "modes": modes}
+        del reqs
 
     if rank == 0:
         peak, peak_src = hbm_peak()
@@ -901,21 +1034,38 @@ def main():
         leaf_launches_per_step = max(1, ktimes["leaf_hash_launches"]) / args.steps
         leaf_ms = ktimes["leaf_hash_ms"] / max(1, ktimes["leaf_hash_launches"])
         frag_bytes = hash_bytes / leaf_launches_per_step
+        blocks = frag_bytes / 64.0
         hash_tops = HASH_ALU_OPS_PER_BYTE * frag_bytes / (leaf_ms * 1e-3) / 1e12
-        alu_peak = NUM_SMS * ALU_OPS_PER_CLK_PER_SM * sm_max_mhz() * 1e6 / 1e12
+        hash_int_tops = HASH_INT_OPS_PER_BLOCK * blocks / (leaf_ms * 1e-3) / 1e12
+        clk = sm_max_mhz() * 1e6
+        alu_peak = num_sms * ALU_OPS_PER_CLK_PER_SM * clk / 1e12
+        int_peak = num_sms * 128 * clk / 1e12
         kernel_render_ms = ktimes["render_ms"] / max(1, ktimes["render_launches"])
+        copy_gbs = copy["median_gbs"]
         render_roof = {
-            "kernel": "render_kernel", "bound": "hbm",
+            "kernel": "render_reg_kernel", "bound": "hbm",
             "achieved": render_bytes / (kernel_render_ms * 1e-3) / 1e9, "peak": peak,
             "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
             else "fallback 6.8 TB/s", "unit": "GB/s",
             "frac": render_bytes / (kernel_render_ms * 1e-3) / 1e9 / peak,
             "traffic": profile_traffic("render.cu", "render_kernel_q4b.md"),
             "algorithmic_bytes_per_launch": render_bytes, "ms_per_launch": kernel_render_ms,
+            "timing": "CUDA events on the render's stream around each launch in the timed steps "
+                      "(the stream is idle when the start event is recorded, so each interval "
+                      "includes the launch's own latency)",
+            "back_to_back_ms": render_b2b_ms,
+            "back_to_back_gbs": render_bytes / (render_b2b_ms * 1e-3) / 1e9,
+            "back_to_back_frac": render_bytes / (render_b2b_ms * 1e-3) / 1e9 / peak,
+            "back_to_back_groups_ms": render_b2b_all,
+            "frac_of_same_box_copy": render_bytes / (kernel_render_ms * 1e-3) / 1e9 / copy_gbs,
+            "back_to_back_frac_of_same_box_copy": render_bytes / (render_b2b_ms * 1e-3) / 1e9 / copy_gbs,
+            "frac_of_8tbs": render_bytes / (kernel_render_ms * 1e-3) / 1e9 / NOMINAL_HBM_GBS,
+            "bar_ms": render_bytes / (0.7 * NOMINAL_HBM_GBS * 1e9) * 1e3,
         }
         hash_roof = {
             "kernel": "leaf_hash_kernel", "bound": "alu", "achieved": hash_tops, "peak": alu_peak,
-            "peak_source": "derived: 152 SMs x 64 integer-ALU lanes x max SM clock",
+            "peak_source": f"derived: {num_sms} SMs (device property) x 64 integer-ALU lanes x "
+                           f"max SM clock {sm_max_mhz():.0f} MHz",
             "unit": "Tops/s", "frac": hash_tops / alu_peak,
             "traffic": profile_traffic("blake2s_tree.cu", "leaf_hash_kernel_q4b.md"),
             "algorithmic_ops_per_launch": HASH_ALU_OPS_PER_BYTE * frag_bytes,
@@ -923,9 +1073,11 @@ def main():
             "fragments_per_launch": ktimes["leaf_hash_fragments"] / max(1, ktimes["leaf_hash_launches"]),
             "hash_gbs": frag_bytes / (leaf_ms * 1e-3) / 1e9,
             "hash_frac_of_measured_hbm": frag_bytes / (leaf_ms * 1e-3) / 1e9 / peak,
-            # against every integer lane of an SM (ALU and FMA pipes, 128 per clock); only
-            # the ALU pipe's 64 can take the xors and rotates, which is what binds
-            "frac_of_128_int_lanes": hash_tops / (alu_peak * 128 / ALU_OPS_PER_CLK_PER_SM),
+            # every integer operation of BLAKE2s (adds included) against every integer lane
+            # of an SM (ALU and FMA pipes, 128 per clock): the looser of the two readings
+            "all_int_ops_per_block": HASH_INT_OPS_PER_BLOCK,
+            "all_int_tops": hash_int_tops, "all_int_peak": int_peak,
+            "frac_all_int_ops_of_128_lanes": hash_int_tops / int_peak,
             # measured on this GPU before the timed steps (cm_measure_int_alu): three-input
             # xors alone, and the same compression function on register data alone
             "measured_xor3_tops": xor3_tops, "measured_compress_tops": compress_tops,
@@ -952,8 +1104,11 @@ def main():
             "render_gbs": render_gbs,
             "render_frac_of_measured_hbm": render_gbs / peak,
             "render_frac_of_8tbs": render_gbs / NOMINAL_HBM_GBS,
+            "render_frac_of_same_box_copy": render_gbs / copy_gbs,
             "render_ms": render_ms,
+            "box_copy": copy,
             "paged_render_gbs": (render_bytes / (paged_ms * 1e-3) / 1e9) if paged_ms else None,
+            "paged_render_ms_back_to_back": paged_ms,
             "ingest_ms_per_merge": ingest_ms,
             "ingest_gbs": hash_bytes / (ingest_ms * 1e-3) / 1e9,
             "roofline": hash_roof if dominant != "render" else render_roof,
@@ -961,6 +1116,11 @@ def main():
             "hash_roofline": hash_roof,
             "kernel_ms_per_step": per_step,
             "dominant_kernel": dominant,
+            "sustained": {"steps": sustained_steps, "value": whole_job_rate(world, sustained_steps, sustained_ms),
+                          "ms_per_step": sustained_ms / sustained_steps, "seconds": sustained_ms / 1e3,
+                          "clocks": sclocks.summary(),
+                          "timing": "the same step loop run again for at least 0.5 s after the "
+                                    "timed steps, CUDA events around all of it"},
             "e2e": {"value": whole_job_rate(world, e2e_steps, e2e_ms), "unit": UNIT,
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e2e_steps,
                     "runs": [whole_job_rate(world, e2e_steps, m) for m in e2e_runs],
@@ -972,9 +1132,9 @@ def main():
             "gpu_launches": int(round(launches_per_step * args.steps)),
             "clocks": clocks.summary(),
         }
+        line.update(extra)
         if world == 1 and not args.no_cpu_baseline and args.workload == WORKLOAD:
-            line["cpu_baseline"] = cpu_baseline_entry()
-            line["cpu_baseline"]["all_cores"] = cpu_baseline_multicore()
+            line["cpu_baseline"] = cpu_baseline_entry(w)
         print(json.dumps(line), flush=True)
     ctx.close()
     if world > 1:
