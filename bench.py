@@ -731,9 +731,24 @@ def box_copy(dev, nbytes):
                    "bytes, 20 copies timed by CUDA events after 3 warm-up copies"}
 
 
-def merge_fn(cm, ctx, fdesc, k_out, v_out, total_T, stream):
+def merge_fn(cm, ctx, fdesc, k_out, v_out, total_T, stream, sequential=False):
     """One whole merge: replica A ingests the first half of the deliveries, replica B the
-    rest (one cm_ingest_many call: one GPU pass, one synchronisation), A := A u B, render A."""
+    rest, A := A u B, render A, as one cm_ingest_render call (the render overlaps the
+    content address when the norm keys decide the order), or with sequential=True as
+    separate calls (cm_ingest_many: one GPU pass and one synchronisation; cm_union;
+    cm_render)."""
+    def fused(timers=None, inputs=None, out=None):
+        k_dst, v_dst = out or (k_out, v_out)
+        a = cm.cm_set_create(ctx.handle)
+        b = cm.cm_set_create(ctx.handle)
+        fd = inputs or fdesc
+        half = (len(fd) + 1) // 2
+        _, n, _, _ = cm.cm_ingest_render([a] * half + [b] * (len(fd) - half), fd, a,
+                                         k_dst.data_ptr(), v_dst.data_ptr(), total_T, stream)
+        cm.cm_set_destroy(b)
+        cm.cm_set_destroy(a)
+        return n
+
     def one_merge(timers=None, inputs=None, out=None):
         k_dst, v_dst = out or (k_out, v_out)
         a = cm.cm_set_create(ctx.handle)
@@ -755,12 +770,13 @@ def merge_fn(cm, ctx, fdesc, k_out, v_out, total_T, stream):
         cm.cm_set_destroy(b)
         cm.cm_set_destroy(a)
         return n
-    return one_merge
+    return one_merge if sequential else fused
 
 
 def small_merge_entry(cm, dev, name, merges=200):
-    """A whole-merge measurement of a small workload (same step as the headline one), with
-    the render's in-step and back-to-back device times."""
+    """A whole-merge measurement of a small workload (the headline step, cm_ingest_render),
+    beside the same merges as separate calls, with the render's in-step (separate calls)
+    and back-to-back device times."""
     import torch
     import synthetic
     w = synthetic.WORKLOADS[name]
@@ -772,35 +788,41 @@ def small_merge_entry(cm, dev, name, merges=200):
     ctx = cm.Context(dev.index or 0, synthetic.ROPE_THETA)
     stream = torch.cuda.current_stream(dev)
     fdesc = [cm.fragment_from_tensors(K, V) for K, V in frags]
-    one = merge_fn(cm, ctx, fdesc, k_out, v_out, T, stream)
-    for _ in range(10):
-        one()
-    torch.cuda.synchronize(dev)
-    cm.cm_context_kernel_times(ctx.handle, reset=True)
-    cm.cm_context_set_timing(ctx.handle, True)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(merges):
-        one()
-    e1.record(stream)
-    torch.cuda.synchronize(dev)
-    cm.cm_context_set_timing(ctx.handle, False)
-    kt = cm.cm_context_kernel_times(ctx.handle, reset=True)
-    ms = e0.elapsed_time(e1) / merges
+
+    def timed(one):
+        for _ in range(10):
+            one()
+        torch.cuda.synchronize(dev)
+        cm.cm_context_kernel_times(ctx.handle, reset=True)
+        cm.cm_context_set_timing(ctx.handle, True)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(merges):
+            one()
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        cm.cm_context_set_timing(ctx.handle, False)
+        kt = cm.cm_context_kernel_times(ctx.handle, reset=True)
+        return e0.elapsed_time(e1) / merges, kt
+
+    ms, kt = timed(merge_fn(cm, ctx, fdesc, k_out, v_out, T, stream))
+    ms_seq, kt_seq = timed(merge_fn(cm, ctx, fdesc, k_out, v_out, T, stream, sequential=True))
     S = cm.FragmentSet(ctx)
     S.ingest_batch(frags)
     b2b, _ = grouped_ms(lambda: S.render(k_out, v_out, stream), stream, groups=10, per=20)
     S.close()
     ctx.close()
     moved = 2 * T * w.bytes_per_token
+    per = lambda k: {"leaf_hash": k["leaf_hash_ms"] / merges, "inner_hash": k["inner_hash_ms"] / merges,
+                     "render": k["render_ms"] / merges}
+    launches = lambda k: (k["leaf_hash_launches"] + k["inner_hash_launches"] + k["render_launches"] +
+                          k["aux_launches"]) / merges
     return {"workload": WORKLOAD_TEXT[name], "value": 1000.0 / ms, "unit": UNIT,
-            "ms_per_merge": ms, "merges": merges,
-            "kernel_ms_per_merge": {"leaf_hash": kt["leaf_hash_ms"] / merges,
-                                    "inner_hash": kt["inner_hash_ms"] / merges,
-                                    "render": kt["render_ms"] / merges},
-            "launches_per_merge": (kt["leaf_hash_launches"] + kt["inner_hash_launches"] +
-                                   kt["render_launches"] + kt["aux_launches"]) / merges,
-            "render_us_in_step": 1000.0 * kt["render_ms"] / merges,
+            "ms_per_merge": ms, "merges": merges, "kernel_ms_per_merge": per(kt),
+            "launches_per_merge": launches(kt),
+            "sequential": {"value": 1000.0 / ms_seq, "ms_per_merge": ms_seq,
+                           "kernel_ms_per_merge": per(kt_seq), "launches_per_merge": launches(kt_seq)},
+            "render_us_in_step": 1000.0 * kt_seq["render_ms"] / merges,
             "render_us_back_to_back": 1000.0 * b2b,
             "render_gbs_back_to_back": moved / (b2b * 1e-3) / 1e9,
             "render_bytes": moved,
@@ -855,7 +877,6 @@ def main():
     xor3_tops, compress_tops = cm.cm_measure_int_alu(local_rank)
 
     # the timed steps: exactly args.steps merges
-    step_timers = [{"ingest": (ev(), ev()), "render": (ev(), ev())} for _ in range(args.steps)]
     start, end = ev(), ev()
     if world > 1:
         dist.barrier()
@@ -865,17 +886,36 @@ def main():
     with ClockSampler(local_rank) as clocks:
         start.record(stream)
         for i in range(args.steps):
-            one_merge(step_timers[i])
+            one_merge()
         end.record(stream)
         torch.cuda.synchronize(dev)
     cm.cm_context_set_timing(ctx.handle, False)
     ktimes = cm.cm_context_kernel_times(ctx.handle, reset=True)
     if world > 1:
         dist.barrier()
-    elapsed_ms = start.elapsed_time(end)
+    elapsed_ms = max_over_ranks(start.elapsed_time(end), dev)
+
+    # the same steps as separate calls (cm_ingest_many, cm_union, cm_render: hashing, then
+    # the full-SM render), each kernel alone: the kernels' own rooflines come from here
+    seq_merge = merge_fn(cm, ctx, fdesc, k_out, v_out, total_T, stream, sequential=True)
+    for _ in range(2):
+        seq_merge()
+    step_timers = [{"ingest": (ev(), ev()), "render": (ev(), ev())} for _ in range(args.steps)]
+    q0, q1 = ev(), ev()
+    torch.cuda.synchronize(dev)
+    cm.cm_context_kernel_times(ctx.handle, reset=True)
+    cm.cm_context_set_timing(ctx.handle, True)
+    with ClockSampler(local_rank) as qclocks:
+        q0.record(stream)
+        for i in range(args.steps):
+            seq_merge(step_timers[i])
+        q1.record(stream)
+        torch.cuda.synchronize(dev)
+    cm.cm_context_set_timing(ctx.handle, False)
+    ktimes_seq = cm.cm_context_kernel_times(ctx.handle, reset=True)
+    seq_ms = max_over_ranks(q0.elapsed_time(q1), dev)
     render_ms = sum(t["render"][0].elapsed_time(t["render"][1]) for t in step_timers) / args.steps
     ingest_ms = sum(t["ingest"][0].elapsed_time(t["ingest"][1]) for t in step_timers) / args.steps
-    elapsed_ms = max_over_ranks(elapsed_ms, dev)
 
     # the same step loop again for at least 0.5 s (reported apart: a short timed region
     # cannot separate the box from the kernels)
@@ -1029,18 +1069,24 @@ def main():
         ms_per_step = elapsed_ms / args.steps
         launches_per_step = (ktimes["leaf_hash_launches"] + ktimes["inner_hash_launches"] +
                              ktimes["render_launches"] + ktimes["aux_launches"]) / args.steps
-        # one leaf-hash launch covers every fragment of an ingest call (up to 32): the
-        # work of a launch is the bytes of the step's fragments divided by its launches
-        leaf_launches_per_step = max(1, ktimes["leaf_hash_launches"]) / args.steps
-        leaf_ms = ktimes["leaf_hash_ms"] / max(1, ktimes["leaf_hash_launches"])
-        frag_bytes = hash_bytes / leaf_launches_per_step
+
+        def leaf_figures(kt):
+            # one leaf-hash launch covers every fragment of an ingest call (up to 32): the
+            # work of a launch is the bytes of the step's fragments divided by its launches
+            launches = max(1, kt["leaf_hash_launches"]) / args.steps
+            ms = kt["leaf_hash_ms"] / max(1, kt["leaf_hash_launches"])
+            return ms, hash_bytes / launches
+
+        leaf_ms, frag_bytes = leaf_figures(ktimes_seq)
+        leaf_ms_ovl, _ = leaf_figures(ktimes)
         blocks = frag_bytes / 64.0
         hash_tops = HASH_ALU_OPS_PER_BYTE * frag_bytes / (leaf_ms * 1e-3) / 1e12
         hash_int_tops = HASH_INT_OPS_PER_BLOCK * blocks / (leaf_ms * 1e-3) / 1e12
         clk = sm_max_mhz() * 1e6
         alu_peak = num_sms * ALU_OPS_PER_CLK_PER_SM * clk / 1e12
         int_peak = num_sms * 128 * clk / 1e12
-        kernel_render_ms = ktimes["render_ms"] / max(1, ktimes["render_launches"])
+        kernel_render_ms = ktimes_seq["render_ms"] / max(1, ktimes_seq["render_launches"])
+        render_ms_ovl = ktimes["render_ms"] / max(1, ktimes["render_launches"])
         copy_gbs = copy["median_gbs"]
         render_roof = {
             "kernel": "render_reg_kernel", "bound": "hbm",
@@ -1050,9 +1096,9 @@ def main():
             "frac": render_bytes / (kernel_render_ms * 1e-3) / 1e9 / peak,
             "traffic": profile_traffic("render.cu", "render_kernel_q4b.md"),
             "algorithmic_bytes_per_launch": render_bytes, "ms_per_launch": kernel_render_ms,
-            "timing": "CUDA events on the render's stream around each launch in the timed steps "
-                      "(the stream is idle when the start event is recorded, so each interval "
-                      "includes the launch's own latency)",
+            "timing": "CUDA events on the render's stream around each launch in the sequential "
+                      "steps (the full-SM render alone; the stream is idle when the start event is "
+                      "recorded, so each interval includes the launch's own latency)",
             "back_to_back_ms": render_b2b_ms,
             "back_to_back_gbs": render_bytes / (render_b2b_ms * 1e-3) / 1e9,
             "back_to_back_frac": render_bytes / (render_b2b_ms * 1e-3) / 1e9 / peak,
@@ -1086,7 +1132,33 @@ def main():
         per_step = {"leaf_hash": ktimes["leaf_hash_ms"] / args.steps,
                     "inner_hash": ktimes["inner_hash_ms"] / args.steps,
                     "render": ktimes["render_ms"] / args.steps}
+        per_step_seq = {"leaf_hash": ktimes_seq["leaf_hash_ms"] / args.steps,
+                        "inner_hash": ktimes_seq["inner_hash_ms"] / args.steps,
+                        "render": ktimes_seq["render_ms"] / args.steps}
         dominant = max(per_step, key=per_step.get)
+        # the dominant kernel of the timed steps as it ran there: the leaf hash, with the
+        # half-SM render of the same merge beside it on the other stream
+        hash_in_step = dict(hash_roof)
+        hash_in_step.update({
+            "achieved": HASH_ALU_OPS_PER_BYTE * frag_bytes / (leaf_ms_ovl * 1e-3) / 1e12,
+            "frac": HASH_ALU_OPS_PER_BYTE * frag_bytes / (leaf_ms_ovl * 1e-3) / 1e12 / alu_peak,
+            "ms_per_launch": leaf_ms_ovl,
+            "hash_gbs": frag_bytes / (leaf_ms_ovl * 1e-3) / 1e9,
+            "frac_all_int_ops_of_128_lanes":
+                HASH_INT_OPS_PER_BLOCK * blocks / (leaf_ms_ovl * 1e-3) / 1e12 / int_peak,
+            "frac_of_measured_compress":
+                HASH_ALU_OPS_PER_BYTE * frag_bytes / (leaf_ms_ovl * 1e-3) / 1e12 / compress_tops,
+            "timing": "CUDA events around each leaf-hash launch in the timed steps, where the "
+                      "render of the same merge runs beside it on another stream (cm_ingest_render); "
+                      "hash_roofline has the same kernel alone",
+        })
+        render_in_step = {
+            "kernel": "render_kernel (4-warp TMA CTAs) beside the leaf hash", "ms_per_launch": render_ms_ovl,
+            "gbs": render_bytes / (render_ms_ovl * 1e-3) / 1e9,
+            "timing": "CUDA events around each render launch on cm_ingest_render's side stream, "
+                      "in the timed steps (overlapping the leaf hash)"}
+        hash_roof["timing"] = ("CUDA events around each leaf-hash launch in the sequential steps "
+                               "(the kernel alone)")
         line = {
             "metric": METRIC,
             "value": whole_job_rate(world, args.steps, elapsed_ms),
@@ -1111,11 +1183,19 @@ def main():
             "paged_render_ms_back_to_back": paged_ms,
             "ingest_ms_per_merge": ingest_ms,
             "ingest_gbs": hash_bytes / (ingest_ms * 1e-3) / 1e9,
-            "roofline": hash_roof if dominant != "render" else render_roof,
+            "roofline": hash_in_step if dominant != "render" else render_roof,
             "render_roofline": render_roof,
             "hash_roofline": hash_roof,
+            "render_in_step": render_in_step,
             "kernel_ms_per_step": per_step,
+            "kernel_ms_per_step_note": "kernels of one step overlap (the render runs beside the "
+                                       "leaf hash), so their sum exceeds ms_per_step",
             "dominant_kernel": dominant,
+            "sequential": {"value": whole_job_rate(world, args.steps, seq_ms),
+                           "ms_per_step": seq_ms / args.steps, "steps": args.steps,
+                           "kernel_ms_per_step": per_step_seq, "clocks": qclocks.summary(),
+                           "timing": "the same merges as separate calls (cm_ingest_many, "
+                                     "cm_union, cm_render), run after the timed steps"},
             "sustained": {"steps": sustained_steps, "value": whole_job_rate(world, sustained_steps, sustained_ms),
                           "ms_per_step": sustained_ms / sustained_steps, "seconds": sustained_ms / 1e3,
                           "clocks": sclocks.summary(),

@@ -44,7 +44,7 @@
 extern "C" {
 #endif
 
-#define CM_ABI_VERSION 4
+#define CM_ABI_VERSION 5
 
 /* Same type as cudaStream_t (a CUDA runtime stream handle); NULL is the legacy default stream. */
 typedef struct CUstream_st *cm_stream_t;
@@ -232,6 +232,43 @@ cm_status cm_set_leq(const cm_set *a, const cm_set *b, int32_t *out);
 cm_status cm_render(const cm_set *set, void *k_out, void *v_out, int64_t capacity_tokens,
                     cm_stream_t stream, int64_t *out_seq_len, cm_id *out_order);
 
+/* Ingest, Merge and Render of Algorithm 2 in one call, with the render overlapping the
+ * content address where the paper's definitions allow it. The result (sets, ids,
+ * absorption flags, rendered bytes, order) is that of
+ *     cm_ingest_many(sets, frags, n, stream, out_ids, out_absorbed);
+ *     cm_union(target, s) for every set s of `sets` other than target, in order of first
+ *         appearance (the replicas' states merged into target, Eq. setunion);
+ *     cm_render(target, k_out, v_out, capacity_tokens, stream, out_seq_len, out_order);
+ * Overlap: the routing-layer norm keys (Eq. rho) of the deliveries are computed first
+ * (one pass over K[l*], 1/(2L) of the bytes, and a synchronisation). Byte-identical
+ * fragments have equal norm keys, so if the integer tail sums S of all fragments the
+ * target will hold (its own, the other sets', every delivery) are pairwise distinct,
+ * no delivery can be absorbed and the canonical order of Algorithm 1 does not depend on
+ * the ids: the render starts at once on a stream of the context, with half-SM CTAs,
+ * while the content address runs on `stream`. When the ids are known the set is
+ * checked to be the one rendered (it always is unless two different fragments share
+ * an address, which the paper's collision assumption excludes; then the target is
+ * rendered again after the first render, so the result is still exact). With any tie
+ * of S, with the re-delivery fast path on, or with an output the render would refuse,
+ * the steps run one after the other.
+ *   sets, frags      HOST arrays of n (n >= 0): delivery i goes into sets[i]; all sets
+ *                    and target from one context (CM_ERR_INVALID_ARG)
+ *   target           the set rendered (it may appear in sets or not)
+ *   k_out, v_out, capacity_tokens   as in cm_render
+ *   out_ids, out_absorbed           nullable HOST arrays of n, as in cm_ingest_many
+ *   out_seq_len, out_order          nullable, as in cm_render (out_order: the target's size)
+ *   out_overlapped   nullable: 1 if the render ran beside the content address, else 0
+ * The target, every other set named and every delivery must share one (L, H, d)
+ * (empty sets excepted): CM_ERR_SHAPE_MISMATCH before any work otherwise. The call
+ * returns after the ids reached the host; the render is then still running, ordered
+ * before any later work on `stream`. On an error after the GPU work began (a collision
+ * under verify_bytes_on_hit, capacity, CUDA) the sets are as the sequence above leaves
+ * them at its failing step and the contents of k_out and v_out are unspecified. */
+cm_status cm_ingest_render(cm_set *const *sets, const cm_fragment *frags, int32_t n,
+                           cm_set *target, void *k_out, void *v_out, int64_t capacity_tokens,
+                           cm_stream_t stream, cm_id *out_ids, int32_t *out_absorbed,
+                           int64_t *out_seq_len, cm_id *out_order, int32_t *out_overlapped);
+
 /* One render job of cm_render_many: a set and its contiguous output, with the
  * meaning of the arguments of the same names in cm_render. */
 typedef struct cm_render_job {
@@ -331,6 +368,13 @@ cm_status cm_context_check(cm_context *ctx, cm_stream_t stream);
  * synchronisation per call that has candidates (two if a prefix matches): turn it on
  * where re-deliveries are common (gossip, retries). The paper has no counterpart. */
 cm_status cm_context_set_dedup_by_bytes(cm_context *ctx, int32_t enable);
+
+/* Whether cm_ingest_render may run its render beside the content address (a scheduling
+ * choice; the results are identical either way; the paper has no counterpart):
+ *   0  never: the call runs cm_ingest_many, the unions and cm_render one after the other
+ *   1  (the default) whenever the norm keys decide the canonical order on their own
+ * CM_ERR_INVALID_ARG for any other value. */
+cm_status cm_context_set_overlap(cm_context *ctx, int32_t mode);
 
 /* Width of the render kernel's CTAs for every later render launched from ctx (a
  * scheduling aid; the paper has no counterpart). The render is one persistent CTA per

@@ -16,8 +16,8 @@ from ._binding import (  # noqa: F401
     cm_context_create, cm_context_destroy, cm_context_check, cm_testing_bounds_violations,
     cm_set_create, cm_set_destroy,
     cm_fragment_id, cm_fragment_id_static, cm_ingest, cm_ingest_batch, cm_ingest_many,
-    cm_render_many, cm_render_job, cm_set_contains, cm_set_leq, ingest_many, render_many,
-    cm_measure_int_alu, cm_context_set_render_warps, cm_context_set_dedup_by_bytes,
+    cm_render_many, cm_ingest_render, cm_render_job, cm_set_contains, cm_set_leq, ingest_many, render_many,
+    cm_measure_int_alu, cm_context_set_render_warps, cm_context_set_overlap, cm_context_set_dedup_by_bytes,
     cm_context_set_timing, cm_context_kernel_times, cm_kernel_times, cm_union, cm_set_size, cm_set_seq_len, cm_set_ids,
     cm_render, cm_render_incremental, cm_render_paged, cm_paged_cache, cm_bagmerge,
     fragment_from_tensors, Context, FragmentSet,

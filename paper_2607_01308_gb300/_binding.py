@@ -102,10 +102,14 @@ _SIGS = {
                                   _c.POINTER(cm_id), _c.POINTER(_c.c_int32)]),
     "cm_render_many": (_c.c_int, [_c.POINTER(cm_render_job), _c.c_int32, _P,
                                   _c.POINTER(_c.c_int64)]),
+    "cm_ingest_render": (_c.c_int, [_c.POINTER(_P), _c.POINTER(cm_fragment), _c.c_int32, _P, _P, _P,
+                                    _c.c_int64, _P, _c.POINTER(cm_id), _c.POINTER(_c.c_int32),
+                                    _c.POINTER(_c.c_int64), _c.POINTER(cm_id), _c.POINTER(_c.c_int32)]),
     "cm_set_contains": (_c.c_int, [_P, _c.POINTER(cm_id), _c.c_int64, _c.POINTER(_c.c_uint8)]),
     "cm_set_leq": (_c.c_int, [_P, _P, _c.POINTER(_c.c_int32)]),
     "cm_measure_int_alu": (_c.c_int, [_c.c_int32, _c.POINTER(_c.c_double), _c.POINTER(_c.c_double)]),
     "cm_context_set_render_warps": (_c.c_int, [_P, _c.c_int32]),
+    "cm_context_set_overlap": (_c.c_int, [_P, _c.c_int32]),
     "cm_context_set_dedup_by_bytes": (_c.c_int, [_P, _c.c_int32]),
     "cm_context_set_timing": (_c.c_int, [_P, _c.c_int32]),
     "cm_context_kernel_times": (_c.c_int, [_P, _c.POINTER(cm_kernel_times), _c.c_int32]),
@@ -247,6 +251,34 @@ def cm_ingest_many(sets: Sequence[int], frags: Sequence[cm_fragment],
     return [(ids[i].to_bytes(), bool(absorbed[i])) for i in range(n)]
 
 
+def cm_ingest_render(sets: Sequence[int], frags: Sequence[cm_fragment], target: int, k_out: int,
+                     v_out: int, capacity_tokens: int, stream=None):
+    """cm_ingest_render: returns ([(id, absorbed)] per delivery, rendered length, canonical
+    order as a list of ids, overlapped flag)."""
+    n = len(frags)
+    if len(sets) != n:
+        raise ValueError("one set per delivery")
+    set_arr = (_P * max(n, 1))(*sets)
+    arr = (cm_fragment * max(n, 1))(*frags)
+    ids = (cm_id * max(n, 1))()
+    absorbed = (ctypes.c_int32 * max(n, 1))()
+    seq = ctypes.c_int64()
+    cap_order = n + 64
+    order = (cm_id * cap_order)()
+    ovl = ctypes.c_int32()
+    # the order array must hold the target's final size: at most its current size plus
+    # every other set's and every delivery's
+    members = cm_set_size(target) + n + sum(cm_set_size(s) for s in set(sets) if s != target)
+    if members > cap_order:
+        order = (cm_id * members)()
+    _check(lib.cm_ingest_render(set_arr, arr, n, target, k_out, v_out, capacity_tokens,
+                                _stream_handle(stream), ids, absorbed, ctypes.byref(seq), order,
+                                ctypes.byref(ovl)))
+    size = cm_set_size(target)
+    return ([(ids[i].to_bytes(), bool(absorbed[i])) for i in range(n)], seq.value,
+            [order[i].to_bytes() for i in range(size)], bool(ovl.value))
+
+
 def cm_render_many(jobs: Sequence[cm_render_job], stream=None) -> List[int]:
     n = len(jobs)
     arr = (cm_render_job * max(n, 1))(*jobs)
@@ -280,6 +312,10 @@ def cm_measure_int_alu(device: int = 0) -> Tuple[float, float]:
 
 def cm_context_set_dedup_by_bytes(ctx: int, enable: bool) -> None:
     _check(lib.cm_context_set_dedup_by_bytes(ctx, int(enable)))
+
+
+def cm_context_set_overlap(ctx: int, mode: int) -> None:
+    _check(lib.cm_context_set_overlap(ctx, mode))
 
 
 def cm_context_set_render_warps(ctx: int, warps: int) -> None:

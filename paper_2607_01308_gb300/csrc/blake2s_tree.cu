@@ -243,7 +243,7 @@ __global__ void __launch_bounds__(kLeafThreads)
 leaf_hash_kernel(const __grid_constant__ LeafGroup grp) {
     // the blocks after the leaf blocks compute norm keys, one thread per row of K[l*]:
     // they fill SMs that the last wave of leaf blocks leaves idle
-    const uint32_t x = blockIdx.x;
+    const uint32_t x = blockIdx.x + grp.first_block;
     const uint32_t leaf_blocks = (uint32_t)grp.block_begin[grp.count];
     if (x >= leaf_blocks) {
         const uint32_t k = x - leaf_blocks;
@@ -489,7 +489,7 @@ __global__ void compare_kernel(const uint4 *__restrict__ a, const uint4 *__restr
 
 CM_DEFINE_BOUNDS_READER(take_hash_bounds_violations)
 
-cudaError_t launch_leaf_hash_group(const LeafGroup &in, cudaStream_t stream) {
+cudaError_t launch_leaf_hash_group(const LeafGroup &in, cudaStream_t stream, LeafPhases phases) {
     if (in.count > (uint32_t)kMaxLeafGroup) return cudaErrorInvalidValue;
     if (in.count == 0) return cudaSuccess;
     LeafGroup g = in;
@@ -502,9 +502,16 @@ cudaError_t launch_leaf_hash_group(const LeafGroup &in, cudaStream_t stream) {
     }
     g.norm_block_begin[g.count] = norm_blocks;
     const uint64_t leaf_blocks = g.block_begin[g.count];
-    const uint64_t blocks = leaf_blocks + norm_blocks;
+    if (leaf_blocks + norm_blocks > 0x7FFFFFFFull) return cudaErrorInvalidValue;
+    // the grid covers blocks [first_block, first_block + blocks) of the combined range:
+    // leaf blocks first, then norm-key blocks
+    uint64_t blocks = 0;
+    switch (phases) {
+        case LeafPhases::kBoth: g.first_block = 0; blocks = leaf_blocks + norm_blocks; break;
+        case LeafPhases::kLeaves: g.first_block = 0; blocks = leaf_blocks; break;
+        case LeafPhases::kNormKeys: g.first_block = (uint32_t)leaf_blocks; blocks = norm_blocks; break;
+    }
     if (blocks == 0) return cudaSuccess;
-    if (blocks > 0x7FFFFFFFull) return cudaErrorInvalidValue;
     leaf_hash_kernel<<<(unsigned)blocks, kLeafThreads, 0, stream>>>(g);
     return cudaGetLastError();
 }
@@ -515,7 +522,7 @@ cudaError_t launch_leaf_hash(const LeafLaunch &a, cudaStream_t stream) {
     g.count = 1;
     g.block_begin[1] = (a.num_leaves + kLeafThreads - 1) / kLeafThreads;   // as the host does
     g.frag[0] = a;
-    return launch_leaf_hash_group(g, stream);
+    return launch_leaf_hash_group(g, stream, LeafPhases::kBoth);
 }
 
 cudaError_t launch_inner_hash(const uint8_t *children, uint64_t num_children, uint8_t *out,

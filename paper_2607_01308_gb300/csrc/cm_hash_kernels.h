@@ -47,12 +47,15 @@ constexpr int kMaxLeafGroup = 32;
 constexpr int kLeafBlockThreads = 128;   // threads (= leaves or rows) per block of the leaf launch
 struct LeafGroup {
     uint32_t count;
-    uint32_t pad_;
+    uint32_t first_block;          // set by the launcher: block index of the grid's block 0
     uint64_t block_begin[kMaxLeafGroup + 1];
     uint64_t norm_block_begin[kMaxLeafGroup + 1];
     LeafLaunch frag[kMaxLeafGroup];
 };
-cudaError_t launch_leaf_hash_group(const LeafGroup &g, cudaStream_t stream);
+// kBoth: leaves and norm keys in one launch; kLeaves / kNormKeys: one of the two (the
+// norm keys alone read only K[l*], 1/(2L) of the bytes).
+enum class LeafPhases { kBoth, kLeaves, kNormKeys };
+cudaError_t launch_leaf_hash_group(const LeafGroup &g, cudaStream_t stream, LeafPhases phases);
 
 // Level 0 of one fragment (a group of one).
 cudaError_t launch_leaf_hash(const LeafLaunch &a, cudaStream_t stream);

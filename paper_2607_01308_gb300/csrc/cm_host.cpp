@@ -149,6 +149,11 @@ struct cm_context {
     // launch parameters of the render kernel (about 31 KB), reused by every launch
     std::unique_ptr<cm::RenderParams> render_params;
     int32_t render_warps = 16;   // warps per render CTA (cm_context_set_render_warps)
+    // cm_ingest_render: the stream its overlapped render runs on and the two events that
+    // order it after the caller's stream and the caller's stream after it (made on first use)
+    cudaStream_t side = nullptr;
+    cudaEvent_t side_begin = nullptr, side_end = nullptr, side_keys = nullptr;
+    int32_t overlap = 1;         // cm_context_set_overlap: 1 render beside the hash when possible
     bool dedup_bytes = false;    // re-delivery fast path (cm_context_set_dedup_by_bytes)
 };
 
@@ -210,16 +215,23 @@ cm_status ensure_scratch(cm_context *ctx, size_t dev_bytes, size_t host_bytes) {
     return CM_OK;
 }
 
-// Reads a small device result (`bytes` at `src`) into ctx->h_pinned, enqueued on
-// `stream`: stored by the SMs through the buffer's mapped address when both are 4-byte
-// granular (so the read does not wait behind bulk device-to-host copies of other
+// Reads a small device result (`bytes` at `src`) into ctx->h_pinned + host_off, enqueued
+// on `stream`: stored by the SMs through the buffer's mapped address when everything is
+// 4-byte granular (so the read does not wait behind bulk device-to-host copies of other
 // streams on the copy engine), else by a copy.
-cudaError_t read_small(cm_context *ctx, const void *src, size_t bytes, cudaStream_t stream) {
-    if (ctx->h_pinned_dev && bytes % 4 == 0 && (reinterpret_cast<uintptr_t>(src) & 3u) == 0) {
+cudaError_t read_small_at(cm_context *ctx, size_t host_off, const void *src, size_t bytes,
+                          cudaStream_t stream) {
+    if (ctx->h_pinned_dev && bytes % 4 == 0 && host_off % 4 == 0 &&
+        (reinterpret_cast<uintptr_t>(src) & 3u) == 0) {
         if (ctx->timing) ++ctx->aux_launches;
-        return cm::launch_readback(ctx->h_pinned_dev, src, bytes, stream);
+        return cm::launch_readback(static_cast<uint8_t *>(ctx->h_pinned_dev) + host_off, src, bytes,
+                                   stream);
     }
-    return cudaMemcpyAsync(ctx->h_pinned, src, bytes, cudaMemcpyDeviceToHost, stream);
+    return cudaMemcpyAsync(ctx->h_pinned + host_off, src, bytes, cudaMemcpyDeviceToHost, stream);
+}
+
+cudaError_t read_small(cm_context *ctx, const void *src, size_t bytes, cudaStream_t stream) {
+    return read_small_at(ctx, 0, src, bytes, stream);
 }
 
 // BLAKE2s parameter block (32 bytes) of the tree, node offset and depth zero,
@@ -287,27 +299,30 @@ cudaError_t timed_launch(cm_context *ctx, int kind, cudaStream_t stream, F &&lau
     return e;
 }
 
-// Id(C) and Q[t] of n fragments in one pass: the leaf-hash launches of all
-// fragments (with their norm keys), then the tree levels above the leaves (level 1,
-// then the levels above it: two launches per kMaxGroup fragments), then a single copy
-// of every root digest and norm key to the host and one synchronisation. Caller holds ctx->mu and the device scope.
-//   device scratch: [roots n x 16][Q of fragment 0]...[Q of fragment n-1][levels...]
-cm_status fragments_digest(cm_context *ctx, const cm_fragment *const *frags, size_t n,
-                           cudaStream_t stream, cm_id *ids, std::vector<uint64_t> *Qs) {
-    struct Layout {
-        std::vector<uint64_t> sizes;
-        std::vector<size_t> level_off;
-        size_t q_off;
-        uint64_t plane, stream_bytes;
-        int32_t rl;
+// The scratch of one content-address pass over n fragments (Section 4.3; Algorithm 2,
+// Id): device [roots n x 16][Q of fragment 0]...[Q of fragment n-1][arrival counters of
+// the nodes at levels >= 2][the levels below each root]; the pinned host buffer receives
+// [roots][Q ...] at the same offsets.
+struct DigestPlan {
+    struct Frag {
+        std::vector<uint64_t> sizes;     // nodes per level, leaves first; the last is the root
+        std::vector<size_t> level_off;   // device offsets of the levels below the root
+        size_t q_off = 0, arr_off = 0;
+        uint64_t plane = 0, stream_bytes = 0;
+        int32_t rl = 0;
         cm::TreeParams tp;
     };
-    std::vector<Layout> lay(n);
-    const size_t roots_bytes = n * 16;
-    size_t off = roots_bytes;
+    std::vector<Frag> f;
+    size_t roots_bytes = 0, host_bytes = 0, zero_end = 0, dev_bytes = 0;
+};
+
+cm_status plan_digest(cm_context *ctx, const cm_fragment *const *frags, size_t n, DigestPlan &plan) {
+    plan.f.assign(n, DigestPlan::Frag());
+    plan.roots_bytes = n * 16;
+    size_t off = plan.roots_bytes;
     for (size_t i = 0; i < n; ++i) {
         const cm_fragment *f = frags[i];
-        Layout &l = lay[i];
+        DigestPlan::Frag &l = plan.f[i];
         l.rl = routing_layer_for(ctx, f->num_layers);
         if (l.rl >= f->num_layers) return fail(CM_ERR_INVALID_ARG, "routing layer >= num_layers");
         l.plane = (uint64_t)f->num_kv_heads * f->seq_len * f->head_dim * 2;
@@ -315,36 +330,43 @@ cm_status fragments_digest(cm_context *ctx, const cm_fragment *const *frags, siz
         l.sizes.assign(1, ceil_div(l.stream_bytes, cm::kLeafBytes));
         while (l.sizes.size() == 1 || l.sizes.back() > 1)
             l.sizes.push_back(ceil_div(l.sizes.back(), cm::kFanout));
+        if (l.sizes.size() > (size_t)cm::kMaxLevels)
+            return fail(CM_ERR_UNSUPPORTED, "fragment too large for the hash tree depth");
         l.q_off = off;
         off += (size_t)f->seq_len * 8;
         l.tp = tree_params(f->num_layers, f->num_kv_heads, f->head_dim, f->seq_len);
     }
-    const size_t host_bytes = off;     // roots and norm keys, copied back in one piece
-    // arrival counters of every node at levels >= 2 follow the norm keys, so that one
-    // memset zeroes both before the launches
-    std::vector<size_t> arr_off(n);
+    plan.host_bytes = off;   // roots and norm keys
+    // the arrival counters follow the norm keys, so that one memset zeroes both
     for (size_t i = 0; i < n; ++i) {
-        arr_off[i] = off;
-        for (size_t k = 2; k < lay[i].sizes.size(); ++k) off += (size_t)lay[i].sizes[k] * 4;
+        plan.f[i].arr_off = off;
+        for (size_t k = 2; k < plan.f[i].sizes.size(); ++k) off += (size_t)plan.f[i].sizes[k] * 4;
     }
-    const size_t zero_end = off;
+    plan.zero_end = off;
     off = (off + 255) & ~(size_t)255;
     for (size_t i = 0; i < n; ++i) {
-        Layout &l = lay[i];
-        if (l.sizes.size() > (size_t)cm::kMaxLevels)
-            return fail(CM_ERR_UNSUPPORTED, "fragment too large for the hash tree depth");
+        DigestPlan::Frag &l = plan.f[i];
         for (size_t k = 0; k + 1 < l.sizes.size(); ++k) {   // the root goes to the roots area
             l.level_off.push_back(off);
             off += ((size_t)l.sizes[k] * cm::kDigestBytes + 255) & ~(size_t)255;
         }
     }
-    cm_status st = ensure_scratch(ctx, off, host_bytes);
-    if (st != CM_OK) return st;
-    uint8_t *base = ctx->d_scratch;
+    plan.dev_bytes = off;
+    return CM_OK;
+}
 
-    CM_CUDA_TRY(cudaMemsetAsync(base + roots_bytes, 0, zero_end - roots_bytes, stream),
+// Enqueues a planned pass on `stream` (the scratch already holds plan.dev_bytes and
+// plan.host_bytes): the leaf launches of up to kMaxLeafGroup fragments each (with the
+// norm keys when with_norms), the tree levels above the leaves (level 1, then the levels
+// above it: two launches per kMaxGroup fragments), and the results' way to the pinned
+// buffer. When the buffer is mapped, the kernels that hash the roots store them there
+// directly and only the norm keys are read back; otherwise roots and keys are copied.
+cm_status enqueue_digest(cm_context *ctx, const DigestPlan &plan, const cm_fragment *const *frags,
+                         size_t n, cudaStream_t stream, bool with_norms) {
+    uint8_t *base = ctx->d_scratch;
+    uint8_t *roots = ctx->h_pinned_dev ? static_cast<uint8_t *>(ctx->h_pinned_dev) : base;
+    CM_CUDA_TRY(cudaMemsetAsync(base + plan.roots_bytes, 0, plan.zero_end - plan.roots_bytes, stream),
                 "zeroing the norm keys and arrival counters");
-    // level 0 of up to kMaxLeafGroup fragments per launch
     std::unique_ptr<cm::LeafGroup> grp(new cm::LeafGroup);
     for (size_t g0 = 0; g0 < n; g0 += (size_t)cm::kMaxLeafGroup) {
         const size_t gn = std::min(n - g0, (size_t)cm::kMaxLeafGroup);
@@ -352,7 +374,7 @@ cm_status fragments_digest(cm_context *ctx, const cm_fragment *const *frags, siz
         grp->count = (uint32_t)gn;
         for (size_t q = 0; q < gn; ++q) {
             const cm_fragment *f = frags[g0 + q];
-            const Layout &l = lay[g0 + q];
+            const DigestPlan::Frag &l = plan.f[g0 + q];
             cm::LeafLaunch &a = grp->frag[q];
             a.k = static_cast<const uint8_t *>(f->k);
             a.v = static_cast<const uint8_t *>(f->v);
@@ -369,8 +391,9 @@ cm_status fragments_digest(cm_context *ctx, const cm_fragment *const *frags, siz
         }
         if (grp->block_begin[gn] > 0x7FFFFFFFull)
             return fail(CM_ERR_UNSUPPORTED, "leaf-hash launch exceeds 2^31 - 1 blocks");
+        const cm::LeafPhases phases = with_norms ? cm::LeafPhases::kBoth : cm::LeafPhases::kLeaves;
         CM_CUDA_TRY(timed_launch(ctx, kTimeLeaf, stream,
-                                 [&] { return cm::launch_leaf_hash_group(*grp, stream); }),
+                                 [&] { return cm::launch_leaf_hash_group(*grp, stream, phases); }),
                     "leaf hash launch");
         if (ctx->timing) ctx->leaf_fragments += (int64_t)gn;
     }
@@ -385,14 +408,14 @@ cm_status fragments_digest(cm_context *ctx, const cm_fragment *const *frags, siz
         return e;
     };
     for (size_t i = 0; i < n; ++i) {
-        const Layout &l = lay[i];
+        const DigestPlan::Frag &l = plan.f[i];
         const uint32_t c = top->count;
         cm::TreeTopFragment &tf = top->frag[c];
         tf.levels = (uint32_t)l.sizes.size();
-        size_t a_off = arr_off[i];
+        size_t a_off = l.arr_off;
         for (size_t k = 0; k < l.sizes.size(); ++k) {
             tf.size[k] = l.sizes[k];
-            tf.level[k] = (k + 1 == l.sizes.size()) ? base + 16 * i : base + l.level_off[k];
+            tf.level[k] = (k + 1 == l.sizes.size()) ? roots + 16 * i : base + l.level_off[k];
             if (k >= 2) {
                 tf.arrivals[k] = reinterpret_cast<uint32_t *>(base + a_off);
                 a_off += (size_t)l.sizes[k] * 4;
@@ -404,16 +427,79 @@ cm_status fragments_digest(cm_context *ctx, const cm_fragment *const *frags, siz
         if (top->count == (uint32_t)cm::kMaxGroup) CM_CUDA_TRY(flush(), "tree-top launch");
     }
     CM_CUDA_TRY(flush(), "tree-top launch");
-    CM_CUDA_TRY(read_small(ctx, base, host_bytes, stream),
-                "digest copy");
-    CM_CUDA_TRY(cudaStreamSynchronize(stream), "ingest synchronisation");
+    if (!ctx->h_pinned_dev)
+        CM_CUDA_TRY(read_small_at(ctx, 0, base, with_norms ? plan.host_bytes : plan.roots_bytes, stream),
+                    "digest copy");
+    else if (with_norms)
+        CM_CUDA_TRY(read_small_at(ctx, plan.roots_bytes, base + plan.roots_bytes,
+                                  plan.host_bytes - plan.roots_bytes, stream),
+                    "norm-key copy");
+    return CM_OK;
+}
+
+// After the stream reached the end of an enqueued pass: ids (and norm keys, if Qs).
+void collect_digest(const cm_context *ctx, const DigestPlan &plan, const cm_fragment *const *frags,
+                    size_t n, cm_id *ids, std::vector<uint64_t> *Qs) {
     for (size_t i = 0; i < n; ++i) {
         std::memcpy(ids[i].b, ctx->h_pinned + 16 * i, 16);
         if (Qs) {
             Qs[i].resize((size_t)frags[i]->seq_len);
-            std::memcpy(Qs[i].data(), ctx->h_pinned + lay[i].q_off, (size_t)frags[i]->seq_len * 8);
+            std::memcpy(Qs[i].data(), ctx->h_pinned + plan.f[i].q_off, (size_t)frags[i]->seq_len * 8);
         }
     }
+}
+
+// Id(C) and Q[t] of n fragments in one pass and one synchronisation of `stream`.
+// Caller holds ctx->mu and the device scope.
+cm_status fragments_digest(cm_context *ctx, const cm_fragment *const *frags, size_t n,
+                           cudaStream_t stream, cm_id *ids, std::vector<uint64_t> *Qs) {
+    DigestPlan plan;
+    cm_status st = plan_digest(ctx, frags, n, plan);
+    if (st == CM_OK) st = ensure_scratch(ctx, plan.dev_bytes, plan.host_bytes);
+    if (st == CM_OK) st = enqueue_digest(ctx, plan, frags, n, stream, true);
+    if (st != CM_OK) return st;
+    CM_CUDA_TRY(cudaStreamSynchronize(stream), "ingest synchronisation");
+    collect_digest(ctx, plan, frags, n, ids, Qs);
+    return CM_OK;
+}
+
+// Enqueues Q[t] of n fragments alone (Eq. rho) on `stream`: one launch of the norm-key
+// row threads per kMaxLeafGroup fragments (they read only K[l*]) into device scratch at
+// dev_off (q_off[i] after it for fragment i; zeroed first), then a copy to the pinned
+// buffer at host_off (same relative offsets).
+cm_status enqueue_norm_keys(cm_context *ctx, const cm_fragment *const *frags, size_t n,
+                            cudaStream_t stream, size_t dev_off, size_t host_off,
+                            const std::vector<size_t> &q_off, size_t bytes) {
+    uint8_t *base = ctx->d_scratch + dev_off;
+    CM_CUDA_TRY(cudaMemsetAsync(base, 0, bytes, stream), "zeroing the norm keys");
+    std::unique_ptr<cm::LeafGroup> grp(new cm::LeafGroup);
+    for (size_t g0 = 0; g0 < n; g0 += (size_t)cm::kMaxLeafGroup) {
+        const size_t gn = std::min(n - g0, (size_t)cm::kMaxLeafGroup);
+        std::memset(grp.get(), 0, sizeof(cm::LeafGroup));
+        grp->count = (uint32_t)gn;
+        for (size_t q = 0; q < gn; ++q) {
+            const cm_fragment *f = frags[g0 + q];
+            cm::LeafLaunch &a = grp->frag[q];
+            a.k = static_cast<const uint8_t *>(f->k);
+            a.v = static_cast<const uint8_t *>(f->v);
+            a.plane_bytes = (uint64_t)f->num_kv_heads * f->seq_len * f->head_dim * 2;
+            a.stream_bytes = 2ull * f->num_layers * a.plane_bytes;
+            a.num_leaves = ceil_div(a.stream_bytes, cm::kLeafBytes);
+            a.norm_begin = 2ull * (uint64_t)routing_layer_for(ctx, f->num_layers) * a.plane_bytes;
+            a.row_bytes = (uint32_t)f->head_dim * 2;
+            a.seq_len = (uint32_t)f->seq_len;
+            a.norm_key = reinterpret_cast<unsigned long long *>(base + q_off[g0 + q]);
+            a.tree = tree_params(f->num_layers, f->num_kv_heads, f->head_dim, f->seq_len);
+            grp->block_begin[q + 1] =
+                grp->block_begin[q] + ceil_div(a.num_leaves, (uint64_t)cm::kLeafBlockThreads);
+        }
+        if (grp->block_begin[gn] > 0x7FFFFFFFull)
+            return fail(CM_ERR_UNSUPPORTED, "leaf-hash launch exceeds 2^31 - 1 blocks");
+        CM_CUDA_TRY(cm::launch_leaf_hash_group(*grp, stream, cm::LeafPhases::kNormKeys),
+                    "norm-key launch");
+        if (ctx->timing) ++ctx->aux_launches;
+    }
+    CM_CUDA_TRY(read_small_at(ctx, host_off, base, bytes, stream), "norm-key copy");
     return CM_OK;
 }
 
@@ -473,10 +559,13 @@ struct Slot {
 // belong to several sets of one shape: each slot carries its own output.
 cm_status launch_slots(cm_context *ctx, const std::vector<Slot> &slots, int32_t L, int32_t H,
                        int32_t d, cudaStream_t stream, uint32_t withhold_warp = 0,
-                       const cm_paged_cache *paged = nullptr) {
-    // the failure-injection hook withholds a TMA copy, so it runs the half-SM kernel (the
-    // only one that waits)
-    const int warps = withhold_warp ? 8 : ctx->render_warps;
+                       const cm_paged_cache *paged = nullptr, const cm::RenderWidth *width = nullptr) {
+    // no width: the context's. The failure-injection hook withholds a TMA copy, so it runs
+    // the half-SM kernel (the TMA kernels are the ones that wait).
+    const cm::RenderWidth warps =
+        withhold_warp ? cm::RenderWidth::kHalf
+                      : width ? *width
+                              : (ctx->render_warps == 8 ? cm::RenderWidth::kHalf : cm::RenderWidth::kFull);
     const int rows_per_chunk = (int)cm::render_item_bytes(warps) / (2 * d);
     const int half = d / 2;
     const int max_group = std::min<int>(cm::kMaxSlots, cm::kMaxTablePairs / half);
@@ -568,6 +657,22 @@ cm_status validate_outputs(void *k_out, void *v_out, int64_t capacity, int64_t t
     return CM_OK;
 }
 
+// S = sum of Q[t] over the last t_star of a fragment's T positions (the integer form of
+// rho, Eq. rho, up to the common factor 2^-20 / (H T*)).
+unsigned __int128 tail_sum(const std::vector<uint64_t> &Q, int64_t T, int32_t H, int64_t t_star) {
+    // each Q[t] is at most H (2^44 - 1): when H T* (2^44 - 1) < 2^64 the tail sum cannot
+    // wrap in 64 bits, and a plain 64-bit sum (which vectorises) is exact
+    const uint64_t *q = Q.data() + (T - t_star);
+    if ((unsigned __int128)H * (uint64_t)t_star * ((1ull << 44) - 1) < ((unsigned __int128)1 << 64)) {
+        uint64_t s64 = 0;
+        for (int64_t t = 0; t < t_star; ++t) s64 += q[t];
+        return s64;
+    }
+    unsigned __int128 S = 0;
+    for (int64_t t = 0; t < t_star; ++t) S += q[t];
+    return S;
+}
+
 // Canonical order of Algorithm 1: descending tail sum of the norm key over the
 // last T* = min T positions (the integer form of rho, Eq. rho), ties by
 // descending id read big-endian.
@@ -586,21 +691,7 @@ std::vector<std::shared_ptr<const Record>> canonical_order(const cm_set *set) {
     };
     std::vector<Keyed> keyed;
     keyed.reserve(recs.size());
-    for (auto &r : recs) {
-        // each Q[t] is at most H (2^44 - 1): when H T* (2^44 - 1) < 2^64 the tail sum
-        // cannot wrap in 64 bits, and a plain 64-bit sum (which vectorises) is exact
-        const uint64_t *q = r->Q.data() + (r->T - t_star);
-        unsigned __int128 S = 0;
-        if ((unsigned __int128)r->H * (uint64_t)t_star * ((1ull << 44) - 1) <
-            ((unsigned __int128)1 << 64)) {
-            uint64_t s64 = 0;
-            for (int64_t t = 0; t < t_star; ++t) s64 += q[t];
-            S = s64;
-        } else {
-            for (int64_t t = 0; t < t_star; ++t) S += q[t];
-        }
-        keyed.push_back({S, key_of(r->id), r});
-    }
+    for (auto &r : recs) keyed.push_back({tail_sum(r->Q, r->T, r->H, t_star), key_of(r->id), r});
     std::sort(keyed.begin(), keyed.end(), [](const Keyed &a, const Keyed &b) {
         if (a.S != b.S) return a.S > b.S;
         return a.id > b.id;
@@ -750,20 +841,18 @@ cm_status find_redeliveries(cm_context *ctx, cm_set *const *sets,
     return CM_OK;
 }
 
-// Ingest (Algorithm 2) of n deliveries, delivery i into sets[i] (several entries
-// may name one set): one GPU pass for all of them, then the insertions in delivery
-// order, so a delivery whose id its set already holds (before the batch or from an
-// earlier delivery of it) is absorbed. Nothing is inserted if validation fails.
-cm_status ingest_deliveries(cm_set *const *sets, const cm_fragment *frags, int32_t n,
-                            cm_stream_t stream, cm_id *out_ids, int32_t *out_absorbed) {
-    if (n == 0) return CM_OK;
+// Validation of n deliveries, delivery i into sets[i]: all sets from one context (*ctx),
+// each delivery of its set's shape (an empty set takes its first delivery's), a valid
+// routing layer. fp receives the descriptors.
+cm_status validate_deliveries(cm_set *const *sets, const cm_fragment *frags, int32_t n,
+                              cm_context **ctx_out, std::vector<const cm_fragment *> &fp) {
     cm_context *ctx = sets[0]->ctx;
     struct Shape {
         bool has;
         int32_t L, H, d;
     };
     std::unordered_map<const cm_set *, Shape> shape;
-    std::vector<const cm_fragment *> fp((size_t)n);
+    fp.assign((size_t)n, nullptr);
     for (int32_t i = 0; i < n; ++i) {
         const cm_set *set = sets[i];
         if (set->ctx != ctx) return fail(CM_ERR_INVALID_ARG, "sets belong to different contexts");
@@ -784,63 +873,70 @@ cm_status ingest_deliveries(cm_set *const *sets, const cm_fragment *frags, int32
             return fail(CM_ERR_INVALID_ARG, "routing layer >= num_layers");
         fp[(size_t)i] = f;
     }
-    std::lock_guard<std::mutex> lock(ctx->mu);
-    DeviceScope scope(ctx->device);
-    if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
-    const cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
-    // with the re-delivery fast path on, deliveries byte-identical to a known fragment
-    // take its id and norm key and are not hashed
-    std::vector<std::shared_ptr<const Record>> same_rec;
-    std::vector<int32_t> same_as;
-    cm_status st = CM_OK;
-    if (ctx->dedup_bytes) {
-        st = find_redeliveries(ctx, sets, fp, cs, same_rec, same_as);
-        if (st != CM_OK) return st;
-    } else {
-        same_rec.assign((size_t)n, nullptr);
-        same_as.assign((size_t)n, -1);
-    }
+    *ctx_out = ctx;
+    return CM_OK;
+}
+
+// Where delivery i's id and norm key come from: a stored record it is byte-identical to
+// (rec[i]), an earlier delivery of the call (from[i] >= 0), or the content-address pass
+// (hashed_as[i] indexes hashed_ids / hashed_Q).
+struct DeliverySources {
+    std::vector<std::shared_ptr<const Record>> rec;
+    std::vector<int32_t> from;
+    std::vector<size_t> hashed_as;
     std::vector<const cm_fragment *> to_hash;
-    std::vector<size_t> hashed_as((size_t)n, 0);
-    for (int32_t i = 0; i < n; ++i)
-        if (!same_rec[(size_t)i] && same_as[(size_t)i] < 0) {
-            hashed_as[(size_t)i] = to_hash.size();
-            to_hash.push_back(fp[(size_t)i]);
-        }
-    std::vector<cm_id> hashed_ids(to_hash.size());
-    std::vector<std::vector<uint64_t>> hashed_Q(to_hash.size());
-    if (!to_hash.empty()) {
-        st = fragments_digest(ctx, to_hash.data(), to_hash.size(), cs, hashed_ids.data(),
-                              hashed_Q.data());
-        if (st != CM_OK) return st;
+};
+
+DeliverySources hash_everything(size_t n, const std::vector<const cm_fragment *> &fp) {
+    DeliverySources src;
+    src.rec.assign(n, nullptr);
+    src.from.assign(n, -1);
+    src.hashed_as.resize(n);
+    for (size_t i = 0; i < n; ++i) {
+        src.hashed_as[i] = i;
+        src.to_hash.push_back(fp[i]);
     }
+    return src;
+}
+
+// The insertions of Ingest (Algorithm 2) in delivery order, once every delivery's id and
+// norm key are known: a delivery whose id its set already holds (before the call or from
+// an earlier delivery of it) is absorbed; with verify_bytes_on_hit its bytes are compared
+// with the stored record's first (CM_ERR_COLLISION if they differ: the deliveries before
+// it stay inserted). hashed_Q is consumed.
+cm_status insert_deliveries(cm_context *ctx, cm_set *const *sets,
+                            const std::vector<const cm_fragment *> &fp, cudaStream_t cs,
+                            const DeliverySources &src, const std::vector<cm_id> &hashed_ids,
+                            std::vector<std::vector<uint64_t>> &hashed_Q, cm_id *out_ids,
+                            int32_t *out_absorbed) {
+    const size_t n = fp.size();
     // ids in delivery order; Qsrc[i] is where delivery i's norm key lives once delivery i
     // has been processed (its own record, a record it matched, or a hashed result)
-    std::vector<cm_id> ids((size_t)n);
-    std::vector<const std::vector<uint64_t> *> Qsrc((size_t)n, nullptr);
-    for (int32_t i = 0; i < n; ++i) {
+    std::vector<cm_id> ids(n);
+    std::vector<const std::vector<uint64_t> *> Qsrc(n, nullptr);
+    for (size_t i = 0; i < n; ++i) {
         cm_set *set = sets[i];
-        const cm_fragment *f = fp[(size_t)i];
+        const cm_fragment *f = fp[i];
         std::vector<uint64_t> *own = nullptr;
-        if (same_rec[(size_t)i]) {
-            ids[(size_t)i] = same_rec[(size_t)i]->id;
-            Qsrc[(size_t)i] = &same_rec[(size_t)i]->Q;
-        } else if (same_as[(size_t)i] >= 0) {
-            ids[(size_t)i] = ids[(size_t)same_as[(size_t)i]];
-            Qsrc[(size_t)i] = Qsrc[(size_t)same_as[(size_t)i]];
+        if (src.rec[i]) {
+            ids[i] = src.rec[i]->id;
+            Qsrc[i] = &src.rec[i]->Q;
+        } else if (src.from[i] >= 0) {
+            ids[i] = ids[(size_t)src.from[i]];
+            Qsrc[i] = Qsrc[(size_t)src.from[i]];
         } else {
-            ids[(size_t)i] = hashed_ids[hashed_as[(size_t)i]];
-            own = &hashed_Q[hashed_as[(size_t)i]];
-            Qsrc[(size_t)i] = own;
+            ids[i] = hashed_ids[src.hashed_as[i]];
+            own = &hashed_Q[src.hashed_as[i]];
+            Qsrc[i] = own;
         }
-        if (out_ids) out_ids[i] = ids[(size_t)i];
-        const IdKey key = key_of(ids[(size_t)i]);
+        if (out_ids) out_ids[i] = ids[i];
+        const IdKey key = key_of(ids[i]);
         auto it = set->items.find(key);
         if (it != set->items.end()) {
             // a byte match against this very record needs no second look at the bytes
-            if (ctx->verify && same_rec[(size_t)i] != it->second) {
+            if (ctx->verify && src.rec[i] != it->second) {
                 bool equal = false;
-                st = bytes_equal(ctx, f, *it->second, cs, &equal);
+                cm_status st = bytes_equal(ctx, f, *it->second, cs, &equal);
                 if (st != CM_OK) return st;
                 if (!equal) return fail(CM_ERR_COLLISION, "content address hit with different bytes");
             }
@@ -848,7 +944,7 @@ cm_status ingest_deliveries(cm_set *const *sets, const cm_fragment *frags, int32
             continue;
         }
         auto rec = std::make_shared<Record>();
-        rec->id = ids[(size_t)i];
+        rec->id = ids[i];
         rec->L = f->num_layers;
         rec->H = f->num_kv_heads;
         rec->T = f->seq_len;
@@ -858,8 +954,8 @@ cm_status ingest_deliveries(cm_set *const *sets, const cm_fragment *frags, int32
         if (own)
             rec->Q = std::move(*own);
         else
-            rec->Q = *Qsrc[(size_t)i];
-        Qsrc[(size_t)i] = &rec->Q;
+            rec->Q = *Qsrc[i];
+        Qsrc[i] = &rec->Q;
         set->items.emplace(key, std::move(rec));
         if (!set->has_shape) {
             set->has_shape = true;
@@ -870,6 +966,66 @@ cm_status ingest_deliveries(cm_set *const *sets, const cm_fragment *frags, int32
         if (out_absorbed) out_absorbed[i] = 0;
     }
     return CM_OK;
+}
+
+// Ingest (Algorithm 2) of the validated deliveries fp, delivery i into sets[i]: one GPU
+// pass for all of them (after the re-delivery fast path, when it is on), then the
+// insertions in delivery order. Caller holds ctx->mu and the device scope.
+cm_status ingest_validated(cm_context *ctx, cm_set *const *sets,
+                           const std::vector<const cm_fragment *> &fp, cudaStream_t cs,
+                           cm_id *out_ids, int32_t *out_absorbed) {
+    const size_t n = fp.size();
+    DeliverySources src;
+    if (ctx->dedup_bytes) {
+        // deliveries byte-identical to a known fragment take its id and norm key and are
+        // not hashed
+        cm_status st = find_redeliveries(ctx, sets, fp, cs, src.rec, src.from);
+        if (st != CM_OK) return st;
+        src.hashed_as.assign(n, 0);
+        for (size_t i = 0; i < n; ++i)
+            if (!src.rec[i] && src.from[i] < 0) {
+                src.hashed_as[i] = src.to_hash.size();
+                src.to_hash.push_back(fp[i]);
+            }
+    } else {
+        src = hash_everything(n, fp);
+    }
+    std::vector<cm_id> hashed_ids(src.to_hash.size());
+    std::vector<std::vector<uint64_t>> hashed_Q(src.to_hash.size());
+    if (!src.to_hash.empty()) {
+        cm_status st = fragments_digest(ctx, src.to_hash.data(), src.to_hash.size(), cs,
+                                        hashed_ids.data(), hashed_Q.data());
+        if (st != CM_OK) return st;
+    }
+    return insert_deliveries(ctx, sets, fp, cs, src, hashed_ids, hashed_Q, out_ids, out_absorbed);
+}
+
+// Ingest (Algorithm 2) of n deliveries, delivery i into sets[i] (several entries
+// may name one set). Nothing is inserted if validation fails.
+cm_status ingest_deliveries(cm_set *const *sets, const cm_fragment *frags, int32_t n,
+                            cm_stream_t stream, cm_id *out_ids, int32_t *out_absorbed) {
+    if (n == 0) return CM_OK;
+    cm_context *ctx = nullptr;
+    std::vector<const cm_fragment *> fp;
+    cm_status st = validate_deliveries(sets, frags, n, &ctx, fp);
+    if (st != CM_OK) return st;
+    std::lock_guard<std::mutex> lock(ctx->mu);
+    DeviceScope scope(ctx->device);
+    if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
+    return ingest_validated(ctx, sets, fp, reinterpret_cast<cudaStream_t>(stream), out_ids,
+                            out_absorbed);
+}
+
+// dst := dst u src (Eq. setunion); shapes already checked. On equal ids dst keeps its
+// record (the bytes are equal).
+void union_into(cm_set *dst, const cm_set *src) {
+    for (const auto &kv : src->items) dst->items.emplace(kv.first, kv.second);
+    if (!dst->has_shape && src->has_shape) {
+        dst->has_shape = true;
+        dst->L = src->L;
+        dst->H = src->H;
+        dst->d = src->d;
+    }
 }
 
 }  // namespace
@@ -933,6 +1089,10 @@ cm_status cm_context_destroy(cm_context *ctx) {
         if (ctx->d_scratch) cudaFree(ctx->d_scratch);
         if (ctx->h_pinned) cudaFreeHost(ctx->h_pinned);
         if (ctx->d_error) cudaFree(ctx->d_error);
+        if (ctx->side) cudaStreamDestroy(ctx->side);
+        if (ctx->side_begin) cudaEventDestroy(ctx->side_begin);
+        if (ctx->side_end) cudaEventDestroy(ctx->side_end);
+        if (ctx->side_keys) cudaEventDestroy(ctx->side_keys);
         for (const auto &pe : ctx->pending) {
             cudaEventDestroy(pe.start);
             cudaEventDestroy(pe.end);
@@ -1027,6 +1187,14 @@ cm_status cm_context_set_dedup_by_bytes(cm_context *ctx, int32_t enable) {
     return CM_OK;
 }
 
+cm_status cm_context_set_overlap(cm_context *ctx, int32_t mode) {
+    if (!ctx) return fail(CM_ERR_INVALID_ARG, "context is NULL");
+    if (mode != 0 && mode != 1) return fail(CM_ERR_INVALID_ARG, "overlap mode must be 0 or 1");
+    std::lock_guard<std::mutex> lock(ctx->mu);
+    ctx->overlap = mode;
+    return CM_OK;
+}
+
 cm_status cm_context_set_render_warps(cm_context *ctx, int32_t warps) {
     if (!ctx) return fail(CM_ERR_INVALID_ARG, "context is NULL");
     if (warps != 8 && warps != 16) return fail(CM_ERR_INVALID_ARG, "render warps must be 8 or 16");
@@ -1090,13 +1258,7 @@ cm_status cm_union(cm_set *dst, const cm_set *src) {
         if (dst->has_shape && src->has_shape &&
             (dst->L != src->L || dst->H != src->H || dst->d != src->d))
             return fail(CM_ERR_SHAPE_MISMATCH, "sets have different shapes");
-        for (const auto &kv : src->items) dst->items.emplace(kv.first, kv.second);
-        if (!dst->has_shape && src->has_shape) {
-            dst->has_shape = true;
-            dst->L = src->L;
-            dst->H = src->H;
-            dst->d = src->d;
-        }
+        union_into(dst, src);
         return CM_OK;
     });
 }
@@ -1185,11 +1347,252 @@ cm_status render_set(const cm_set *set, void *k_out, void *v_out, int64_t capaci
     });
 }
 
+// Slots of the set's canonical order at offsets s = exclusive prefix sums of T, into
+// one contiguous output; *order receives the records in that order.
+std::vector<Slot> canonical_slots(const cm_set *set, void *k_out, void *v_out, int64_t capacity,
+                                  std::vector<std::shared_ptr<const Record>> *order) {
+    *order = canonical_order(set);
+    std::vector<Slot> slots;
+    int64_t s = 0;
+    for (const auto &r : *order) {
+        slots.push_back({r->k, r->v, r->T, s, k_out, v_out, capacity});
+        s += r->T;
+    }
+    return slots;
+}
+
+// A render beside the leaf hash (cm_ingest_render) whose fragments hold at least this
+// many bytes takes the 4-warp TMA kernel, a smaller one the register kernel with one CTA
+// per SM: measured on the Qwen3 shapes, the register kernel was the faster neighbour of
+// the hash for 0.3 GB of fragments, the TMA kernel from 1.2 GB on.
+constexpr uint64_t kBesideLargeBytes = 512ull << 20;
+
+cm_status ensure_side_stream(cm_context *ctx) {
+    if (!ctx->side) {
+        // the highest priority: the render's CTAs, launched while the leaf hash's grid is
+        // already queued, are dispatched as soon as any of its blocks retire
+        int least = 0, greatest = 0;
+        CM_CUDA_TRY(cudaDeviceGetStreamPriorityRange(&least, &greatest), "stream priorities");
+        CM_CUDA_TRY(cudaStreamCreateWithPriority(&ctx->side, cudaStreamNonBlocking, greatest),
+                    "side stream");
+    }
+    if (!ctx->side_begin)
+        CM_CUDA_TRY(cudaEventCreateWithFlags(&ctx->side_begin, cudaEventDisableTiming), "side event");
+    if (!ctx->side_end)
+        CM_CUDA_TRY(cudaEventCreateWithFlags(&ctx->side_end, cudaEventDisableTiming), "side event");
+    if (!ctx->side_keys)
+        CM_CUDA_TRY(cudaEventCreateWithFlags(&ctx->side_keys, cudaEventDisableTiming), "side event");
+    return CM_OK;
+}
+
+// cm_ingest_render (see include/cm.h). The norm keys of the deliveries are computed on
+// the context's side stream while the content address runs on `stream`. Equal bytes give
+// equal norm keys, so when the integer tail sums S (Eq. rho) of the prospective set's
+// members are pairwise distinct, no delivery can be absorbed and no two members can tie,
+// and the canonical order of Algorithm 1 is decided before any id is known: the render
+// then starts on the side stream (half-SM CTAs) beside the rest of the content address.
+// Once the ids are known the insertions and unions are made as usual; if the set that
+// results is not the one the render assumed (only a collision of the address, which the
+// paper excludes, could do that), it is rendered again after the first render.
+cm_status ingest_render_impl(cm_set *const *sets, const cm_fragment *frags, int32_t n,
+                             cm_set *target, void *k_out, void *v_out, int64_t capacity,
+                             cm_stream_t stream, cm_id *out_ids, int32_t *out_absorbed,
+                             int64_t *out_seq_len, cm_id *out_order, int32_t *out_overlapped) {
+    if (!target) return fail(CM_ERR_INVALID_ARG, "target set is NULL");
+    if (capacity < 0) return fail(CM_ERR_INVALID_ARG, "capacity_tokens < 0");
+    if (n < 0 || (n > 0 && (!frags || !sets)))
+        return fail(CM_ERR_INVALID_ARG, "need n >= 0 fragments and their sets");
+    for (int32_t i = 0; i < n; ++i)
+        if (!sets[i]) return fail(CM_ERR_INVALID_ARG, "a set is NULL");
+    if (out_overlapped) *out_overlapped = 0;
+    cm_context *ctx = target->ctx;
+    std::vector<const cm_fragment *> fp;
+    if (n > 0) {
+        cm_context *dctx = nullptr;
+        cm_status st = validate_deliveries(sets, frags, n, &dctx, fp);
+        if (st != CM_OK) return st;
+        if (dctx != ctx) return fail(CM_ERR_INVALID_ARG, "sets belong to different contexts");
+    }
+    // the union sources: the sets the deliveries go to, other than the target, in order
+    std::vector<cm_set *> sources;
+    for (int32_t i = 0; i < n; ++i)
+        if (sets[i] != target && std::find(sources.begin(), sources.end(), sets[i]) == sources.end())
+            sources.push_back(sets[i]);
+    bool has = false;
+    int32_t L = 0, H = 0, d = 0;
+    auto same_shape = [&](bool h, int32_t l, int32_t hh, int32_t dd) {
+        if (!h) return true;
+        if (!has) {
+            has = true;
+            L = l;
+            H = hh;
+            d = dd;
+            return true;
+        }
+        return l == L && hh == H && dd == d;
+    };
+    bool one_shape = same_shape(target->has_shape, target->L, target->H, target->d);
+    for (const cm_set *src : sources) one_shape = same_shape(src->has_shape, src->L, src->H, src->d) && one_shape;
+    for (const cm_fragment *f : fp)
+        one_shape = same_shape(true, f->num_layers, f->num_kv_heads, f->head_dim) && one_shape;
+    if (!one_shape)
+        return fail(CM_ERR_SHAPE_MISMATCH, "the target, the other sets and the deliveries of one "
+                                           "cm_ingest_render call must share one shape");
+    std::lock_guard<std::mutex> lock(ctx->mu);
+    DeviceScope scope(ctx->device);
+    if (!scope.ok()) return fail(CM_ERR_CUDA, "cannot select the CUDA device");
+    const cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+
+    // the one-after-the-other path: the re-delivery fast path compares bytes before any
+    // hashing, and overlap mode 0 asks for it
+    if (n == 0 || ctx->dedup_bytes || ctx->overlap == 0) {
+        cm_status st = n > 0 ? ingest_validated(ctx, sets, fp, cs, out_ids, out_absorbed) : CM_OK;
+        if (st != CM_OK) return st;
+        for (const cm_set *src : sources) union_into(target, src);
+        std::vector<std::shared_ptr<const Record>> order;
+        const std::vector<Slot> slots = canonical_slots(target, k_out, v_out, capacity, &order);
+        int64_t total = 0;
+        for (const auto &r : order) total += r->T;
+        st = validate_outputs(k_out, v_out, capacity, total);
+        if (st != CM_OK) return st;
+        if (out_seq_len) *out_seq_len = total;
+        if (out_order)
+            for (size_t i = 0; i < order.size(); ++i) out_order[i] = order[i]->id;
+        if (slots.empty()) return CM_OK;
+        return launch_slots(ctx, slots, target->L, target->H, target->d, cs);
+    }
+
+    // scratch: the content-address pass, then the norm keys (device and pinned host)
+    DigestPlan plan;
+    cm_status st = plan_digest(ctx, fp.data(), fp.size(), plan);
+    if (st != CM_OK) return st;
+    const size_t q_dev = (plan.dev_bytes + 255) & ~(size_t)255;
+    const size_t q_host = (plan.host_bytes + 255) & ~(size_t)255;
+    std::vector<size_t> q_off((size_t)n);
+    size_t q_bytes = 0;
+    for (int32_t i = 0; i < n; ++i) {
+        q_off[(size_t)i] = q_bytes;
+        q_bytes += (size_t)fp[(size_t)i]->seq_len * 8;
+    }
+    st = ensure_scratch(ctx, q_dev + q_bytes, q_host + q_bytes);
+    if (st == CM_OK) st = ensure_side_stream(ctx);
+    if (st != CM_OK) return st;
+    CM_CUDA_TRY(cudaEventRecord(ctx->side_begin, cs), "side stream ordering");
+    CM_CUDA_TRY(cudaStreamWaitEvent(ctx->side, ctx->side_begin, 0), "side stream ordering");
+    // from here on, every return joins the side stream into the caller's stream first
+    auto join = [&](cm_status prior) -> cm_status {
+        cudaError_t e = cudaEventRecord(ctx->side_end, ctx->side);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, ctx->side_end, 0);
+        if (e != cudaSuccess && prior == CM_OK) return cuda_fail(e, "side stream ordering");
+        return prior;
+    };
+    st = enqueue_norm_keys(ctx, fp.data(), fp.size(), ctx->side, q_dev, q_host, q_off, q_bytes);
+    if (st != CM_OK) return join(st);
+    cudaError_t e = cudaEventRecord(ctx->side_keys, ctx->side);
+    if (e != cudaSuccess) return join(cuda_fail(e, "side stream ordering"));
+    st = enqueue_digest(ctx, plan, fp.data(), fp.size(), cs, false);
+    if (st != CM_OK) return join(st);
+    e = cudaEventSynchronize(ctx->side_keys);
+    if (e != cudaSuccess) return join(cuda_fail(e, "norm-key synchronisation"));
+    std::vector<std::vector<uint64_t>> Qd((size_t)n);
+    for (int32_t i = 0; i < n; ++i) {
+        Qd[(size_t)i].resize((size_t)fp[(size_t)i]->seq_len);
+        std::memcpy(Qd[(size_t)i].data(), ctx->h_pinned + q_host + q_off[(size_t)i],
+                    (size_t)fp[(size_t)i]->seq_len * 8);
+    }
+
+    // the prospective set: the records of the target and of the sources (one per id),
+    // then every delivery; distinct tail sums decide its order
+    bool spec = true;
+    std::vector<Slot> spec_slots;
+    {
+        std::map<IdKey, std::shared_ptr<const Record>> have(target->items.begin(), target->items.end());
+        for (const cm_set *src : sources) have.insert(src->items.begin(), src->items.end());
+        int64_t t_star = INT64_MAX;
+        for (const auto &kv : have) t_star = std::min<int64_t>(t_star, kv.second->T);
+        for (const cm_fragment *f : fp) t_star = std::min<int64_t>(t_star, f->seq_len);
+        struct Member {
+            const void *k, *v;
+            int64_t T;
+            unsigned __int128 S;
+        };
+        std::vector<Member> m;
+        for (const auto &kv : have) {
+            const Record &r = *kv.second;
+            m.push_back({r.k, r.v, r.T, tail_sum(r.Q, r.T, r.H, t_star)});
+        }
+        for (size_t i = 0; i < fp.size(); ++i)
+            m.push_back({fp[i]->k, fp[i]->v, fp[i]->seq_len,
+                         tail_sum(Qd[i], fp[i]->seq_len, fp[i]->num_kv_heads, t_star)});
+        std::sort(m.begin(), m.end(), [](const Member &a, const Member &b) { return a.S > b.S; });
+        int64_t total = 0;
+        for (size_t i = 0; i < m.size(); ++i) {
+            if (i + 1 < m.size() && m[i].S == m[i + 1].S) spec = false;
+            total += m[i].T;
+        }
+        // an output the render would refuse: no speculation (the call then fails as
+        // cm_render does, after the ingest); a small merge: the render follows the hash
+        if (capacity < total || !k_out || !v_out || !aligned16(k_out) || !aligned16(v_out))
+            spec = false;
+        if (spec) {
+            int64_t s = 0;
+            for (const Member &x : m) {
+                spec_slots.push_back({x.k, x.v, x.T, s, k_out, v_out, capacity});
+                s += x.T;
+            }
+            // beside the leaf hash: a narrow render, its kernel chosen by size
+            const uint64_t frag_bytes = 2ull * (uint64_t)total * (uint64_t)L * (uint64_t)H * (uint64_t)d * 2;
+            const cm::RenderWidth beside = frag_bytes >= kBesideLargeBytes
+                                               ? cm::RenderWidth::kBeside
+                                               : cm::RenderWidth::kBesideSmall;
+            st = launch_slots(ctx, spec_slots, L, H, d, ctx->side, 0, nullptr, &beside);
+            if (st != CM_OK) return join(st);
+        }
+    }
+    e = cudaStreamSynchronize(cs);
+    if (e != cudaSuccess) return join(cuda_fail(e, "ingest synchronisation"));
+    std::vector<cm_id> ids((size_t)n);
+    collect_digest(ctx, plan, fp.data(), fp.size(), ids.data(), nullptr);
+    st = insert_deliveries(ctx, sets, fp, cs, hash_everything(fp.size(), fp), ids, Qd, out_ids,
+                           out_absorbed);
+    if (st != CM_OK) return join(st);
+    for (const cm_set *src : sources) union_into(target, src);
+    std::vector<std::shared_ptr<const Record>> order;
+    const std::vector<Slot> slots = canonical_slots(target, k_out, v_out, capacity, &order);
+    int64_t total = 0;
+    for (const auto &r : order) total += r->T;
+    st = validate_outputs(k_out, v_out, capacity, total);
+    if (st != CM_OK) return join(st);
+    if (out_seq_len) *out_seq_len = total;
+    if (out_order)
+        for (size_t i = 0; i < order.size(); ++i) out_order[i] = order[i]->id;
+    bool kept = spec && slots.size() == spec_slots.size();
+    for (size_t i = 0; kept && i < slots.size(); ++i)
+        kept = slots[i].k == spec_slots[i].k && slots[i].v == spec_slots[i].v &&
+               slots[i].T == spec_slots[i].T && slots[i].offset == spec_slots[i].offset;
+    // no speculation, or not the set that resulted: render now, after anything before
+    if (!kept && !slots.empty()) st = launch_slots(ctx, slots, target->L, target->H, target->d, ctx->side);
+    st = join(st);
+    if (st == CM_OK && out_overlapped) *out_overlapped = kept ? 1 : 0;
+    return st;
+}
+
 }  // namespace
 
 cm_status cm_render(const cm_set *set, void *k_out, void *v_out, int64_t capacity_tokens,
                     cm_stream_t stream, int64_t *out_seq_len, cm_id *out_order) {
     return render_set(set, k_out, v_out, capacity_tokens, stream, out_seq_len, out_order, 0);
+}
+
+cm_status cm_ingest_render(cm_set *const *sets, const cm_fragment *frags, int32_t n,
+                           cm_set *target, void *k_out, void *v_out, int64_t capacity_tokens,
+                           cm_stream_t stream, cm_id *out_ids, int32_t *out_absorbed,
+                           int64_t *out_seq_len, cm_id *out_order, int32_t *out_overlapped) {
+    TraceRange trace("cm_ingest_render");
+    return guarded([&]() -> cm_status {
+        return ingest_render_impl(sets, frags, n, target, k_out, v_out, capacity_tokens, stream,
+                                  out_ids, out_absorbed, out_seq_len, out_order, out_overlapped);
+    });
 }
 
 cm_status cm_render_many(const cm_render_job *jobs, int32_t n, cm_stream_t stream,

@@ -37,7 +37,7 @@ struct RenderParams {
     int32_t num_heads;
     int32_t head_dim;
     int32_t num_slots;
-    int32_t rows_per_chunk;     // render_item_bytes(warps) / (2 d)
+    int32_t rows_per_chunk;     // render_item_bytes(width) / (2 d)
     int32_t log2_pairs_per_row; // log2(d / 16)
     uint32_t total_chunks;
     uint32_t pad_;
@@ -58,16 +58,23 @@ struct RenderParams {
     double cs[2 * kMaxTablePairs];   // (cos a, sin a) of a = s * theta^(-2j/d), interleaved
 };
 
-// warps = 16: the full-SM render (all of each SM's warp slots it needs, no shared-memory
-// staging); warps = 8: the half-SM render (one 8-warp CTA per SM, leaving half of each
-// SM's registers to kernels of other streams). A launch group's work items are row
-// chunks of render_item_bytes(warps) bytes of one source plane; render_grid gives the
-// launch's CTA count for `chunks` items. render_prepare() once per device before the
-// first launch.
-cudaError_t launch_render(const RenderParams &p, int grid, int warps, cudaStream_t stream);
+// How much of each SM a render takes:
+//   kFull         the register kernel, 3 CTAs of 8 warps per SM (cm_context_set_render_warps(16),
+//                 the default): the fastest render alone
+//   kHalf         the TMA kernel, one CTA of 8 warps (3 stages each) per SM
+//                 (cm_context_set_render_warps(8)): half of each SM's registers stay free for
+//                 kernels of other streams
+//   kBeside       the TMA kernel, one CTA of 4 warps (6 stages each) per SM: a large render
+//                 beside the leaf hash of the same merge (cm_ingest_render)
+//   kBesideSmall  the register kernel, one 8-warp CTA per SM: a small render beside the leaf hash
+// A launch group's work items are row chunks of render_item_bytes(w) bytes of one source
+// plane; render_grid gives the launch's CTA count for `chunks` items. render_prepare() once
+// per device before the first launch.
+enum class RenderWidth { kFull, kHalf, kBeside, kBesideSmall };
+cudaError_t launch_render(const RenderParams &p, int grid, RenderWidth w, cudaStream_t stream);
 cudaError_t render_prepare();
-uint32_t render_item_bytes(int warps);
-int render_grid(uint64_t chunks, int num_sms, int warps);
+uint32_t render_item_bytes(RenderWidth w);
+int render_grid(uint64_t chunks, int num_sms, RenderWidth w);
 
 // Bounds-checked builds: reads and zeroes the render kernels' violation count on the
 // current device (0 in other builds).

@@ -20,7 +20,10 @@
 // streams; its warps keep three 4 KiB items in flight each as 1-D TMA bulk copies
 // into shared memory, which needs fewer warps for the same bytes in flight. For a
 // rotated K item a lane takes vector v of a row's first half and vector v of its
-// second half: 8 (x, y) pairs that share the lane's 8 (cos, sin) values.
+// second half: 8 (x, y) pairs that share the lane's 8 (cos, sin) values. A render that
+// runs beside the content address (cm_ingest_render) takes a narrower width still: the
+// TMA kernel with one CTA of 4 warps and 6 stages per SM for large renders, the register
+// kernel with one 8-warp CTA per SM for small ones (see RenderWidth).
 //
 // Rounding. The result must equal round-to-nearest-even-bf16 of
 // fl64(fl64(x c) - fl64(y s)) (and fl64(fl64(y c) + fl64(x s))), c and s the fp64
@@ -239,11 +242,11 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-constexpr int kStages = 3;                          // per warp
+constexpr int kStagesDefault = 3;                   // per warp
 constexpr uint32_t kItemBytes = 4096;               // one work item = one stage
 constexpr size_t kTableBytes = sizeof(float4) * kMaxTablePairs;
 // Dynamic shared memory of a CTA of kW warps: the warps' stages, then the (cos, sin) table.
-template <int kW>
+template <int kW, int kStages = kStagesDefault>
 constexpr size_t dyn_smem() { return (size_t)kW * kStages * kItemBytes + kTableBytes; }
 
 // One work item: up to kItemBytes of one source plane and where it goes.
@@ -477,8 +480,8 @@ __device__ __forceinline__ float2 split16(double c) {
 // place comes from the block table), and lane 0 refills the stage with the warp's
 // next item. Every wait is bounded: on timeout the warp records an error, waits
 // (bounded) for its own copies in flight and returns.
-template <bool kPaged, int kW>
-__global__ void __launch_bounds__(kW * 32, 16 / kW)
+template <bool kPaged, int kW, int kStages = kStagesDefault, int kMinBlocks = 16 / kW>
+__global__ void __launch_bounds__(kW * 32, kMinBlocks)
 render_kernel(const __grid_constant__ RenderParams p) {
     constexpr int kThreads = kW * 32;
     extern __shared__ __align__(128) uint8_t smem[];
@@ -550,10 +553,11 @@ render_kernel(const __grid_constant__ RenderParams p) {
     }
 }
 
-template <bool kPaged, int kW>
+template <bool kPaged, int kW, int kStages = kStagesDefault, int kMinBlocks = 16 / kW>
 cudaError_t set_smem_attribute() {
-    return cudaFuncSetAttribute(render_kernel<kPaged, kW>,
-                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn_smem<kW>());
+    return cudaFuncSetAttribute(render_kernel<kPaged, kW, kStages, kMinBlocks>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)dyn_smem<kW, kStages>());
 }
 
 // ---------------------------------------------------------------- full-SM render
@@ -801,29 +805,44 @@ CM_DEFINE_BOUNDS_READER(take_render_bounds_violations)
 cudaError_t render_prepare() {
     cudaError_t e = set_smem_attribute<false, 8>();
     if (e == cudaSuccess) e = set_smem_attribute<true, 8>();
+    if (e == cudaSuccess) e = set_smem_attribute<false, 4, 6, 4>();
+    if (e == cudaSuccess) e = set_smem_attribute<true, 4, 6, 4>();
     return e;
 }
 
-uint32_t render_item_bytes(int warps) { return warps == 8 ? kItemBytes : kRegItemBytes; }
-
-int render_grid(uint64_t chunks, int num_sms, int warps) {
-    if (warps == 8) return (int)std::max<uint64_t>(1, std::min<uint64_t>(chunks, (uint64_t)num_sms));
-    const uint64_t ctas = (chunks / 2 + kRegThreads / 32 - 1) / (kRegThreads / 32);
-    return (int)std::max<uint64_t>(1, std::min<uint64_t>(ctas, (uint64_t)kRegBlocksPerSm * num_sms));
+uint32_t render_item_bytes(RenderWidth w) {
+    return (w == RenderWidth::kHalf || w == RenderWidth::kBeside) ? kItemBytes : kRegItemBytes;
 }
 
-cudaError_t launch_render(const RenderParams &p, int grid, int warps, cudaStream_t stream) {
+int render_grid(uint64_t chunks, int num_sms, RenderWidth w) {
+    if (w == RenderWidth::kHalf || w == RenderWidth::kBeside)
+        return (int)std::max<uint64_t>(1, std::min<uint64_t>(chunks, (uint64_t)num_sms));
+    const uint64_t ctas = (chunks / 2 + kRegThreads / 32 - 1) / (kRegThreads / 32);
+    const uint64_t per_sm = w == RenderWidth::kFull ? (uint64_t)kRegBlocksPerSm : 1;
+    return (int)std::max<uint64_t>(1, std::min<uint64_t>(ctas, per_sm * num_sms));
+}
+
+cudaError_t launch_render(const RenderParams &p, int grid, RenderWidth w, cudaStream_t stream) {
     if (p.total_chunks == 0) return cudaSuccess;
-    if (warps == 8) {
-        if (p.paged)
-            render_kernel<true, 8><<<grid, 8 * 32, dyn_smem<8>(), stream>>>(p);
-        else
-            render_kernel<false, 8><<<grid, 8 * 32, dyn_smem<8>(), stream>>>(p);
-    } else {
-        if (p.paged)
-            render_reg_kernel<true><<<grid, kRegThreads, 0, stream>>>(p);
-        else
-            render_reg_kernel<false><<<grid, kRegThreads, 0, stream>>>(p);
+    switch (w) {
+        case RenderWidth::kHalf:
+            if (p.paged)
+                render_kernel<true, 8><<<grid, 8 * 32, dyn_smem<8>(), stream>>>(p);
+            else
+                render_kernel<false, 8><<<grid, 8 * 32, dyn_smem<8>(), stream>>>(p);
+            break;
+        case RenderWidth::kBeside:
+            if (p.paged)
+                render_kernel<true, 4, 6, 4><<<grid, 4 * 32, dyn_smem<4, 6>(), stream>>>(p);
+            else
+                render_kernel<false, 4, 6, 4><<<grid, 4 * 32, dyn_smem<4, 6>(), stream>>>(p);
+            break;
+        default:   // kFull, kBesideSmall: the register kernel (grid sizes differ)
+            if (p.paged)
+                render_reg_kernel<true><<<grid, kRegThreads, 0, stream>>>(p);
+            else
+                render_reg_kernel<false><<<grid, kRegThreads, 0, stream>>>(p);
+            break;
     }
     return cudaGetLastError();
 }

@@ -4,7 +4,8 @@ named by the environment variable CM_LIBRARY; started by test_gpu_bounds.py).
 Every global access of the render and content-address kernels is checked against the
 buffer it belongs to in that build. The cases below cover every kernel path (both render
 widths, contiguous, paged with power-of-two and other block sizes, both tree-top schemes,
-the allocation-free path, the re-delivery comparison, BagMerge and the incremental render);
+the allocation-free path, the re-delivery comparison, BagMerge, the incremental render and
+both renders that run beside the leaf hash in cm_ingest_render);
 their results are checked against the oracle or against each other, and the violation
 count must stay 0. A last case renders into a paged cache whose block table holds a
 negative entry, an input the host does not check: the bounds-checked build must count it
@@ -141,7 +142,39 @@ def main():
                                    for K, V in big]
     for S in sets:
         S.close()
-    del big
+    # the same fragments through cm_ingest_render (1.2 GB of fragments: the 4-warp TMA
+    # render beside the leaf hash), byte-equal to the separate calls' render
+    total = sum(K.shape[2] for K, _ in big)
+    fused_k, fused_v = empty_out(w.num_layers, w.num_kv_heads, total, w.head_dim)
+    A, B = cm.FragmentSet(ctx), cm.FragmentSet(ctx)
+    _, n, _, overlapped = cm.cm_ingest_render([A.handle, A.handle, B.handle, B.handle],
+                                              [cm.fragment_from_tensors(K, V) for K, V in big],
+                                              A.handle, fused_k.data_ptr(), fused_v.data_ptr(), total)
+    assert overlapped and n == total
+    S = cm.FragmentSet(ctx)
+    S.ingest_batch(big)
+    seq_k, seq_v = empty_out(w.num_layers, w.num_kv_heads, total, w.head_dim)
+    S.render(seq_k, seq_v)
+    torch.cuda.synchronize()
+    assert torch.equal(fused_k.view(torch.int16), seq_k.view(torch.int16))
+    assert torch.equal(fused_v.view(torch.int16), seq_v.view(torch.int16))
+    for X in (A, B, S):
+        X.close()
+    del big, fused_k, fused_v, seq_k, seq_v
+    cases += 1
+    # a small merge through cm_ingest_render (the register render, one CTA per SM, beside
+    # the hash), checked against the oracle
+    fs = frags_of(61, 3, 2, 64, (37, 53, 90))
+    kc3, vc3, order3 = check_render(ctx, fs)
+    A = cm.FragmentSet(ctx)
+    k3, v3 = empty_out(3, 2, 180, 64)
+    _, n, order, overlapped = cm.cm_ingest_render([A.handle] * 3,
+                                                  [cm.fragment_from_tensors(K, V) for K, V in fs],
+                                                  A.handle, k3.data_ptr(), v3.data_ptr(), 180)
+    torch.cuda.synchronize()
+    assert overlapped and n == 180 and order == order3
+    assert torch.equal(k3, kc3) and torch.equal(v3, vc3)
+    A.close()
     cases += 1
 
     # re-delivery fast path: clones take their originals' ids without being hashed

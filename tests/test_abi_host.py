@@ -33,7 +33,8 @@ def test_header_declares_the_documented_calls():
             "cm_context_set_timing", "cm_context_kernel_times", "cm_fragment_id_static",
             "cm_render_incremental", "cm_render_paged", "cm_ingest_many", "cm_render_many",
             "cm_set_contains", "cm_set_leq", "cm_measure_int_alu",
-            "cm_context_set_render_warps", "cm_context_set_dedup_by_bytes"}
+            "cm_context_set_render_warps", "cm_context_set_dedup_by_bytes", "cm_ingest_render",
+            "cm_context_set_overlap"}
     assert want <= set(_declared_functions())
 
 
@@ -45,7 +46,7 @@ def test_library_exports_every_declared_symbol(cm):
 
 
 def test_abi_version_and_status_strings(cm):
-    assert cm.cm_abi_version() == 4
+    assert cm.cm_abi_version() == 5
     for st in cm.Status:
         assert cm.cm_status_string(int(st)) == "CM_" + st.name
     assert cm.cm_status_string(99) == "CM_ERR_UNKNOWN"

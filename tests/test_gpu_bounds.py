@@ -29,7 +29,7 @@ def test_bounds_checked_build_sees_no_access_outside_its_buffers():
     assert r.returncode == 0, r.stdout[-4000:]
     res = json.loads(r.stdout.strip().splitlines()[-1])
     assert res["enabled"]
-    assert res["cases"] >= 34
+    assert res["cases"] >= 35
     assert res["violations"] == 0
     assert res["negative_table_entry_violations"] > 0
     assert res["violations_after"] == 0
