@@ -132,8 +132,9 @@ cm_status cm_fragment_id(cm_context *ctx, const cm_fragment *frag, cm_stream_t s
  *                  on `stream` first, then accumulated)
  * Limit: the fragment's K and V bytes (2 * L * H * T * d * 2) must not exceed 1 GiB;
  * larger fragments return CM_ERR_UNSUPPORTED (use cm_fragment_id).
- * The first call on a device looks up the array's device address (cudaGetSymbolAddress)
- * and caches it; make that first call before any stream capture on that device.
+ * Every call looks the array's device address up (cudaGetSymbolAddress, on the calling
+ * thread's current device) and keeps no copy of it, so a device reset or another context
+ * on the device never leaves a stale address in use.
  * Every call shares the one array: calls whose GPU work overlaps (on different
  * streams, or from several threads) race and corrupt each other's results; order
  * them on one stream or synchronise between them. Returns after enqueueing. */

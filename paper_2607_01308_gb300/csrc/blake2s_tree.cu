@@ -588,21 +588,16 @@ cudaError_t launch_compare(const void *a, const void *b, uint64_t bytes, unsigne
 // cannot allocate device memory: its scratch (the digests of every tree level
 // below the root) lives in the file-scope array below, which every GPU that loads
 // this library holds for the life of the process. Host code never uses the
-// array's name as an address: the first call on a device looks its device address
-// up with cudaGetSymbolAddress (with that device current) and caches it.
-
-#include <mutex>
+// array's name as an address: every call looks the array's device address up with
+// cudaGetSymbolAddress, with the calling thread's device current, and keeps no copy
+// of it, so a device reset or another context on the device, either of which can
+// move the array, never leaves a stale address in use.
 
 namespace cm {
 namespace {
 
 constexpr uint64_t kStaticMaxLeaves = 1ull << 20;                // byte stream of at most 1 GiB
 constexpr size_t kStaticScratchBytes = (17u << 20) + (256u << 10);   // 17.25 MiB
-constexpr int kStaticMaxDevices = 128;
-
-std::mutex g_static_mu;
-void *g_static_addr[kStaticMaxDevices] = {};
-
 }  // namespace
 
 static __device__ __align__(256) uint8_t g_static_scratch[kStaticScratchBytes];
@@ -645,26 +640,15 @@ extern "C" cm_status cm_fragment_id_static(const cm_fragment *frag, int32_t rout
         }
         if (used > kStaticScratchBytes)
             return report_error(CM_ERR_UNSUPPORTED, "static scratch layout overflow");
-        int dev = 0;
-        cudaError_t e = cudaGetDevice(&dev);
-        if (e != cudaSuccess) return report_error(CM_ERR_CUDA, cudaGetErrorString(e));
-        if (dev < 0 || dev >= kStaticMaxDevices)
-            return report_error(CM_ERR_UNSUPPORTED, "device ordinal beyond 127");
-        uint8_t *scratch = nullptr;
-        {
-            std::lock_guard<std::mutex> lock(g_static_mu);
-            if (!g_static_addr[dev]) {
-                void *p = nullptr;
-                e = cudaGetSymbolAddress(&p, g_static_scratch);
-                if (e != cudaSuccess) {
-                    cudaGetLastError();
-                    return report_error(CM_ERR_CUDA, cudaGetErrorString(e));
-                }
-                g_static_addr[dev] = p;
-            }
-            scratch = static_cast<uint8_t *>(g_static_addr[dev]);
-        }
+        cudaError_t e = cudaSuccess;
         const cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+        void *addr = nullptr;
+        e = cudaGetSymbolAddress(&addr, g_static_scratch);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return report_error(CM_ERR_CUDA, cudaGetErrorString(e));
+        }
+        uint8_t *scratch = static_cast<uint8_t *>(addr);
         e = cudaMemsetAsync(norm_key_out, 0, (size_t)T * sizeof(uint64_t), cs);
         if (e != cudaSuccess) return report_error(CM_ERR_CUDA, cudaGetErrorString(e));
         LeafLaunch a;
