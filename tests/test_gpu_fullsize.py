@@ -1,11 +1,10 @@
 """GPU parity at the benchmark's full sizes, in the launch configuration bench.py
-times (one cm_ingest_many call feeds two replicas half the fragments each, union,
-render), and at the full sizes of the other workloads.
+times (one cm_ingest_render call: two replicas take half the fragments each, union,
+render, with the render beside the content address), and at the full sizes of the
+other workloads.
 
 The oracle computes every content address and norm key in full (hashlib over all
-bytes) and the render on sampled (slot, layer, head) planes: each output plane
-depends only on its source plane and the slot's offset, so a sampled plane is
-checked exactly as a full render would check it. V planes are compared bit for
+bytes) and renders every (slot, layer, head) plane: V planes are compared bit for
 bit, K planes within 1 bf16 ulp with the non-exact count asserted to be 0.
 """
 import itertools
@@ -49,20 +48,20 @@ def _oracle_order(keys, lengths):
     return sorted(range(len(keys)), key=lambda i: (-S[i], -id_as_int(keys[i][0])))
 
 
-def _check_sampled_planes(frags, order, k_out, v_out, layers, heads):
+def _check_all_planes(frags, order, k_out, v_out):
+    """Every plane of the render against the oracle: each slot's K rotated by its offset
+    (oracle.rotate_k over all layers and heads at once), each slot's V copied."""
+    kb, vb = synthetic.to_bits(k_out), synthetic.to_bits(v_out)
     s = 0
     for i in order:
         K, V = frags[i]
         T = K.shape[2]
-        for l in layers:
-            for h in heads:
-                src_k = synthetic.to_bits(K[l, h])
-                got_k = synthetic.to_bits(k_out[l, h, s:s + T])
-                want_k = oracle.rotate_k(src_k, s, THETA)
-                assert assert_k_parity(got_k, want_k, f"K slot@{s} l={l} h={h}") == 0
-                assert np.array_equal(synthetic.to_bits(v_out[l, h, s:s + T]),
-                                      synthetic.to_bits(V[l, h]))
+        want_k = oracle.rotate_k(synthetic.to_bits(K), s, THETA)
+        assert assert_k_parity(kb[:, :, s:s + T], want_k, f"K slot@{s}") == 0
+        assert np.array_equal(vb[:, :, s:s + T], synthetic.to_bits(V)), f"V slot@{s}"
+        del want_k
         s += T
+    assert s == kb.shape[2]
 
 
 def test_q4b_full_size_bench_configuration(ctx):
@@ -71,29 +70,45 @@ def test_q4b_full_size_bench_configuration(ctx):
     frags = [synthetic.make_fragment_torch(sp, w.num_layers, w.num_kv_heads, w.head_dim, "cuda:0")
              for sp in specs]
     A, B = cm.FragmentSet(ctx), cm.FragmentSet(ctx)
-    # the bench's launch configuration: one cm_ingest_many call feeds both replicas
-    cm.cm_context_kernel_times(ctx.handle, reset=True)
-    cm.cm_context_set_timing(ctx.handle, True)
-    res = cm.ingest_many([(A, *frags[0]), (A, *frags[1]), (B, *frags[2]), (B, *frags[3])])
-    cm.cm_context_set_timing(ctx.handle, False)
-    t = cm.cm_context_kernel_times(ctx.handle, reset=True)
-    # 4 x 36,864 level-1 nodes: level 1 in its own kernel, then the levels above it
-    assert t["leaf_hash_launches"] == 1 and t["inner_hash_launches"] == 2
-    ra, rb = res[:2], res[2:]
-    A.union(B)
     total = sum(sp.seq_len for sp in specs)
     k_out, v_out = empty_out(w.num_layers, w.num_kv_heads, total, w.head_dim)
-    n, order_ids = A.render(k_out, v_out)
+    # the bench's launch configuration: one cm_ingest_render call, replicas A (fragments 0,
+    # 1) and B (2, 3), A rendered with the render beside the content address
+    cm.cm_context_kernel_times(ctx.handle, reset=True)
+    cm.cm_context_set_timing(ctx.handle, True)
+    res, n, order_ids, overlapped = cm.cm_ingest_render(
+        [A.handle, A.handle, B.handle, B.handle],
+        [cm.fragment_from_tensors(K, V) for K, V in frags], A.handle, k_out.data_ptr(),
+        v_out.data_ptr(), total)
+    cm.cm_context_set_timing(ctx.handle, False)
+    t = cm.cm_context_kernel_times(ctx.handle, reset=True)
     ctx.check()
     torch.cuda.synchronize()
+    assert overlapped
+    # 4 x 36,864 level-1 nodes: level 1 in its own kernel, then the levels above it
+    assert t["leaf_hash_launches"] == 1 and t["inner_hash_launches"] == 2
+    assert t["render_launches"] == 1
     keys = _oracle_keys(frags, w.num_layers // 2)
-    assert [fid for fid, _ in ra + rb] == [k[0] for k in keys]
+    assert [fid for fid, _ in res] == [k[0] for k in keys]
+    assert [a for _, a in res] == [False] * 4
     order = _oracle_order(keys, [sp.seq_len for sp in specs])
     assert order_ids == [keys[i][0] for i in order]
     assert n == total
-    _check_sampled_planes(frags, order, k_out, v_out, layers=[0, 18, 35], heads=[0, 7])
-    A.close()
-    B.close()
+    _check_all_planes(frags, order, k_out, v_out)
+    # the same merge as separate calls: cm_ingest_many, cm_union, cm_render (the full-SM
+    # render after the hash), byte for byte
+    A2, B2 = cm.FragmentSet(ctx), cm.FragmentSet(ctx)
+    res2 = cm.ingest_many([(A2, *frags[0]), (A2, *frags[1]), (B2, *frags[2]), (B2, *frags[3])])
+    assert res2 == res
+    A2.union(B2)
+    k2, v2 = empty_out(w.num_layers, w.num_kv_heads, total, w.head_dim)
+    n2, order2 = A2.render(k2, v2)
+    torch.cuda.synchronize()
+    assert n2 == n and order2 == order_ids
+    assert torch.equal(k2.view(torch.int16), k_out.view(torch.int16))
+    assert torch.equal(v2.view(torch.int16), v_out.view(torch.int16))
+    for S in (A, B, A2, B2):
+        S.close()
 
 
 def test_split_tree_top_with_roots_at_levels_one_and_two(ctx):
@@ -148,7 +163,7 @@ def test_redelivery_fast_path_at_full_size():
     torch.cuda.synchronize()
     order = _oracle_order(keys, [sp.seq_len for sp in specs])
     assert n == total and order_ids == [keys[i][0] for i in order]
-    _check_sampled_planes(frags, order, k_out, v_out, layers=[0, 18, 35], heads=[2, 5])
+    _check_all_planes(frags, order, k_out, v_out)
     S.close()
     c.close()
 
@@ -175,7 +190,7 @@ def test_serving_requests_with_redelivery(ctx, request_index):
     keys = _oracle_keys(frags, w.num_layers // 2)
     order = _oracle_order(keys, [sp.seq_len for sp in specs])
     assert order_ids == [keys[i][0] for i in order] and n == total
-    _check_sampled_planes(frags, order, k_out, v_out, layers=[1, 18], heads=[3])
+    _check_all_planes(frags, order, k_out, v_out)
     S.close()
 
 
@@ -205,7 +220,7 @@ def test_arity_batch_matches_sequential_ingest_and_oracle(ctx):
     assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
     order = _oracle_order(keys, [sp.seq_len for sp in specs])
     assert outs[0][2] == [keys[i][0] for i in order]
-    _check_sampled_planes(frags, order, outs[0][0], outs[0][1], layers=[0, 14, 27], heads=[0, 5])
+    _check_all_planes(frags, order, outs[0][0], outs[0][1])
     S1.close()
     S2.close()
 
@@ -252,7 +267,7 @@ def test_arity_all_120_orders_render_identically_at_full_length(ctx):
     keys = _oracle_keys(frags, w.num_layers // 2)
     order = _oracle_order(keys, [sp.seq_len for sp in specs])
     assert ref[2] == [keys[i][0] for i in order]
-    _check_sampled_planes(frags, order, ref[0], ref[1], layers=[0, 14, 27], heads=[0, 7])
+    _check_all_planes(frags, order, ref[0], ref[1])
     for S in singles:
         S.close()
 

@@ -114,6 +114,12 @@ def _paged_check(ctx, frags, block_size, layout, seed):
         kg = kp[blk, :, :, off].permute(1, 2, 0, 3)
         vg = vp[blk, :, :, off].permute(1, 2, 0, 3)
     assert torch.equal(kg, kc) and torch.equal(vg, vc)
+    # and the gathered paged result against the oracle directly
+    K_ref, V_ref, o_order = oracle.render(
+        oracle.from_deliveries([oracle_fragment(K, V) for K, V in frags]), THETA)
+    assert order == [f.fid for f in o_order]
+    assert np.array_equal(synthetic.to_bits(vg), V_ref)
+    assert assert_k_parity(synthetic.to_bits(kg), K_ref) == 0
     # the spare blocks and the tail of the last used block are untouched
     used = set(table.tolist())
     spare = [b for b in range(num_blocks) if b not in used]

@@ -63,6 +63,25 @@ def test_fragment_id_and_norm_key_match_oracle(ctx, shape):
     assert np.array_equal(np.array(Q, dtype=np.uint64), ref.Q)
 
 
+def test_fragment_id_matches_the_frozen_golden_ids(ctx):
+    # the ids recorded in tests/golden/content_address_ids.json by the oracle
+    import importlib.util
+    import json
+    import os
+    here = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+    spec = importlib.util.spec_from_file_location("_golden_ca", os.path.join(here, "content_address_ids.py"))
+    gen = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(gen)
+    with open(os.path.join(here, "content_address_ids.json")) as fh:
+        rows = json.load(fh)["fragments"]
+    for row in rows:
+        Kb, Vb = gen.fragment_bits(row["shape"], row["seed"])
+        K = torch.from_numpy(Kb.view(np.int16)).to("cuda:0").view(torch.bfloat16)
+        V = torch.from_numpy(Vb.view(np.int16)).to("cuda:0").view(torch.bfloat16)
+        fid, _ = ctx.fragment_id(K, V)
+        assert fid.hex() == row["id_hex"], row["name"]
+
+
 def test_norm_key_special_values(ctx):
     L, H, T, d = 2, 2, 6, 16
     K = torch.zeros((L, H, T, d), dtype=torch.bfloat16, device="cuda:0")
@@ -76,6 +95,21 @@ def test_norm_key_special_values(ctx):
     ref = oracle_fragment(K, V)
     assert fid == ref.fid
     assert np.array_equal(np.array(Q, dtype=np.uint64), ref.Q)
+
+
+def test_norm_key_rounds_exact_halves_to_even(ctx):
+    # rows of 16 equal entries k 2^-23: 2^20 n = k / 2 exactly, rounded half to even
+    # (0, 2, 2, 4, 4 for k = 1, 3, 5, 7, 9), for one head and summed over two
+    ks, want = [1, 3, 5, 7, 9], [0, 2, 2, 4, 4]
+    for H in (1, 2):
+        K = torch.zeros((2, H, len(ks), 16), dtype=torch.bfloat16, device="cuda:0")
+        for t, k in enumerate(ks):
+            K[1, :, t, :] = k * 2.0 ** -23
+        V = torch.zeros_like(K)
+        fid, Q = ctx.fragment_id(K, V)
+        assert list(Q) == [H * q for q in want]
+        ref = oracle_fragment(K, V)
+        assert fid == ref.fid and np.array_equal(np.array(Q, dtype=np.uint64), ref.Q)
 
 
 def test_norm_key_wide_exponent_range(ctx):

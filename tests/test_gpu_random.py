@@ -114,6 +114,12 @@ def test_random_paged_render_matches_contiguous(ctx, seed):
     else:
         kg, vg = kp[blk, :, :, off].permute(1, 2, 0, 3), vp[blk, :, :, off].permute(1, 2, 0, 3)
     assert torch.equal(kg, k) and torch.equal(vg, v)
+    # and the gathered paged result against the oracle directly
+    refs = [oracle_fragment(K, V) for K, V in frags]
+    K_ref, V_ref, o_order = oracle.render(oracle.from_deliveries([refs[i] for i in deliveries]), THETA)
+    assert order2 == [f.fid for f in o_order]
+    assert np.array_equal(synthetic.to_bits(vg), V_ref)
+    assert assert_k_parity(synthetic.to_bits(kg), K_ref) == 0
     spare = [b for b in range(num_blocks) if b not in set(table.tolist())]
     untouched = kp.view(torch.int16)[:, spare] if layout == "per_layer" else kp.view(torch.int16)[spare]
     assert (untouched == 0x1357).all()

@@ -133,3 +133,26 @@ def test_salt_and_personalisation_byte_layout():
     assert pb[8:14] == (5).to_bytes(6, "little") and pb[14:16] == bytes([2, 16])
     assert pb[16:24] == bytes([28, 0, 8, 0, 128, 0, 1, 0])
     assert pb[24:32] == bytes([0, 0x10, 0, 0, 0, 0, 0, 0])
+
+
+def _golden_ids():
+    import importlib.util
+    import json
+    import os
+    here = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+    spec = importlib.util.spec_from_file_location("_golden_ca", os.path.join(here, "content_address_ids.py"))
+    gen = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(gen)
+    with open(os.path.join(here, "content_address_ids.json")) as fh:
+        return gen, json.load(fh)["fragments"]
+
+
+def test_content_address_is_frozen_on_golden_fragments():
+    # the ids recorded when the address's definition was fixed: any change to the leaf
+    # size, fanout, parameter block or byte stream changes them
+    from oracle.content_address import fragment_id
+    gen, rows = _golden_ids()
+    assert len(rows) == 3
+    for row in rows:
+        K, V = gen.fragment_bits(row["shape"], row["seed"])
+        assert fragment_id(K, V).hex() == row["id_hex"], row["name"]

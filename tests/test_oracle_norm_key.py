@@ -94,3 +94,23 @@ def test_sum_over_heads_and_default_layer():
     for t in range(7):
         if all(q[h][t] is not None for h in range(5)):
             assert int(Q[t]) == sum(q[h][t] for h in range(5))
+
+
+# rows of d = 16 equal entries k 2^-23 have norm 4 k 2^-23, so 2^20 n = k / 2 exactly:
+# half-integers for odd k, which round half to even (0.5 -> 0, 1.5 -> 2, 2.5 -> 2,
+# 3.5 -> 4, 4.5 -> 4); floor(x + 0.5) or rounding half away from zero would give
+# 1, 2, 3, 4, 5
+HALF_TIE_K = [1, 3, 5, 7, 9]
+HALF_TIE_Q = [0, 2, 2, 4, 4]
+
+
+def test_quantise_rounds_exact_halves_to_even():
+    n = np.array([k * 2.0 ** -21 for k in HALF_TIE_K])          # 2^20 n = k / 2
+    assert list(nk.quantise(n)) == HALF_TIE_Q
+    K = np.zeros((2, 1, len(HALF_TIE_K), 16), dtype=np.uint16)
+    K[1] = _const_layer([[k * 2.0 ** -23 for k in HALF_TIE_K]], 16)
+    assert list(nk.norm_key(K, 1)) == HALF_TIE_Q
+    # two heads: each adds its own rounded term
+    K2 = np.zeros((2, 2, len(HALF_TIE_K), 16), dtype=np.uint16)
+    K2[1] = _const_layer([[k * 2.0 ** -23 for k in HALF_TIE_K]] * 2, 16)
+    assert list(nk.norm_key(K2, 1)) == [2 * q for q in HALF_TIE_Q]
