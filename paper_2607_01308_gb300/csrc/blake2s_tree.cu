@@ -243,7 +243,7 @@ __global__ void __launch_bounds__(kLeafThreads)
 leaf_hash_kernel(const __grid_constant__ LeafGroup grp) {
     // the blocks after the leaf blocks compute norm keys, one thread per row of K[l*]:
     // they fill SMs that the last wave of leaf blocks leaves idle
-    const uint32_t x = blockIdx.x + grp.first_block;
+    const uint32_t x = blockIdx.x;
     const uint32_t leaf_blocks = (uint32_t)grp.block_begin[grp.count];
     if (x >= leaf_blocks) {
         const uint32_t k = x - leaf_blocks;
@@ -305,6 +305,18 @@ leaf_hash_kernel(const __grid_constant__ LeafGroup grp) {
     if (CM_IN_BOUNDS(a.digests + leaf * kDigestBytes, kDigestBytes, a.digests,
                      a.num_leaves * kDigestBytes))
         store_digest(a.digests + leaf * kDigestBytes, h);
+}
+
+// The norm-key rows of a group alone (the blocks that follow the leaf blocks in
+// leaf_hash_kernel, as their own launch): one thread per row of K[l*].
+__global__ void __launch_bounds__(kLeafThreads)
+norm_key_kernel(const __grid_constant__ LeafGroup grp) {
+    const uint32_t k = blockIdx.x;
+    uint32_t fi = 0;
+    while (fi + 1 < grp.count && k >= grp.norm_block_begin[fi + 1]) ++fi;
+    const LeafLaunch &a = grp.frag[fi];
+    const uint64_t r = (uint64_t)(k - grp.norm_block_begin[fi]) * kLeafThreads + threadIdx.x;
+    if (r < (a.plane_bytes >> (__ffs(a.row_bytes) - 1))) norm_row(a, r);
 }
 
 constexpr int kInnerThreads = 32;
@@ -503,14 +515,14 @@ cudaError_t launch_leaf_hash_group(const LeafGroup &in, cudaStream_t stream, Lea
     g.norm_block_begin[g.count] = norm_blocks;
     const uint64_t leaf_blocks = g.block_begin[g.count];
     if (leaf_blocks + norm_blocks > 0x7FFFFFFFull) return cudaErrorInvalidValue;
-    // the grid covers blocks [first_block, first_block + blocks) of the combined range:
-    // leaf blocks first, then norm-key blocks
-    uint64_t blocks = 0;
-    switch (phases) {
-        case LeafPhases::kBoth: g.first_block = 0; blocks = leaf_blocks + norm_blocks; break;
-        case LeafPhases::kLeaves: g.first_block = 0; blocks = leaf_blocks; break;
-        case LeafPhases::kNormKeys: g.first_block = (uint32_t)leaf_blocks; blocks = norm_blocks; break;
+    // leaf blocks first, then norm-key blocks; a grid of the leaf blocks alone has no
+    // norm-key block, and the norm keys alone run in their own kernel
+    if (phases == LeafPhases::kNormKeys) {
+        if (norm_blocks == 0) return cudaSuccess;
+        norm_key_kernel<<<(unsigned)norm_blocks, kLeafThreads, 0, stream>>>(g);
+        return cudaGetLastError();
     }
+    const uint64_t blocks = phases == LeafPhases::kBoth ? leaf_blocks + norm_blocks : leaf_blocks;
     if (blocks == 0) return cudaSuccess;
     leaf_hash_kernel<<<(unsigned)blocks, kLeafThreads, 0, stream>>>(g);
     return cudaGetLastError();

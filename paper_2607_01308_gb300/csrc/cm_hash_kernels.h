@@ -47,7 +47,7 @@ constexpr int kMaxLeafGroup = 32;
 constexpr int kLeafBlockThreads = 128;   // threads (= leaves or rows) per block of the leaf launch
 struct LeafGroup {
     uint32_t count;
-    uint32_t first_block;          // set by the launcher: block index of the grid's block 0
+    uint32_t pad_;
     uint64_t block_begin[kMaxLeafGroup + 1];
     uint64_t norm_block_begin[kMaxLeafGroup + 1];
     LeafLaunch frag[kMaxLeafGroup];
