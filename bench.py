@@ -1094,7 +1094,7 @@ def main():
             "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
             else "fallback 6.8 TB/s", "unit": "GB/s",
             "frac": render_bytes / (kernel_render_ms * 1e-3) / 1e9 / peak,
-            "traffic": profile_traffic("render.cu", "render_kernel_q4b.md"),
+            "traffic": profile_traffic("render.cu", "render_reg_kernel_q4b.md"),
             "algorithmic_bytes_per_launch": render_bytes, "ms_per_launch": kernel_render_ms,
             "timing": "CUDA events on the render's stream around each launch in the sequential "
                       "steps (the full-SM render alone; the stream is idle when the start event is "
