@@ -589,7 +589,9 @@ struct PairWalk {
     uint32_t pr, npairs, stride;
     int si;
     uint32_t lhp, c, st_l, st_c;
+    uint32_t l, h, st_pl, st_ph;   // paged outputs: lhp = l * H + h, st_l = st_pl * H + st_ph
 
+    template <bool kPaged>
     __device__ __forceinline__ void enter(const RenderParams &p) {
         si = 0;
         while (si + 1 < p.num_slots && 2 * pr >= p.slot[si + 1].chunk_begin) ++si;
@@ -599,22 +601,43 @@ struct PairWalk {
         c = local - lhp * S.chunks_per_plane;
         st_l = stride / S.chunks_per_plane;
         st_c = stride - st_l * S.chunks_per_plane;
+        if (kPaged) {
+            const uint32_t H = (uint32_t)p.num_heads;
+            l = lhp / H;
+            h = lhp - l * H;
+            st_pl = st_l / H;
+            st_ph = st_l - st_pl * H;
+        }
     }
+    template <bool kPaged>
     __device__ __forceinline__ bool next(const RenderParams &p) {
         pr += stride;
         if (pr >= npairs) return false;
         const uint32_t cpp = p.slot[si].chunks_per_plane;
         c += st_c;
         lhp += st_l;
+        uint32_t carry = 0;
         if (c >= cpp) {
             c -= cpp;
             ++lhp;
+            carry = 1;
         }
-        if (lhp >= (uint32_t)(p.num_layers * p.num_heads)) enter(p);
+        if (lhp >= (uint32_t)(p.num_layers * p.num_heads)) {
+            enter<kPaged>(p);
+        } else if (kPaged) {
+            const uint32_t H = (uint32_t)p.num_heads;
+            h += st_ph + carry;   // < 2H: one correction
+            l += st_pl;
+            if (h >= H) {
+                h -= H;
+                ++l;
+            }
+        }
         return true;
     }
 };
 
+template <bool kPaged>
 __device__ __forceinline__ Pair pair_of(const RenderParams &p, const PairWalk &w) {
     const RenderSlot &S = p.slot[w.si];
     const int64_t row_bytes = (int64_t)p.head_dim * 2;
@@ -625,10 +648,8 @@ __device__ __forceinline__ Pair pair_of(const RenderParams &p, const PairWalk &w
     const int64_t so = ((int64_t)w.lhp * S.seq_len + row0) * row_bytes;
     q.ks = static_cast<const uint8_t *>(S.k) + so;
     q.vs = static_cast<const uint8_t *>(S.v) + so;
-    if (p.paged) {
-        const uint32_t l32 = w.lhp / (uint32_t)p.num_heads;
-        const int64_t l = l32, h = (int64_t)(w.lhp - l32 * (uint32_t)p.num_heads);
-        const int64_t o = (l * p.stride_layer + h * p.stride_head) * 2;
+    if (kPaged) {
+        const int64_t o = ((int64_t)w.l * p.stride_layer + (int64_t)w.h * p.stride_head) * 2;
         q.kd = static_cast<uint8_t *>(p.k_pool) + o;
         q.vd = static_cast<uint8_t *>(p.v_pool) + o;
     } else {
@@ -676,12 +697,54 @@ __device__ __forceinline__ Item half_item(const Pair &q, bool v) {
     return it;
 }
 
+// Paged outputs: where the rows of a pair go, for K and V alike (the two halves differ only
+// in their pool). When the block size is a power of two no smaller than the pair's row
+// count, the rows lie in at most two logical blocks: row r goes to half + da + r * stride
+// before the block boundary (r < split), to half + db + r * stride after it, the block
+// table read once per pair; otherwise (fast false) every row looks its block up.
+struct PagedOffsets {
+    int64_t da, db, stride;
+    int split;
+    bool fast;
+};
+
+__device__ __forceinline__ PagedOffsets paged_offsets(const RenderParams &p, int64_t pos0, int rows) {
+    PagedOffsets o;
+    o.fast = p.log2_block_size >= 0 && (int64_t)rows <= p.block_size;
+    o.stride = p.stride_token * 2;
+    o.split = rows;
+    o.da = o.db = 0;
+    if (o.fast) {
+        const int64_t b0 = pos0 >> p.log2_block_size;
+        const int64_t o0 = pos0 & (p.block_size - 1);
+        const int64_t k = p.block_size - o0;                 // rows left in block b0
+        o.da = table_entry(p, b0) * p.stride_block * 2 + o0 * o.stride;
+        if (k < rows) {
+            o.split = (int)k;
+            o.db = table_entry(p, b0 + 1) * p.stride_block * 2 - k * o.stride;
+        }
+    }
+    return o;
+}
+
+// Row r of one half of a pair (half = the half's item).
+template <bool kPaged>
+__device__ __forceinline__ uint4 *pair_row(const RenderParams &p, const Item &half,
+                                           const PagedOffsets &po, int r) {
+    if (!kPaged) return reinterpret_cast<uint4 *>(half.dst) + (int64_t)r * (p.head_dim >> 3);
+    if (po.fast)
+        return reinterpret_cast<uint4 *>(half.dst + (r < po.split ? po.da : po.db) + (int64_t)r * po.stride);
+    PagedRows slow{};
+    slow.fast = false;
+    return row_dst<true>(p, half, r, slow);
+}
+
 // Stores vector v (0 <= v < rows * d / 8) of a copied item.
 template <bool kPaged>
-__device__ __forceinline__ void store_vec(const RenderParams &p, const Item &it, const PagedRows &pr,
-                                          int v, const uint4 &x) {
+__device__ __forceinline__ void store_vec(const RenderParams &p, const Item &it,
+                                          const PagedOffsets &po, int v, const uint4 &x) {
     const int log2_vpr = p.log2_pairs_per_row + 1;   // vectors per row = d / 8
-    uint4 *d = row_dst<kPaged>(p, it, v >> log2_vpr, pr) + (v & ((1 << log2_vpr) - 1));
+    uint4 *d = pair_row<kPaged>(p, it, po, v >> log2_vpr) + (v & ((1 << log2_vpr) - 1));
     if (CM_IN_BOUNDS(d, 16, it.dst_base, it.dst_size)) st_stream(d, x);
 }
 
@@ -710,7 +773,7 @@ render_reg_kernel(const __grid_constant__ RenderParams p) {
     w.stride = gridDim.x * (kRegThreads / 32);
     w.npairs = p.total_chunks / 2;
     if (w.pr >= w.npairs) return;
-    w.enter(p);
+    w.enter<kPaged>(p);
     const int half_vecs = p.head_dim >> 4;
     const int vecs_per_row = p.head_dim >> 3;
     const int log2_hv = p.log2_pairs_per_row;
@@ -718,7 +781,7 @@ render_reg_kernel(const __grid_constant__ RenderParams p) {
     int cur = -1;
     float c[8], s[8];
     do {
-        const Pair q = pair_of(p, w);
+        const Pair q = pair_of<kPaged>(p, w);
         const int n_vec = q.rows * vecs_per_row;
         const int n_pairs = q.rows * half_vecs;
         const uint4 *ks = reinterpret_cast<const uint4 *>(q.ks);
@@ -750,15 +813,13 @@ render_reg_kernel(const __grid_constant__ RenderParams p) {
             rv[u] = make_uint4(0, 0, 0, 0);
             if (v < n_vec && CM_IN_BOUNDS(vs + v, 16, q.vs_base, q.src_size)) rv[u] = __ldcs(vs + v);
         }
+        PagedOffsets po{};
+        if (kPaged) po = paged_offsets(p, q.pos0, q.rows);
         const Item vi = half_item(q, true);
-        PagedRows pv{};
-        if (kPaged) pv = paged_rows(p, vi);
 #pragma unroll
         for (int u = 0; u < kRegVecs; ++u)
-            if (lane + 32 * u < n_vec) store_vec<kPaged>(p, vi, pv, lane + 32 * u, rv[u]);
+            if (lane + 32 * u < n_vec) store_vec<kPaged>(p, vi, po, lane + 32 * u, rv[u]);
         const Item ki = half_item(q, false);
-        PagedRows pk{};
-        if (kPaged) pk = paged_rows(p, ki);
         if (q.rotate) {
             if (q.cs_index != cur) {
                 cur = q.cs_index;
@@ -784,7 +845,7 @@ render_reg_kernel(const __grid_constant__ RenderParams p) {
                     rotate_word(a.w, b.w, c[6], s[6], c[7], s[7], ao.w, bo.w, b3);
                     if ((b0 | b1 | b2 | b3) != 0u)
                         fixup_pair(p, tab, cur + 8 * lane_v, a, b, b0, b1, b2, b3, ao, bo);
-                    uint4 *d = row_dst<kPaged>(p, ki, qq >> log2_hv, pk) + lane_v;
+                    uint4 *d = pair_row<kPaged>(p, ki, po, qq >> log2_hv) + lane_v;
                     if (CM_IN_BOUNDS(d, 16, ki.dst_base, ki.dst_size)) st_stream(d, ao);
                     if (CM_IN_BOUNDS(d + half_vecs, 16, ki.dst_base, ki.dst_size))
                         st_stream(d + half_vecs, bo);
@@ -793,9 +854,9 @@ render_reg_kernel(const __grid_constant__ RenderParams p) {
         } else {
 #pragma unroll
             for (int u = 0; u < kRegVecs; ++u)
-                if (lane + 32 * u < n_vec) store_vec<kPaged>(p, ki, pk, lane + 32 * u, rk[u]);
+                if (lane + 32 * u < n_vec) store_vec<kPaged>(p, ki, po, lane + 32 * u, rk[u]);
         }
-    } while (w.next(p));
+    } while (w.next<kPaged>(p));
 }
 
 }  // namespace
