@@ -1151,6 +1151,9 @@ def main():
             "timing": "CUDA events around each leaf-hash launch in the timed steps, where the "
                       "render of the same merge runs beside it on another stream (cm_ingest_render); "
                       "hash_roofline has the same kernel alone",
+            "note": "in the timed steps the render shares the SMs with this kernel, so this "
+                    "fraction counts the hash's own work only; alone the kernel reaches "
+                    "hash_roofline.frac",
         })
         render_in_step = {
             "kernel": "render_kernel (4-warp TMA CTAs) beside the leaf hash", "ms_per_launch": render_ms_ovl,
