@@ -1479,10 +1479,24 @@ cm_status ingest_render_impl(cm_set *const *sets, const cm_fragment *frags, int3
     if (st != CM_OK) return st;
     CM_CUDA_TRY(cudaEventRecord(ctx->side_begin, cs), "side stream ordering");
     CM_CUDA_TRY(cudaStreamWaitEvent(ctx->side, ctx->side_begin, 0), "side stream ordering");
-    // from here on, every return joins the side stream into the caller's stream first
+    // from here on, every way out (a C++ exception included) orders the caller's stream
+    // after the side stream's work: explicitly through join(), else in the destructor
+    struct SideJoin {
+        cm_context *ctx;
+        cudaStream_t cs;
+        bool done = false;
+        cudaError_t run() {
+            done = true;
+            cudaError_t e = cudaEventRecord(ctx->side_end, ctx->side);
+            if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, ctx->side_end, 0);
+            return e;
+        }
+        ~SideJoin() {
+            if (!done) run();
+        }
+    } side_join{ctx, cs};
     auto join = [&](cm_status prior) -> cm_status {
-        cudaError_t e = cudaEventRecord(ctx->side_end, ctx->side);
-        if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, ctx->side_end, 0);
+        const cudaError_t e = side_join.run();
         if (e != cudaSuccess && prior == CM_OK) return cuda_fail(e, "side stream ordering");
         return prior;
     };
