@@ -28,11 +28,12 @@
 // Rounding. The result must equal round-to-nearest-even-bf16 of
 // fl64(fl64(x c) - fl64(y s)) (and fl64(fl64(y c) + fl64(x s))), c and s the fp64
 // cosine and sine. The fast path computes z in fp32 with one fma from c and s
-// rounded to fp32 and bounds its distance to the fp64 value by
-// E = (1 + 2^-9) 2^-24 (|z| + |x||c| + 2|y||s|) + 2^-148 (|x| + |y|) + 2^-146 (see
-// err_bound). If z - E and z + E (rounded outward) round to the same bf16, every
-// value between them does (rounding is monotone), the fp64 value included, and z's
-// rounding is the answer. Otherwise (about one element in eight thousand) a second
+// rounded to fp32 and bounds its distance to the fp64 value by one bound for both
+// outputs of an element pair, E = k_j (|x| + |y|) + 2^-145 with a per-frequency constant
+// k_j = (1 + 2^-8) 2^-24 max(2|c|, 3|s|) (see bound_scale). If z - E and z + E (rounded
+// outward) round to the same bf16, every value between them does (rounding is
+// monotone), the fp64 value included, and z's rounding is the answer. Otherwise (about
+// one element in five thousand) a second
 // fp32 level with error-free products and a ~2^-36 bound decides, and the few it
 // cannot certify are recomputed in fp64 with the operation sequence of the
 // definition and rounded directly to bf16 (fp64 throughput is very low on this part,
@@ -86,33 +87,37 @@ __device__ uint32_t f64_to_bf16_bits(double z) {
 //                     <= (1 + 2^-9) u (|z| + |x||c32| + 2 |y||s32|) + 2^-148 (|x| + |y|) + 2^-146,
 // the last two terms covering roundings in the subnormal range (absolute error 2^-150
 // each) and the fp64 value's own distance to x c - y s (below 2^-52 of the products).
-// `rest` is the shared 2^-148 (|x| + |y|) + 2^-146; p1, p2 are the two operands whose
-// products enter the rounded sum (p1 multiplies c, p2 multiplies s).
-__device__ __forceinline__ float err_bound(float z, float p1, float c, float p2, float s,
-                                           float rest) {
-    const float a = __fmaf_ru(2.0f, __fmul_ru(fabsf(p2), fabsf(s)), __fmul_ru(fabsf(p1), fabsf(c)));
-    return __fmaf_ru(__fadd_ru(a, fabsf(z)), 0x1.008p-24f, rest);
+// With M = max(2|c32|, 3|s32|): |z| <= (1 + u)|x||c32| + (1 + u)^2 |y||s32| + 2^-148, so
+// |z| + |x||c32| + 2|y||s32| <= (1 + u) M (|x| + |y|) + 2^-148; and M >= 6/sqrt(13) > 1.66
+// (c32^2 + s32^2 is within 2^-22 of 1), so 2^-148 (|x| + |y|) is far below the margin
+// (2^-8 - 2^-9 - u - 2^-33) u M (|x| + |y|). Hence
+//   |z - X| <= (1 + 2^-8) u M (|x| + |y|) + 2^-145 = k (|x| + |y|) + 2^-145,
+// X the fp64 value, and the same for y' = fl(y c32 + fl(x s32)) (|x| and |y| swap roles,
+// M stays). bound_scale returns k rounded up, from the fp32 (c32, s32) of one frequency.
+__device__ __forceinline__ float bound_scale(float c32, float s32) {
+    const float m = fmaxf(2.0f * fabsf(c32), __fmul_ru(3.0f, fabsf(s32)));
+    return __fmul_ru(m, 0x1.01p-24f);
 }
 
-// Rotate the pairs (x0, y0), (x1, y1) held in word xw (x0 low, x1 high) and word yw.
-// Returns the rotated words and a mask whose nonzero 16-bit halves mark elements
-// whose fp32 result is not certified.
-__device__ __forceinline__ void rotate_word(uint32_t xw, uint32_t yw, float c0, float s0, float c1,
-                                            float s1, uint32_t &xo, uint32_t &yo, uint32_t &bad) {
+// Rotate the pairs (x0, y0), (x1, y1) held in word xw (x0 low, x1 high) and word yw
+// (frequency of pair e: c_e, s_e and bound scale k_e). Returns the rotated words and a
+// mask whose nonzero 16-bit halves mark elements whose fp32 result is not certified.
+__device__ __forceinline__ void rotate_word(uint32_t xw, uint32_t yw, float c0, float s0, float k0,
+                                            float c1, float s1, float k1, uint32_t &xo,
+                                            uint32_t &yo, uint32_t &bad) {
     const float x0 = bf16_lo(xw), x1 = bf16_hi(xw);
     const float y0 = bf16_lo(yw), y1 = bf16_hi(yw);
     const float zx0 = __fmaf_rn(x0, c0, -__fmul_rn(y0, s0));
     const float zx1 = __fmaf_rn(x1, c1, -__fmul_rn(y1, s1));
     const float zy0 = __fmaf_rn(y0, c0, __fmul_rn(x0, s0));
     const float zy1 = __fmaf_rn(y1, c1, __fmul_rn(x1, s1));
-    const float r0 = __fmaf_ru(__fadd_ru(fabsf(x0), fabsf(y0)), 0x1p-148f, 0x1p-146f);
-    const float r1 = __fmaf_ru(__fadd_ru(fabsf(x1), fabsf(y1)), 0x1p-148f, 0x1p-146f);
-    const float ex0 = err_bound(zx0, x0, c0, y0, s0, r0), ex1 = err_bound(zx1, x1, c1, y1, s1, r1);
-    const float ey0 = err_bound(zy0, y0, c0, x0, s0, r0), ey1 = err_bound(zy1, y1, c1, x1, s1, r1);
-    const uint32_t bx = pack_bf16x2(__fsub_rd(zx0, ex0), __fsub_rd(zx1, ex1)) ^
-                        pack_bf16x2(__fadd_ru(zx0, ex0), __fadd_ru(zx1, ex1));
-    const uint32_t by = pack_bf16x2(__fsub_rd(zy0, ey0), __fsub_rd(zy1, ey1)) ^
-                        pack_bf16x2(__fadd_ru(zy0, ey0), __fadd_ru(zy1, ey1));
+    // one bound for both outputs of a pair: E = k (|x| + |y|) + 2^-145, rounded up
+    const float e0 = __fmaf_ru(__fadd_ru(fabsf(x0), fabsf(y0)), k0, 0x1p-145f);
+    const float e1 = __fmaf_ru(__fadd_ru(fabsf(x1), fabsf(y1)), k1, 0x1p-145f);
+    const uint32_t bx = pack_bf16x2(__fsub_rd(zx0, e0), __fsub_rd(zx1, e1)) ^
+                        pack_bf16x2(__fadd_ru(zx0, e0), __fadd_ru(zx1, e1));
+    const uint32_t by = pack_bf16x2(__fsub_rd(zy0, e0), __fsub_rd(zy1, e1)) ^
+                        pack_bf16x2(__fadd_ru(zy0, e0), __fadd_ru(zy1, e1));
     xo = pack_bf16x2(zx0, zx1);
     yo = pack_bf16x2(zy0, zy1);
     bad = bx | by;
@@ -161,8 +166,11 @@ __device__ __forceinline__ void put_half(uint4 &v, int e, uint32_t bits) {
     else v.w = (v.w & keep) | val;
 }
 
-// Re-evaluates the elements of one vector pair whose masks b0..b3 flag them.
-__device__ __noinline__ void fixup_pair(const RenderParams &p, const float4 *tab, int cs_index,
+// Re-evaluates the elements of one vector pair whose masks b0..b3 flag them. Inlined: as a
+// called function its call (argument and result registers, a stack frame) cost the
+// full-SM render 0.80 instead of 0.754 ms on the Qwen3-4B-shaped merge, though only about
+// one warp iteration in twenty takes it.
+__device__ __forceinline__ void fixup_pair(const RenderParams &p, const float4 *tab, int cs_index,
                                         const uint4 &a, const uint4 &b, uint32_t b0, uint32_t b1,
                                         uint32_t b2, uint32_t b3, uint4 &ao, uint4 &bo) {
     const uint32_t bw[4] = {b0, b1, b2, b3};
@@ -244,7 +252,8 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 
 constexpr int kStagesDefault = 3;                   // per warp
 constexpr uint32_t kItemBytes = 4096;               // one work item = one stage
-constexpr size_t kTableBytes = sizeof(float4) * kMaxTablePairs;
+// (c1, c2, s1, s2) per frequency, then the first-level bound scale k per frequency
+constexpr size_t kTableBytes = (sizeof(float4) + sizeof(float)) * kMaxTablePairs;
 // Dynamic shared memory of a CTA of kW warps: the warps' stages, then the (cos, sin) table.
 template <int kW, int kStages = kStagesDefault>
 constexpr size_t dyn_smem() { return (size_t)kW * kStages * kItemBytes + kTableBytes; }
@@ -425,8 +434,8 @@ __device__ __forceinline__ void copy_from_smem(const RenderParams &p, const Item
 // the same for every q, so its 8 (cos, sin) values are loaded once per item.
 template <bool kPaged>
 __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const float4 *tab,
-                                                 const Item &it, const uint8_t *buf, int lane,
-                                                 int lane_v) {
+                                                 const float *kt, const Item &it,
+                                                 const uint8_t *buf, int lane, int lane_v) {
     const int vecs_per_row = p.head_dim >> 3;
     const int half_vecs = p.head_dim >> 4;
     const int n_pairs = it.rows * half_vecs;
@@ -447,12 +456,14 @@ __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const fl
         const int off = row * vecs_per_row + lane_v;
         const uint4 a = src[off];
         const uint4 b = src[off + half_vecs];
+        const float4 ka = *reinterpret_cast<const float4 *>(kt + cs_index);
+        const float4 kb = *reinterpret_cast<const float4 *>(kt + cs_index + 4);
         uint4 ao, bo;
         uint32_t b0, b1, b2, b3;
-        rotate_word(a.x, b.x, c[0], s[0], c[1], s[1], ao.x, bo.x, b0);
-        rotate_word(a.y, b.y, c[2], s[2], c[3], s[3], ao.y, bo.y, b1);
-        rotate_word(a.z, b.z, c[4], s[4], c[5], s[5], ao.z, bo.z, b2);
-        rotate_word(a.w, b.w, c[6], s[6], c[7], s[7], ao.w, bo.w, b3);
+        rotate_word(a.x, b.x, c[0], s[0], ka.x, c[1], s[1], ka.y, ao.x, bo.x, b0);
+        rotate_word(a.y, b.y, c[2], s[2], ka.z, c[3], s[3], ka.w, ao.y, bo.y, b1);
+        rotate_word(a.z, b.z, c[4], s[4], kb.x, c[5], s[5], kb.y, ao.z, bo.z, b2);
+        rotate_word(a.w, b.w, c[6], s[6], kb.z, c[7], s[7], kb.w, ao.w, bo.w, b3);
         if ((b0 | b1 | b2 | b3) != 0u) fixup_pair(p, tab, cs_index, a, b, b0, b1, b2, b3, ao, bo);
         uint4 *d = row_dst<kPaged>(p, it, row, pr) + lane_v;
         if (CM_IN_BOUNDS(d, 16, it.dst_base, it.dst_size)) st_stream(d, ao);
@@ -488,12 +499,14 @@ render_kernel(const __grid_constant__ RenderParams p) {
     __shared__ __align__(8) uint64_t full[kW][kStages];
     __shared__ Item items[kW][kStages];
     float4 *tab = reinterpret_cast<float4 *>(smem + (size_t)kW * kStages * kItemBytes);
+    float *kt = reinterpret_cast<float *>(tab + kMaxTablePairs);
 
     const int half = p.head_dim >> 1;
     const int n_table = p.num_slots * half;
     for (int i = threadIdx.x; i < n_table; i += kThreads) {
         const float2 cc = split16(p.cs[2 * i]), ss = split16(p.cs[2 * i + 1]);
         tab[i] = make_float4(cc.x, cc.y, ss.x, ss.y);
+        kt[i] = bound_scale(__fadd_rn(cc.x, cc.y), __fadd_rn(ss.x, ss.y));
     }
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (lane == 0) {
@@ -537,7 +550,7 @@ render_kernel(const __grid_constant__ RenderParams p) {
         const Item it = items[warp][s];
         const uint8_t *buf = wbuf + (size_t)s * kItemBytes;
         if (it.rotate)
-            rotate_from_smem<kPaged>(p, tab, it, buf, lane, lane_v);
+            rotate_from_smem<kPaged>(p, tab, kt, it, buf, lane, lane_v);
         else
             copy_from_smem<kPaged>(p, it, buf, lane);
         __syncwarp();                          // every lane is done reading stage s
@@ -758,13 +771,13 @@ template <bool kPaged>
 __global__ void __launch_bounds__(kRegThreads, kRegBlocksPerSm)
 render_reg_kernel(const __grid_constant__ RenderParams p) {
     __shared__ float4 tab[kMaxTablePairs];   // (c1, c2, s1, s2) for the second level
-    __shared__ float2 cs32[kMaxTablePairs];  // (c32, s32) = (fl(c1 + c2), fl(s1 + s2))
+    __shared__ __align__(16) float kt[kMaxTablePairs];   // first-level bound scale per frequency
     const int half = p.head_dim >> 1;
     const int n_table = p.num_slots * half;
     for (int i = threadIdx.x; i < n_table; i += kRegThreads) {
         const float2 cc = split16(p.cs[2 * i]), ss = split16(p.cs[2 * i + 1]);
         tab[i] = make_float4(cc.x, cc.y, ss.x, ss.y);
-        cs32[i] = make_float2(__fadd_rn(cc.x, cc.y), __fadd_rn(ss.x, ss.y));
+        kt[i] = bound_scale(__fadd_rn(cc.x, cc.y), __fadd_rn(ss.x, ss.y));
     }
     __syncthreads();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -825,24 +838,25 @@ render_reg_kernel(const __grid_constant__ RenderParams p) {
                 cur = q.cs_index;
 #pragma unroll
                 for (int e = 0; e < 8; ++e) {
-                    const float2 t = cs32[cur + 8 * lane_v + e];
-                    c[e] = t.x;
-                    s[e] = t.y;
+                    const float4 t = tab[cur + 8 * lane_v + e];
+                    c[e] = __fadd_rn(t.x, t.y);   // (c32, s32) = (fl(c1 + c2), fl(s1 + s2))
+                    s[e] = __fadd_rn(t.z, t.w);
                 }
             }
 #pragma unroll
             for (int k = 0; k < kRegVecs / 2; ++k) {
                 const int qq = lane + 32 * k;
                 if (qq < n_pairs) {
-                    // copies, not references into rk: the non-inlined fixup must not
-                    // force the register arrays into local memory
+                    // copies of the two vectors, which the fix-up also reads
                     const uint4 a = rk[2 * k], b = rk[2 * k + 1];
+                    const float4 ka = *reinterpret_cast<const float4 *>(kt + cur + 8 * lane_v);
+                    const float4 kb = *reinterpret_cast<const float4 *>(kt + cur + 8 * lane_v + 4);
                     uint4 ao, bo;
                     uint32_t b0, b1, b2, b3;
-                    rotate_word(a.x, b.x, c[0], s[0], c[1], s[1], ao.x, bo.x, b0);
-                    rotate_word(a.y, b.y, c[2], s[2], c[3], s[3], ao.y, bo.y, b1);
-                    rotate_word(a.z, b.z, c[4], s[4], c[5], s[5], ao.z, bo.z, b2);
-                    rotate_word(a.w, b.w, c[6], s[6], c[7], s[7], ao.w, bo.w, b3);
+                    rotate_word(a.x, b.x, c[0], s[0], ka.x, c[1], s[1], ka.y, ao.x, bo.x, b0);
+                    rotate_word(a.y, b.y, c[2], s[2], ka.z, c[3], s[3], ka.w, ao.y, bo.y, b1);
+                    rotate_word(a.z, b.z, c[4], s[4], kb.x, c[5], s[5], kb.y, ao.z, bo.z, b2);
+                    rotate_word(a.w, b.w, c[6], s[6], kb.z, c[7], s[7], kb.w, ao.w, bo.w, b3);
                     if ((b0 | b1 | b2 | b3) != 0u)
                         fixup_pair(p, tab, cur + 8 * lane_v, a, b, b0, b1, b2, b3, ao, bo);
                     uint4 *d = pair_row<kPaged>(p, ki, po, qq >> log2_hv) + lane_v;
