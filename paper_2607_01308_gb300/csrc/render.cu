@@ -99,27 +99,63 @@ __device__ __forceinline__ float bound_scale(float c32, float s32) {
     return __fmul_ru(m, 0x1.01p-24f);
 }
 
+// Paired fp32 arithmetic (sm_100 and later): two fp32 operations, elementwise, in one
+// instruction on a register pair; the rounding of each half is that of the scalar op.
+__device__ __forceinline__ uint64_t pair_of(float lo, float hi) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+__device__ __forceinline__ void halves(uint64_t v, float &lo, float &hi) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t mul2_rn(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+__device__ __forceinline__ uint64_t fma2_rn(uint64_t a, uint64_t b, uint64_t c) {
+    uint64_t r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+__device__ __forceinline__ uint64_t sub2_rd(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("sub.rm.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+__device__ __forceinline__ uint64_t add2_ru(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("add.rp.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+// the two halves of a pair as bf16, round to nearest even (lo in bits 0..15)
+__device__ __forceinline__ uint32_t pack_pair(uint64_t v) {
+    float lo, hi;
+    halves(v, lo, hi);
+    return pack_bf16x2(lo, hi);
+}
+
 // Rotate the pairs (x0, y0), (x1, y1) held in word xw (x0 low, x1 high) and word yw
-// (frequency of pair e: c_e, s_e and bound scale k_e). Returns the rotated words and a
-// mask whose nonzero 16-bit halves mark elements whose fp32 result is not certified.
-__device__ __forceinline__ void rotate_word(uint32_t xw, uint32_t yw, float c0, float s0, float k0,
-                                            float c1, float s1, float k1, uint32_t &xo,
-                                            uint32_t &yo, uint32_t &bad) {
+// (frequency of pair e: c_e, s_e, ns_e = -s_e and bound scale k_e), the two pairs of a
+// word in paired instructions: x' = fma(x, c, fl(y ns)), y' = fma(y, c, fl(x s)), the
+// scalar operations of the bound's proof. Returns the rotated words and a mask whose
+// nonzero 16-bit halves mark elements whose fp32 result is not certified.
+__device__ __forceinline__ void rotate_word(uint32_t xw, uint32_t yw, float c0, float s0,
+                                            float ns0, float k0, float c1, float s1, float ns1,
+                                            float k1, uint32_t &xo, uint32_t &yo, uint32_t &bad) {
     const float x0 = bf16_lo(xw), x1 = bf16_hi(xw);
     const float y0 = bf16_lo(yw), y1 = bf16_hi(yw);
-    const float zx0 = __fmaf_rn(x0, c0, -__fmul_rn(y0, s0));
-    const float zx1 = __fmaf_rn(x1, c1, -__fmul_rn(y1, s1));
-    const float zy0 = __fmaf_rn(y0, c0, __fmul_rn(x0, s0));
-    const float zy1 = __fmaf_rn(y1, c1, __fmul_rn(x1, s1));
+    const uint64_t X = pair_of(x0, x1), Y = pair_of(y0, y1), C = pair_of(c0, c1);
+    const uint64_t ZX = fma2_rn(X, C, mul2_rn(Y, pair_of(ns0, ns1)));
+    const uint64_t ZY = fma2_rn(Y, C, mul2_rn(X, pair_of(s0, s1)));
     // one bound for both outputs of a pair: E = k (|x| + |y|) + 2^-145, rounded up
-    const float e0 = __fmaf_ru(__fadd_ru(fabsf(x0), fabsf(y0)), k0, 0x1p-145f);
-    const float e1 = __fmaf_ru(__fadd_ru(fabsf(x1), fabsf(y1)), k1, 0x1p-145f);
-    const uint32_t bx = pack_bf16x2(__fsub_rd(zx0, e0), __fsub_rd(zx1, e1)) ^
-                        pack_bf16x2(__fadd_ru(zx0, e0), __fadd_ru(zx1, e1));
-    const uint32_t by = pack_bf16x2(__fsub_rd(zy0, e0), __fsub_rd(zy1, e1)) ^
-                        pack_bf16x2(__fadd_ru(zy0, e0), __fadd_ru(zy1, e1));
-    xo = pack_bf16x2(zx0, zx1);
-    yo = pack_bf16x2(zy0, zy1);
+    const uint64_t E = pair_of(__fmaf_ru(__fadd_ru(fabsf(x0), fabsf(y0)), k0, 0x1p-145f),
+                               __fmaf_ru(__fadd_ru(fabsf(x1), fabsf(y1)), k1, 0x1p-145f));
+    const uint32_t bx = pack_pair(sub2_rd(ZX, E)) ^ pack_pair(add2_ru(ZX, E));
+    const uint32_t by = pack_pair(sub2_rd(ZY, E)) ^ pack_pair(add2_ru(ZY, E));
+    xo = pack_pair(ZX);
+    yo = pack_pair(ZY);
     bad = bx | by;
 }
 
@@ -252,8 +288,8 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 
 constexpr int kStagesDefault = 3;                   // per warp
 constexpr uint32_t kItemBytes = 4096;               // one work item = one stage
-// (c1, c2, s1, s2) per frequency, then the first-level bound scale k per frequency
-constexpr size_t kTableBytes = (sizeof(float4) + sizeof(float)) * kMaxTablePairs;
+// (c1, c2, s1, s2) per frequency, then the first-level bound scale k, then -s32
+constexpr size_t kTableBytes = (sizeof(float4) + 2 * sizeof(float)) * kMaxTablePairs;
 // Dynamic shared memory of a CTA of kW warps: the warps' stages, then the (cos, sin) table.
 template <int kW, int kStages = kStagesDefault>
 constexpr size_t dyn_smem() { return (size_t)kW * kStages * kItemBytes + kTableBytes; }
@@ -434,7 +470,7 @@ __device__ __forceinline__ void copy_from_smem(const RenderParams &p, const Item
 // the same for every q, so its 8 (cos, sin) values are loaded once per item.
 template <bool kPaged>
 __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const float4 *tab,
-                                                 const float *kt, const Item &it,
+                                                 const float *kt, const float *nst, const Item &it,
                                                  const uint8_t *buf, int lane, int lane_v) {
     const int vecs_per_row = p.head_dim >> 3;
     const int half_vecs = p.head_dim >> 4;
@@ -458,12 +494,14 @@ __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const fl
         const uint4 b = src[off + half_vecs];
         const float4 ka = *reinterpret_cast<const float4 *>(kt + cs_index);
         const float4 kb = *reinterpret_cast<const float4 *>(kt + cs_index + 4);
+        const float4 na = *reinterpret_cast<const float4 *>(nst + cs_index);
+        const float4 nb = *reinterpret_cast<const float4 *>(nst + cs_index + 4);
         uint4 ao, bo;
         uint32_t b0, b1, b2, b3;
-        rotate_word(a.x, b.x, c[0], s[0], ka.x, c[1], s[1], ka.y, ao.x, bo.x, b0);
-        rotate_word(a.y, b.y, c[2], s[2], ka.z, c[3], s[3], ka.w, ao.y, bo.y, b1);
-        rotate_word(a.z, b.z, c[4], s[4], kb.x, c[5], s[5], kb.y, ao.z, bo.z, b2);
-        rotate_word(a.w, b.w, c[6], s[6], kb.z, c[7], s[7], kb.w, ao.w, bo.w, b3);
+        rotate_word(a.x, b.x, c[0], s[0], na.x, ka.x, c[1], s[1], na.y, ka.y, ao.x, bo.x, b0);
+        rotate_word(a.y, b.y, c[2], s[2], na.z, ka.z, c[3], s[3], na.w, ka.w, ao.y, bo.y, b1);
+        rotate_word(a.z, b.z, c[4], s[4], nb.x, kb.x, c[5], s[5], nb.y, kb.y, ao.z, bo.z, b2);
+        rotate_word(a.w, b.w, c[6], s[6], nb.z, kb.z, c[7], s[7], nb.w, kb.w, ao.w, bo.w, b3);
         if ((b0 | b1 | b2 | b3) != 0u) fixup_pair(p, tab, cs_index, a, b, b0, b1, b2, b3, ao, bo);
         uint4 *d = row_dst<kPaged>(p, it, row, pr) + lane_v;
         if (CM_IN_BOUNDS(d, 16, it.dst_base, it.dst_size)) st_stream(d, ao);
@@ -500,6 +538,7 @@ render_kernel(const __grid_constant__ RenderParams p) {
     __shared__ Item items[kW][kStages];
     float4 *tab = reinterpret_cast<float4 *>(smem + (size_t)kW * kStages * kItemBytes);
     float *kt = reinterpret_cast<float *>(tab + kMaxTablePairs);
+    float *nst = kt + kMaxTablePairs;
 
     const int half = p.head_dim >> 1;
     const int n_table = p.num_slots * half;
@@ -507,6 +546,7 @@ render_kernel(const __grid_constant__ RenderParams p) {
         const float2 cc = split16(p.cs[2 * i]), ss = split16(p.cs[2 * i + 1]);
         tab[i] = make_float4(cc.x, cc.y, ss.x, ss.y);
         kt[i] = bound_scale(__fadd_rn(cc.x, cc.y), __fadd_rn(ss.x, ss.y));
+        nst[i] = -__fadd_rn(ss.x, ss.y);
     }
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (lane == 0) {
@@ -550,7 +590,7 @@ render_kernel(const __grid_constant__ RenderParams p) {
         const Item it = items[warp][s];
         const uint8_t *buf = wbuf + (size_t)s * kItemBytes;
         if (it.rotate)
-            rotate_from_smem<kPaged>(p, tab, kt, it, buf, lane, lane_v);
+            rotate_from_smem<kPaged>(p, tab, kt, nst, it, buf, lane, lane_v);
         else
             copy_from_smem<kPaged>(p, it, buf, lane);
         __syncwarp();                          // every lane is done reading stage s
@@ -772,12 +812,14 @@ __global__ void __launch_bounds__(kRegThreads, kRegBlocksPerSm)
 render_reg_kernel(const __grid_constant__ RenderParams p) {
     __shared__ float4 tab[kMaxTablePairs];   // (c1, c2, s1, s2) for the second level
     __shared__ __align__(16) float kt[kMaxTablePairs];   // first-level bound scale per frequency
+    __shared__ __align__(16) float nst[kMaxTablePairs];  // -s32 per frequency
     const int half = p.head_dim >> 1;
     const int n_table = p.num_slots * half;
     for (int i = threadIdx.x; i < n_table; i += kRegThreads) {
         const float2 cc = split16(p.cs[2 * i]), ss = split16(p.cs[2 * i + 1]);
         tab[i] = make_float4(cc.x, cc.y, ss.x, ss.y);
         kt[i] = bound_scale(__fadd_rn(cc.x, cc.y), __fadd_rn(ss.x, ss.y));
+        nst[i] = -__fadd_rn(ss.x, ss.y);
     }
     __syncthreads();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -851,12 +893,14 @@ render_reg_kernel(const __grid_constant__ RenderParams p) {
                     const uint4 a = rk[2 * k], b = rk[2 * k + 1];
                     const float4 ka = *reinterpret_cast<const float4 *>(kt + cur + 8 * lane_v);
                     const float4 kb = *reinterpret_cast<const float4 *>(kt + cur + 8 * lane_v + 4);
+                    const float4 na = *reinterpret_cast<const float4 *>(nst + cur + 8 * lane_v);
+                    const float4 nb = *reinterpret_cast<const float4 *>(nst + cur + 8 * lane_v + 4);
                     uint4 ao, bo;
                     uint32_t b0, b1, b2, b3;
-                    rotate_word(a.x, b.x, c[0], s[0], ka.x, c[1], s[1], ka.y, ao.x, bo.x, b0);
-                    rotate_word(a.y, b.y, c[2], s[2], ka.z, c[3], s[3], ka.w, ao.y, bo.y, b1);
-                    rotate_word(a.z, b.z, c[4], s[4], kb.x, c[5], s[5], kb.y, ao.z, bo.z, b2);
-                    rotate_word(a.w, b.w, c[6], s[6], kb.z, c[7], s[7], kb.w, ao.w, bo.w, b3);
+                    rotate_word(a.x, b.x, c[0], s[0], na.x, ka.x, c[1], s[1], na.y, ka.y, ao.x, bo.x, b0);
+                    rotate_word(a.y, b.y, c[2], s[2], na.z, ka.z, c[3], s[3], na.w, ka.w, ao.y, bo.y, b1);
+                    rotate_word(a.z, b.z, c[4], s[4], nb.x, kb.x, c[5], s[5], nb.y, kb.y, ao.z, bo.z, b2);
+                    rotate_word(a.w, b.w, c[6], s[6], nb.z, kb.z, c[7], s[7], nb.w, kb.w, ao.w, bo.w, b3);
                     if ((b0 | b1 | b2 | b3) != 0u)
                         fixup_pair(p, tab, cur + 8 * lane_v, a, b, b0, b1, b2, b3, ao, bo);
                     uint4 *d = pair_row<kPaged>(p, ki, po, qq >> log2_hv) + lane_v;
