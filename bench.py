@@ -829,6 +829,71 @@ def small_merge_entry(cm, dev, name, merges=200):
             "render_bar_us": moved / (0.7 * NOMINAL_HBM_GBS * 1e9) * 1e6}
 
 
+def arity_entry(cm, dev, merges=50):
+    """The Qwen3-1.7B-shaped arity merge (5 distinct fragments, T ~ U{256..2048}, delivered
+    as 8 messages: the 5 and 3 byte-duplicates in buffers of their own, in seeded order):
+    replica A ingests the first half of the messages, replica B the rest, A := A u B,
+    render A, as one cm_ingest_render call (the duplicates make tail sums repeat, so the
+    call takes its one-after-the-other path) and as separate calls."""
+    import torch
+    import synthetic
+    w = synthetic.WORKLOADS["q17_arity"]
+    L, H, d = w.num_layers, w.num_kv_heads, w.head_dim
+    distinct = [synthetic.make_fragment_torch(s, L, H, d, dev) for s in synthetic.fragment_specs(w)]
+    schedule = synthetic.delivery_schedule(w)
+    seen, msgs = set(), []
+    for i in schedule:   # a repeated index is a byte copy in a buffer of its own
+        K, V = distinct[i]
+        msgs.append((K, V) if i not in seen else (K.clone(), V.clone()))
+        seen.add(i)
+    T = sum(K.shape[2] for K, _ in distinct)
+    k_out = torch.empty((L, H, T, d), dtype=torch.bfloat16, device=dev)
+    v_out = torch.empty_like(k_out)
+    ctx = cm.Context(dev.index or 0, synthetic.ROPE_THETA)
+    stream = torch.cuda.current_stream(dev)
+    fdesc = [cm.fragment_from_tensors(K, V) for K, V in msgs]
+
+    def timed(one):
+        for _ in range(5):
+            one()
+        torch.cuda.synchronize(dev)
+        cm.cm_context_kernel_times(ctx.handle, reset=True)
+        cm.cm_context_set_timing(ctx.handle, True)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(merges):
+            one()
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        cm.cm_context_set_timing(ctx.handle, False)
+        kt = cm.cm_context_kernel_times(ctx.handle, reset=True)
+        return e0.elapsed_time(e1) / merges, kt
+
+    ms, kt = timed(merge_fn(cm, ctx, fdesc, k_out, v_out, T, stream))
+    ms_seq, kt_seq = timed(merge_fn(cm, ctx, fdesc, k_out, v_out, T, stream, sequential=True))
+    S = cm.FragmentSet(ctx)
+    S.ingest_batch(distinct)
+    b2b, _ = grouped_ms(lambda: S.render(k_out, v_out, stream), stream, groups=10, per=10)
+    S.close()
+    ctx.close()
+    moved = 2 * T * w.bytes_per_token
+    return {"workload": "Qwen3-1.7B-shaped arity merge: 28 layers, 8 KV heads, head_dim 128, RoPE "
+                        "theta 1e6, 5 distinct fragments (T ~ U{256..2048}) delivered as 8 messages "
+                        "(3 byte-duplicates), bf16",
+            "value": 1000.0 / ms, "unit": UNIT, "ms_per_merge": ms, "merges": merges,
+            "messages": len(msgs), "distinct": len(distinct), "merged_tokens": T,
+            "hashed_gb_per_merge": sum(2 * K.numel() * 2 for K, _ in msgs) / 1e9,
+            "kernel_ms_per_merge": {"leaf_hash": kt["leaf_hash_ms"] / merges,
+                                    "inner_hash": kt["inner_hash_ms"] / merges,
+                                    "render": kt["render_ms"] / merges},
+            "sequential": {"value": 1000.0 / ms_seq, "ms_per_merge": ms_seq},
+            "render_us_in_step": 1000.0 * kt_seq["render_ms"] / merges,
+            "render_us_back_to_back": 1000.0 * b2b,
+            "render_gbs_back_to_back": moved / (b2b * 1e-3) / 1e9,
+            "render_bytes": moved,
+            "render_bar_us": moved / (0.7 * NOMINAL_HBM_GBS * 1e9) * 1e6}
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
@@ -1047,10 +1112,12 @@ def main():
     del dev_in, dev_desc, dev_out, host_in, host_out
 
     # the other workloads of the benchmark, measured on rank 0 of a single-GPU run: the
-    # Qwen3-1.7B-shaped 2 x 512-token merge, and the first 16 requests of the serving sweep
+    # Qwen3-1.7B-shaped 2 x 512-token merge, its arity merge (5 fragments in 8 messages), and
+    # the first 16 requests of the serving sweep
     extra = {}
     if rank == 0 and world == 1 and args.workload == WORKLOAD and not args.no_extra:
         extra["q17_n2"] = small_merge_entry(cm, dev, "q17_n2")
+        extra["q17_arity"] = arity_entry(cm, dev)
         wserve = synthetic.WORKLOADS["serve"]
         reqs = serve_requests(wserve, dev, 16)
         sctx = cm.Context(local_rank, synthetic.ROPE_THETA)

@@ -242,23 +242,26 @@ cm_status cm_render(const cm_set *set, void *k_out, void *v_out, int64_t capacit
  *     cm_render(target, k_out, v_out, capacity_tokens, stream, out_seq_len, out_order);
  * Overlap: the routing-layer norm keys (Eq. rho) of the deliveries are computed first
  * (one pass over K[l*], 1/(2L) of the bytes, and a synchronisation). Byte-identical
- * fragments have equal norm keys, so if the integer tail sums S of all fragments the
- * target will hold (its own, the other sets', every delivery) are pairwise distinct,
- * no delivery can be absorbed and the canonical order of Algorithm 1 does not depend on
- * the ids: the render starts at once on a stream of the context, with half-SM CTAs,
- * while the content address runs on `stream`. When the ids are known the set is
- * checked to be the one rendered (it always is unless two different fragments share
- * an address, which the paper's collision assumption excludes; then the target is
- * rendered again after the first render, so the result is still exact). With any tie
- * of S, with the re-delivery fast path on, or with an output the render would refuse,
- * the steps run one after the other.
+ * fragments have equal norm keys, so members of the prospective set (the target's
+ * fragments, the other sets', every delivery) whose integer tail sums S, lengths and
+ * per-token norm keys all agree are taken for one fragment; if the remaining S are
+ * pairwise distinct, the canonical order of Algorithm 1 does not depend on the ids: the
+ * render starts at once on a stream of the context, with narrow CTAs, while the content
+ * address runs on `stream`. When the ids are known the set is checked to hold exactly
+ * the fragments rendered, in that order (different fragments taken for one, or sharing
+ * an address, which the paper's collision assumption excludes, fail the check; then the
+ * target is rendered again after the first render, so the result is still exact). With
+ * a tie of S between members that differ in length or norm keys, with the re-delivery
+ * fast path on, or with an output the render would refuse, the steps run one after the
+ * other.
  *   sets, frags      HOST arrays of n (n >= 0): delivery i goes into sets[i]; all sets
  *                    and target from one context (CM_ERR_INVALID_ARG)
  *   target           the set rendered (it may appear in sets or not)
  *   k_out, v_out, capacity_tokens   as in cm_render
  *   out_ids, out_absorbed           nullable HOST arrays of n, as in cm_ingest_many
  *   out_seq_len, out_order          nullable, as in cm_render (out_order: the target's size)
- *   out_overlapped   nullable: 1 if the render ran beside the content address, else 0
+ *   out_overlapped   nullable: 1 if the render that ran beside the content address
+ *                    stood, else 0
  * The target, every other set named and every delivery must share one (L, H, d)
  * (empty sets excepted): CM_ERR_SHAPE_MISMATCH before any work otherwise. The call
  * returns after the ids reached the host; the render is then still running, ordered

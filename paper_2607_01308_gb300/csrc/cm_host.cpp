@@ -1516,33 +1516,49 @@ cm_status ingest_render_impl(cm_set *const *sets, const cm_fragment *frags, int3
     }
 
     // the prospective set: the records of the target and of the sources (one per id),
-    // then every delivery; distinct tail sums decide its order
+    // then every delivery; distinct tail sums decide its order. Members with equal sums,
+    // lengths and norm keys are taken for one fragment (byte-identical fragments always
+    // agree so; a duplicate delivery is absorbed): the render uses the first of them, whose
+    // bytes then equal those of whichever copy the set keeps. Equal sums with different
+    // lengths or norm keys are a tie only the ids can break.
     bool spec = true;
     std::vector<Slot> spec_slots;
+    struct Member {
+        const void *k, *v;
+        int64_t T;
+        unsigned __int128 S;
+        const std::vector<uint64_t> *Q;
+        bool has_id;       // a record: its id; a delivery: known once hashed
+        IdKey id;
+        size_t delivery;
+    };
+    std::vector<Member> spec_members;
     {
         std::map<IdKey, std::shared_ptr<const Record>> have(target->items.begin(), target->items.end());
         for (const cm_set *src : sources) have.insert(src->items.begin(), src->items.end());
         int64_t t_star = INT64_MAX;
         for (const auto &kv : have) t_star = std::min<int64_t>(t_star, kv.second->T);
         for (const cm_fragment *f : fp) t_star = std::min<int64_t>(t_star, f->seq_len);
-        struct Member {
-            const void *k, *v;
-            int64_t T;
-            unsigned __int128 S;
-        };
         std::vector<Member> m;
         for (const auto &kv : have) {
             const Record &r = *kv.second;
-            m.push_back({r.k, r.v, r.T, tail_sum(r.Q, r.T, r.H, t_star)});
+            m.push_back({r.k, r.v, r.T, tail_sum(r.Q, r.T, r.H, t_star), &r.Q, true, kv.first, 0});
         }
         for (size_t i = 0; i < fp.size(); ++i)
             m.push_back({fp[i]->k, fp[i]->v, fp[i]->seq_len,
-                         tail_sum(Qd[i], fp[i]->seq_len, fp[i]->num_kv_heads, t_star)});
-        std::sort(m.begin(), m.end(), [](const Member &a, const Member &b) { return a.S > b.S; });
+                         tail_sum(Qd[i], fp[i]->seq_len, fp[i]->num_kv_heads, t_star), &Qd[i], false,
+                         IdKey{}, i});
+        // records first, then deliveries in order, within equal sums
+        std::stable_sort(m.begin(), m.end(), [](const Member &a, const Member &b) { return a.S > b.S; });
         int64_t total = 0;
-        for (size_t i = 0; i < m.size(); ++i) {
-            if (i + 1 < m.size() && m[i].S == m[i + 1].S) spec = false;
-            total += m[i].T;
+        for (const Member &x : m) {
+            if (!spec_members.empty() && spec_members.back().S == x.S) {
+                const Member &y = spec_members.back();
+                if (y.T == x.T && *y.Q == *x.Q) continue;   // taken for the same fragment
+                spec = false;
+            }
+            spec_members.push_back(x);
+            total += x.T;
         }
         // an output the render would refuse: no speculation (the call then fails as
         // cm_render does, after the ingest); a small merge: the render follows the hash
@@ -1550,7 +1566,7 @@ cm_status ingest_render_impl(cm_set *const *sets, const cm_fragment *frags, int3
             spec = false;
         if (spec) {
             int64_t s = 0;
-            for (const Member &x : m) {
+            for (const Member &x : spec_members) {
                 spec_slots.push_back({x.k, x.v, x.T, s, k_out, v_out, capacity});
                 s += x.T;
             }
@@ -1580,10 +1596,13 @@ cm_status ingest_render_impl(cm_set *const *sets, const cm_fragment *frags, int3
     if (out_seq_len) *out_seq_len = total;
     if (out_order)
         for (size_t i = 0; i < order.size(); ++i) out_order[i] = order[i]->id;
-    bool kept = spec && slots.size() == spec_slots.size();
-    for (size_t i = 0; kept && i < slots.size(); ++i)
-        kept = slots[i].k == spec_slots[i].k && slots[i].v == spec_slots[i].v &&
-               slots[i].T == spec_slots[i].T && slots[i].offset == spec_slots[i].offset;
+    // the render stands if the set holds exactly the members assumed, in the same order:
+    // the same ids (so the same bytes, rendered from whichever copy) and lengths
+    bool kept = spec && order.size() == spec_members.size();
+    for (size_t i = 0; kept && i < order.size(); ++i) {
+        const Member &x = spec_members[i];
+        kept = key_of(order[i]->id) == (x.has_id ? x.id : key_of(ids[x.delivery])) && order[i]->T == x.T;
+    }
     // no speculation, or not the set that resulted: render now, after anything before
     if (!kept && !slots.empty()) st = launch_slots(ctx, slots, target->L, target->H, target->d, ctx->side);
     st = join(st);

@@ -5,9 +5,11 @@ the canonical order (Algorithm 1) on their own.
 Every case is compared with the CPU oracle (ids, absorption flags, order and V
 bit-exact, K within 1 ulp with 0 non-exact elements) and with the same sequence of
 separate calls (cm_ingest_many, cm_union, cm_render) on the library, byte for byte;
-the overlapped flag says which path ran: the speculative one for distinct sums, the
-sequential one for an exact tie of the sums, a duplicate delivery, the re-delivery
-fast path and an output the render refuses.
+the overlapped flag says whether the render started beside the content address stood:
+it does for distinct sums and for duplicate deliveries (equal sums, lengths and norm keys
+are taken for one fragment, which the ids then confirm); it does not for an exact tie
+of the sums between different fragments (the speculative render is replaced once the
+ids are known), the re-delivery fast path and an output the render refuses.
 """
 import numpy as np
 import pytest
@@ -109,12 +111,13 @@ def test_prior_records_and_other_replicas_join_the_speculation(ctx):
     # C receives two deliveries, A one, B one; the target is A
     sets = [C, A, B, C]
     out, (res, n, order, overlapped) = _fused(ctx, sets, frags[3:] + frags[:1], A, 400)
-    # the last delivery repeats A's record: equal sums, so the steps ran in sequence
-    assert not overlapped
+    # the last delivery repeats A's record: equal sums, lengths and norm keys, taken for
+    # the same fragment, which the ids confirm (A keeps its record)
+    assert overlapped
     assert [a for _, a in res] == [False, False, False, False]   # C did not hold it
     assert order == _check(out, n, frags)
     out, (res, n, order, overlapped) = _fused(ctx, [C], frags[3:4], A, 400)
-    assert not overlapped and res[0][1]                          # absorbed by C
+    assert overlapped and res[0][1]                              # absorbed by C
     assert order == _check(out, n, frags)
     for s in (A, B, C):
         s.close()
@@ -131,25 +134,45 @@ def test_prior_records_and_other_replicas_join_the_speculation(ctx):
 
 
 def test_exact_tie_of_the_sums_runs_after_the_ids(ctx):
-    # equal K (so equal norm keys and equal sums), different V: the order needs the ids
+    # equal K (so equal norm keys and equal sums), different V: taken for one fragment by
+    # the speculation, which the ids refute; the order needs the ids, and the target is
+    # rendered again after the speculative render
     (K0, V0), (_, V1), (K2, V2) = _fragments(13, [40, 40, 47])
     frags = [(K0, V0), (K0.clone(), V1), (K2, V2)]
     A = cm.FragmentSet(ctx)
     out, (res, n, order, overlapped) = _fused(ctx, [A, A, A], frags, A, 200)
     assert not overlapped
+    assert [a for _, a in res] == [False, False, False]
     assert order == _check(out, n, frags)
-    A.close()
+    # the same with the tie across two replicas and a byte copy of the third fragment
+    B, A2 = cm.FragmentSet(ctx), cm.FragmentSet(ctx)
+    out, (res, n, order, overlapped) = _fused(ctx, [A2, B, B, A2],
+                                              frags + [(K2.clone(), V2.clone())], A2, 200)
+    assert not overlapped
+    assert [a for _, a in res] == [False, False, False, False]   # the copy went to A2
+    assert order == _check(out, n, frags)
+    for s in (A, B, A2):
+        s.close()
 
 
 def test_duplicate_delivery_is_absorbed(ctx):
     frags = _fragments(14, [33, 66, 99])
     deliveries = frags + [(frags[1][0].clone(), frags[1][1].clone())]
     A, B = cm.FragmentSet(ctx), cm.FragmentSet(ctx)
-    # the copy of fragment 1 goes to the replica that already received it
+    # the copy of fragment 1 goes to the replica that already received it: the copy is
+    # taken for the same fragment, the render overlaps and stands
     out, (res, n, order, overlapped) = _fused(ctx, [A, B, A, B], deliveries, A, 300)
-    assert not overlapped
+    assert overlapped
     assert [a for _, a in res] == [False, False, False, True]
     assert order == _check(out, n, frags)
+    # byte-equal to the separate calls
+    A2, B2 = cm.FragmentSet(ctx), cm.FragmentSet(ctx)
+    out2, res2, n2, order2 = _sequence(ctx, [A2, B2, A2, B2], deliveries, A2, 300)
+    assert res2 == res and n2 == n and order2 == order
+    assert torch.equal(out[0].view(torch.int16), out2[0].view(torch.int16))
+    assert torch.equal(out[1].view(torch.int16), out2[1].view(torch.int16))
+    A2.close()
+    B2.close()
     A.close()
     B.close()
 
