@@ -225,6 +225,42 @@ def test_arity_batch_matches_sequential_ingest_and_oracle(ctx):
     S2.close()
 
 
+def test_arity_fused_with_duplicates_matches_the_oracle(ctx):
+    # the arity merge through cm_ingest_render: 8 messages (3 byte-duplicates, in buffers
+    # of their own) into two replicas; the duplicates are taken for their originals, the
+    # render overlaps the content address and stands; every plane against the oracle
+    w = synthetic.WORKLOADS["q17_arity"]
+    specs = synthetic.fragment_specs(w)
+    frags = [synthetic.make_fragment_torch(sp, w.num_layers, w.num_kv_heads, w.head_dim, "cuda:0")
+             for sp in specs]
+    sched = synthetic.delivery_schedule(w)
+    seen, msgs = set(), []
+    for i in sched:
+        msgs.append(frags[i] if i not in seen else (frags[i][0].clone(), frags[i][1].clone()))
+        seen.add(i)
+    A, B = cm.FragmentSet(ctx), cm.FragmentSet(ctx)
+    half = len(msgs) // 2
+    total = sum(sp.seq_len for sp in specs)
+    k_out, v_out = empty_out(w.num_layers, w.num_kv_heads, total, w.head_dim)
+    res, n, order_ids, overlapped = cm.cm_ingest_render(
+        [A.handle] * half + [B.handle] * (len(msgs) - half),
+        [cm.fragment_from_tensors(K, V) for K, V in msgs], A.handle, k_out.data_ptr(),
+        v_out.data_ptr(), total)
+    torch.cuda.synchronize()
+    assert overlapped and n == total and len(A) == 5
+    keys = _oracle_keys(frags, w.num_layers // 2)
+    assert [r[0] for r in res] == [keys[i][0] for i in sched]
+    # absorbed: an earlier message of the same fragment went to the same replica
+    dest = [0] * half + [1] * (len(msgs) - half)
+    assert [r[1] for r in res] == [any(sched[j] == sched[i] and dest[j] == dest[i] for j in range(i))
+                                   for i in range(len(msgs))]
+    order = _oracle_order(keys, [sp.seq_len for sp in specs])
+    assert order_ids == [keys[i][0] for i in order]
+    _check_all_planes(frags, order, k_out, v_out)
+    A.close()
+    B.close()
+
+
 def test_arity_all_120_orders_render_identically_at_full_length(ctx):
     # the arity configuration at its real lengths (T ~ U{256..2048}): every order of the
     # five distinct fragments, as unions of single-fragment sets, renders the same bytes;
