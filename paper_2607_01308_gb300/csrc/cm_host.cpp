@@ -1387,13 +1387,14 @@ cm_status ensure_side_stream(cm_context *ctx) {
 
 // cm_ingest_render (see include/cm.h). The norm keys of the deliveries are computed on
 // the context's side stream while the content address runs on `stream`. Equal bytes give
-// equal norm keys, so when the integer tail sums S (Eq. rho) of the prospective set's
-// members are pairwise distinct, no delivery can be absorbed and no two members can tie,
-// and the canonical order of Algorithm 1 is decided before any id is known: the render
-// then starts on the side stream (half-SM CTAs) beside the rest of the content address.
-// Once the ids are known the insertions and unions are made as usual; if the set that
-// results is not the one the render assumed (only a collision of the address, which the
-// paper excludes, could do that), it is rendered again after the first render.
+// equal norm keys, so members of the prospective set whose integer tail sums S (Eq. rho),
+// lengths and norm keys agree are taken for one fragment, and when the remaining S are
+// pairwise distinct the canonical order of Algorithm 1 is decided before any id is known:
+// the render then starts on the side stream (narrow CTAs) beside the rest of the content
+// address. Once the ids are known the insertions and unions are made as usual; if the set
+// that results does not hold exactly the fragments the render assumed, in that order
+// (different fragments taken for one, or an address collision, which the paper excludes),
+// it is rendered again after the first render.
 cm_status ingest_render_impl(cm_set *const *sets, const cm_fragment *frags, int32_t n,
                              cm_set *target, void *k_out, void *v_out, int64_t capacity,
                              cm_stream_t stream, cm_id *out_ids, int32_t *out_absorbed,
