@@ -689,6 +689,67 @@ def test_rotation_stress_random_bit_patterns(theta):
     c.close()
 
 
+def _midpoint_distance_ulps(z):
+    """Distance of fp64 values z (normal range) to the nearest bf16 rounding midpoint, in
+    fp32 ulps of z."""
+    _, e = np.frexp(z)                          # z = m 2^e, 0.5 <= |m| < 1
+    q = np.ldexp(1.0, e - 8)                    # the bf16 quantum of that binade
+    m = (np.floor(z / q) + 0.5) * q
+    return np.abs(z - m) / np.ldexp(1.0, e - 24)
+
+
+@pytest.mark.parametrize("theta", [1.0e4, 1.0e6])
+def test_rotation_near_rounding_midpoints(theta):
+    # keys chosen so that their rotated values lie within a few fp32 ulps of a bf16
+    # rounding midpoint, where the fp32 first level cannot certify them: the second level
+    # and the fp64 level decide; the render must still equal the oracle bit for bit
+    from oracle.bf16 import bits_to_f64
+    from oracle.merge import delta_cos_sin
+    c = cm.Context(0, theta)
+    L, H, d, T = 1, 2, 128, 16
+    half = d // 2
+    rng = np.random.default_rng(int(theta) % 997)
+
+    def rand_bf16(n):
+        e = rng.integers(118, 134, size=n)
+        return ((rng.integers(0, 2, size=n) << 15) | (e << 7) | rng.integers(0, 128, size=n)).astype(np.uint16)
+
+    frags, bits_list, near = [], [], []
+    for p, s in enumerate([0, T, 2 * T, 3 * T]):
+        bits = np.empty((L, H, T, d), dtype=np.uint16)
+        cs, sn = delta_cos_sin(s, d, theta)
+        for j in range(half):
+            # the H T pairs (x, y) of frequency j closest to a midpoint, out of 512 x 512
+            xs, ys = rand_bf16(512), rand_bf16(512)
+            if s == 0:
+                ix, iy = rng.integers(0, 512, size=H * T), rng.integers(0, 512, size=H * T)
+            else:
+                x, y = bits_to_f64(xs)[:, None], bits_to_f64(ys)[None, :]
+                dist = np.minimum(_midpoint_distance_ulps(x * cs[j] - y * sn[j]),
+                                  _midpoint_distance_ulps(y * cs[j] + x * sn[j]))
+                best = np.argsort(dist, axis=None)[:H * T]
+                ix, iy = np.unravel_index(best, dist.shape)
+                near.append(np.median(dist.ravel()[best]))
+            bits[0, :, :, j] = xs[ix].reshape(H, T)
+            bits[0, :, :, j + half] = ys[iy].reshape(H, T)
+        K = torch.from_numpy(bits.view(np.int16)).to("cuda:0").view(torch.bfloat16).contiguous()
+        V = torch.from_numpy(rng.integers(0, 1 << 15, size=bits.shape).astype(np.int16)).to(
+            "cuda:0").view(torch.bfloat16).contiguous()
+        frags.append((K, V))
+        bits_list.append(bits)
+    assert np.median(near) < 4.0          # the construction does land near the midpoints
+    total = 4 * T
+    k_out, v_out = empty_out(L, H, total, d)
+    assert c.bagmerge(frags, k_out, v_out) == total
+    torch.cuda.synchronize()
+    kb = synthetic.to_bits(k_out)
+    for p, bits in enumerate(bits_list):
+        s = p * T
+        want = oracle.rotate_k(bits, s, theta)
+        assert assert_k_parity(kb[:, :, s:s + T], want, f"slot@{s}") == 0
+    c.close()
+
+
 # ---------------------------------------------------------------- concurrent use of one context
 
 def test_two_threads_share_a_context(ctx):
