@@ -101,7 +101,7 @@ __device__ __forceinline__ float bound_scale(float c32, float s32) {
 
 // Paired fp32 arithmetic (sm_100 and later): two fp32 operations, elementwise, in one
 // instruction on a register pair; the rounding of each half is that of the scalar op.
-__device__ __forceinline__ uint64_t pair_of(float lo, float hi) {
+__device__ __forceinline__ uint64_t f32x2_of(float lo, float hi) {
     uint64_t r;
     asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
     return r;
@@ -146,11 +146,11 @@ __device__ __forceinline__ void rotate_word(uint32_t xw, uint32_t yw, float c0, 
                                             float k1, uint32_t &xo, uint32_t &yo, uint32_t &bad) {
     const float x0 = bf16_lo(xw), x1 = bf16_hi(xw);
     const float y0 = bf16_lo(yw), y1 = bf16_hi(yw);
-    const uint64_t X = pair_of(x0, x1), Y = pair_of(y0, y1), C = pair_of(c0, c1);
-    const uint64_t ZX = fma2_rn(X, C, mul2_rn(Y, pair_of(ns0, ns1)));
-    const uint64_t ZY = fma2_rn(Y, C, mul2_rn(X, pair_of(s0, s1)));
+    const uint64_t X = f32x2_of(x0, x1), Y = f32x2_of(y0, y1), C = f32x2_of(c0, c1);
+    const uint64_t ZX = fma2_rn(X, C, mul2_rn(Y, f32x2_of(ns0, ns1)));
+    const uint64_t ZY = fma2_rn(Y, C, mul2_rn(X, f32x2_of(s0, s1)));
     // one bound for both outputs of a pair: E = k (|x| + |y|) + 2^-145, rounded up
-    const uint64_t E = pair_of(__fmaf_ru(__fadd_ru(fabsf(x0), fabsf(y0)), k0, 0x1p-145f),
+    const uint64_t E = f32x2_of(__fmaf_ru(__fadd_ru(fabsf(x0), fabsf(y0)), k0, 0x1p-145f),
                                __fmaf_ru(__fadd_ru(fabsf(x1), fabsf(y1)), k1, 0x1p-145f));
     const uint32_t bx = pack_pair(sub2_rd(ZX, E)) ^ pack_pair(add2_ru(ZX, E));
     const uint32_t by = pack_pair(sub2_rd(ZY, E)) ^ pack_pair(add2_ru(ZY, E));
