@@ -773,6 +773,26 @@ def merge_fn(cm, ctx, fdesc, k_out, v_out, total_T, stream, sequential=False):
     return one_merge if sequential else fused
 
 
+def timed_merges(cm, ctx, one, merges, dev, stream, warm):
+    """Mean device time of `merges` calls of `one` back to back (CUDA events on `stream`,
+    after `warm` untimed calls) and the library's kernel times over them."""
+    import torch
+    for _ in range(warm):
+        one()
+    torch.cuda.synchronize(dev)
+    cm.cm_context_kernel_times(ctx.handle, reset=True)
+    cm.cm_context_set_timing(ctx.handle, True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(merges):
+        one()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    cm.cm_context_set_timing(ctx.handle, False)
+    kt = cm.cm_context_kernel_times(ctx.handle, reset=True)
+    return e0.elapsed_time(e1) / merges, kt
+
+
 def small_merge_entry(cm, dev, name, merges=200):
     """A whole-merge measurement of a small workload (the headline step, cm_ingest_render),
     beside the same merges as separate calls, with the render's in-step (separate calls)
@@ -789,22 +809,7 @@ def small_merge_entry(cm, dev, name, merges=200):
     stream = torch.cuda.current_stream(dev)
     fdesc = [cm.fragment_from_tensors(K, V) for K, V in frags]
 
-    def timed(one):
-        for _ in range(10):
-            one()
-        torch.cuda.synchronize(dev)
-        cm.cm_context_kernel_times(ctx.handle, reset=True)
-        cm.cm_context_set_timing(ctx.handle, True)
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        for _ in range(merges):
-            one()
-        e1.record(stream)
-        torch.cuda.synchronize(dev)
-        cm.cm_context_set_timing(ctx.handle, False)
-        kt = cm.cm_context_kernel_times(ctx.handle, reset=True)
-        return e0.elapsed_time(e1) / merges, kt
-
+    timed = lambda one: timed_merges(cm, ctx, one, merges, dev, stream, warm=10)
     ms, kt = timed(merge_fn(cm, ctx, fdesc, k_out, v_out, T, stream))
     ms_seq, kt_seq = timed(merge_fn(cm, ctx, fdesc, k_out, v_out, T, stream, sequential=True))
     S = cm.FragmentSet(ctx)
@@ -853,22 +858,7 @@ def arity_entry(cm, dev, merges=50):
     stream = torch.cuda.current_stream(dev)
     fdesc = [cm.fragment_from_tensors(K, V) for K, V in msgs]
 
-    def timed(one):
-        for _ in range(5):
-            one()
-        torch.cuda.synchronize(dev)
-        cm.cm_context_kernel_times(ctx.handle, reset=True)
-        cm.cm_context_set_timing(ctx.handle, True)
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        for _ in range(merges):
-            one()
-        e1.record(stream)
-        torch.cuda.synchronize(dev)
-        cm.cm_context_set_timing(ctx.handle, False)
-        kt = cm.cm_context_kernel_times(ctx.handle, reset=True)
-        return e0.elapsed_time(e1) / merges, kt
-
+    timed = lambda one: timed_merges(cm, ctx, one, merges, dev, stream, warm=5)
     ms, kt = timed(merge_fn(cm, ctx, fdesc, k_out, v_out, T, stream))
     ms_seq, kt_seq = timed(merge_fn(cm, ctx, fdesc, k_out, v_out, T, stream, sequential=True))
     S = cm.FragmentSet(ctx)
