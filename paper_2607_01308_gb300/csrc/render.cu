@@ -140,7 +140,9 @@ __device__ __forceinline__ uint32_t pack_pair(uint64_t v) {
 // (frequency of pair e: c_e, s_e, ns_e = -s_e and bound scale k_e), the two pairs of a
 // word in paired instructions: x' = fma(x, c, fl(y ns)), y' = fma(y, c, fl(x s)), the
 // scalar operations of the bound's proof. Returns the rotated words and a mask whose
-// nonzero 16-bit halves mark elements whose fp32 result is not certified.
+// nonzero 16-bit halves mark elements whose fp32 result is not certified. A certified
+// half's z - E, z and z + E round to the same bf16 (rounding is monotone), so the
+// rounding of z + E is the output there; uncertified halves are replaced by the fix-up.
 __device__ __forceinline__ void rotate_word(uint32_t xw, uint32_t yw, float c0, float s0,
                                             float ns0, float k0, float c1, float s1, float ns1,
                                             float k1, uint32_t &xo, uint32_t &yo, uint32_t &bad) {
@@ -152,11 +154,9 @@ __device__ __forceinline__ void rotate_word(uint32_t xw, uint32_t yw, float c0, 
     // one bound for both outputs of a pair: E = k (|x| + |y|) + 2^-145, rounded up
     const uint64_t E = f32x2_of(__fmaf_ru(__fadd_ru(fabsf(x0), fabsf(y0)), k0, 0x1p-145f),
                                __fmaf_ru(__fadd_ru(fabsf(x1), fabsf(y1)), k1, 0x1p-145f));
-    const uint32_t bx = pack_pair(sub2_rd(ZX, E)) ^ pack_pair(add2_ru(ZX, E));
-    const uint32_t by = pack_pair(sub2_rd(ZY, E)) ^ pack_pair(add2_ru(ZY, E));
-    xo = pack_pair(ZX);
-    yo = pack_pair(ZY);
-    bad = bx | by;
+    xo = pack_pair(add2_ru(ZX, E));
+    yo = pack_pair(add2_ru(ZY, E));
+    bad = (pack_pair(sub2_rd(ZX, E)) ^ xo) | (pack_pair(sub2_rd(ZY, E)) ^ yo);
 }
 
 // Second level for one element pair (x, y) whose first-level result was not
@@ -310,53 +310,6 @@ struct Item {
     uint64_t dst_size;         // library is not told: only the lower end is checked)
 #endif
 };
-
-// Item g: pair g / 2 of its slot (row chunk c of (layer, head) plane lh), K if g is
-// even, V if odd.
-__device__ __forceinline__ Item item_of(const RenderParams &p, uint32_t g) {
-    int si = 0;
-    while (si + 1 < p.num_slots && g >= p.slot[si + 1].chunk_begin) ++si;
-    const RenderSlot &S = p.slot[si];
-    const uint32_t local = g - S.chunk_begin;
-    const bool is_v = (local & 1u) != 0;             // K and V items alternate
-    const uint32_t pair = local >> 1;
-    const uint32_t lhp = pair / S.chunks_per_plane;
-    const uint32_t c = pair - lhp * S.chunks_per_plane;
-    const int64_t lh = lhp;
-    const int64_t row0 = (int64_t)c * p.rows_per_chunk;
-    const int64_t left = S.seq_len - row0;
-    const int rows = left < p.rows_per_chunk ? (int)left : p.rows_per_chunk;
-    const int64_t row_bytes = (int64_t)p.head_dim * 2;
-    Item it;
-    it.src = static_cast<const uint8_t *>(is_v ? S.v : S.k) + (lh * S.seq_len + row0) * row_bytes;
-    if (p.paged) {
-        const uint32_t l32 = lhp / (uint32_t)p.num_heads;      // 32-bit: lhp < 2^32
-        const int64_t l = l32, h = (int64_t)(lhp - l32 * (uint32_t)p.num_heads);
-        it.dst = static_cast<uint8_t *>(is_v ? p.v_pool : p.k_pool) +
-                 (l * p.stride_layer + h * p.stride_head) * 2;
-    } else {
-        it.dst = static_cast<uint8_t *>(is_v ? S.v_out : S.k_out) +
-                 (lh * S.capacity + S.offset + row0) * row_bytes;
-    }
-    it.pos0 = S.offset + row0;
-    it.bytes = (uint32_t)(rows * row_bytes);
-    it.rows = rows;
-    it.rotate = (!is_v && S.rotate) ? 1 : 0;
-    it.cs_index = S.table_base;
-#ifdef CM_DEBUG_BOUNDS
-    const uint64_t lh_planes = (uint64_t)p.num_layers * (uint64_t)p.num_heads;
-    it.src_base = static_cast<const uint8_t *>(is_v ? S.v : S.k);
-    it.src_size = (uint64_t)lh_planes * (uint64_t)S.seq_len * (uint64_t)row_bytes;
-    if (p.paged) {
-        it.dst_base = static_cast<const uint8_t *>(is_v ? p.v_pool : p.k_pool);
-        it.dst_size = ~0ull - reinterpret_cast<uint64_t>(it.dst_base);
-    } else {
-        it.dst_base = static_cast<const uint8_t *>(is_v ? S.v_out : S.k_out);
-        it.dst_size = (uint64_t)lh_planes * (uint64_t)S.capacity * (uint64_t)row_bytes;
-    }
-#endif
-    return it;
-}
 
 // Physical block of logical block b of a paged output (in bounds-checked builds: an index
 // outside the table or a negative entry counts a violation and reads as block 0).
@@ -516,110 +469,6 @@ __device__ __forceinline__ float2 split16(double c) {
     return make_float2(c1, __double2float_rn(c - (double)c1));
 }
 
-// Half-SM render: a persistent kernel with one CTA of kW = 8 warps per SM (half of the
-// register file, leaving room for kernels of other streams on the same SMs); every
-// warp runs its own
-// pipeline over its own items, with no block-wide barrier after set-up. Items come
-// in (K, V) pairs of the same (slot, layer, head, row chunk); a warp takes pairs
-// warp id + m * total warps and does the K item, then the V item, so rotation work
-// and pure copies alternate within every warp. Lane 0 keeps up to kStages items in
-// flight as 1-D TMA bulk loads into the warp's stages (completion on one mbarrier
-// per stage); all lanes wait for an item, move it from shared memory to its place
-// in the output (rotating K rows of slots at a nonzero offset; kPaged: each row's
-// place comes from the block table), and lane 0 refills the stage with the warp's
-// next item. Every wait is bounded: on timeout the warp records an error, waits
-// (bounded) for its own copies in flight and returns.
-template <bool kPaged, int kW, int kStages = kStagesDefault, int kMinBlocks = 16 / kW>
-__global__ void __launch_bounds__(kW * 32, kMinBlocks)
-render_kernel(const __grid_constant__ RenderParams p) {
-    constexpr int kThreads = kW * 32;
-    extern __shared__ __align__(128) uint8_t smem[];
-    __shared__ __align__(8) uint64_t full[kW][kStages];
-    __shared__ Item items[kW][kStages];
-    float4 *tab = reinterpret_cast<float4 *>(smem + (size_t)kW * kStages * kItemBytes);
-    float *kt = reinterpret_cast<float *>(tab + kMaxTablePairs);
-    float *nst = kt + kMaxTablePairs;
-
-    const int half = p.head_dim >> 1;
-    const int n_table = p.num_slots * half;
-    for (int i = threadIdx.x; i < n_table; i += kThreads) {
-        const float2 cc = split16(p.cs[2 * i]), ss = split16(p.cs[2 * i + 1]);
-        tab[i] = make_float4(cc.x, cc.y, ss.x, ss.y);
-        kt[i] = bound_scale(__fadd_rn(cc.x, cc.y), __fadd_rn(ss.x, ss.y));
-        nst[i] = -__fadd_rn(ss.x, ss.y);
-    }
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (lane == 0) {
-        for (int s = 0; s < kStages; ++s) mbar_init(&full[warp][s], 1);
-        fence_mbar_init();
-    }
-    __syncthreads();
-
-    const uint32_t first = blockIdx.x * kW + warp;
-    const uint32_t stride = gridDim.x * kW;
-    const uint32_t npairs = p.total_chunks / 2;
-    const uint32_t n = npairs > first ? 2 * ((npairs - first + stride - 1) / stride) : 0;
-    const int lane_v = lane & ((p.head_dim >> 4) - 1);
-    uint8_t *wbuf = smem + (size_t)warp * kStages * kItemBytes;
-
-    auto produce = [&](uint32_t j) {
-        const uint32_t s = j % kStages;
-        const Item it = item_of(p, 2 * (first + (j >> 1) * stride) + (j & 1));
-        items[warp][s] = it;
-        // bounds-checked builds: a source outside the slot's fragment is not copied (the
-        // stage keeps stale bytes, the barrier completes without them)
-        const bool src_ok = CM_IN_BOUNDS(it.src, it.bytes, it.src_base, it.src_size);
-        mbar_arrive_expect_tx(&full[warp][s], src_ok ? it.bytes : 0u);
-        if (j == 0 && p.withhold_warp == first + 1) return;   // injected: the wait runs out
-        if (src_ok) bulk_load(wbuf + (size_t)s * kItemBytes, it.src, it.bytes, &full[warp][s]);
-    };
-
-    uint32_t produced = 0;
-    if (lane == 0)
-        for (; produced < n && produced < (uint32_t)kStages; ++produced) produce(produced);
-
-    uint32_t i = 0;
-    bool aborted = false;
-    for (; i < n; ++i) {
-        const uint32_t s = i % kStages;
-        const bool ok = mbar_wait(&full[warp][s], (i / kStages) & 1u);
-        if (__any_sync(0xFFFFFFFFu, !ok)) {
-            aborted = true;
-            break;
-        }
-        const Item it = items[warp][s];
-        const uint8_t *buf = wbuf + (size_t)s * kItemBytes;
-        if (it.rotate)
-            rotate_from_smem<kPaged>(p, tab, kt, nst, it, buf, lane, lane_v);
-        else
-            copy_from_smem<kPaged>(p, it, buf, lane);
-        __syncwarp();                          // every lane is done reading stage s
-        if (lane == 0 && produced < n) {
-            fence_proxy_async_smem();
-            produce(produced++);               // item i + kStages into stage s
-        }
-    }
-    if (aborted && lane == 0) {
-        atomicOr(p.error, 1u);
-        for (uint32_t j = i; j < produced; ++j)
-            mbar_wait(&full[warp][j % kStages], (j / kStages) & 1u);
-    }
-}
-
-template <bool kPaged, int kW, int kStages = kStagesDefault, int kMinBlocks = 16 / kW>
-cudaError_t set_smem_attribute() {
-    return cudaFuncSetAttribute(render_kernel<kPaged, kW, kStages, kMinBlocks>,
-                                cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)dyn_smem<kW, kStages>());
-}
-
-// ---------------------------------------------------------------- full-SM render
-
-constexpr int kRegThreads = 256;           // 8 warps per CTA
-constexpr int kRegBlocksPerSm = 3;         // 24 warps per SM
-constexpr uint32_t kRegItemBytes = 1024;   // one work item: 2 vectors per lane
-constexpr int kRegVecs = kRegItemBytes / 16 / 32;
-
 // A (K, V) item pair: the same rows of one (slot, layer, head) plane of K and of V.
 struct Pair {
     const uint8_t *ks, *vs;   // sources
@@ -749,6 +598,140 @@ __device__ __forceinline__ Item half_item(const Pair &q, bool v) {
 #endif
     return it;
 }
+
+// Half-SM render: a persistent kernel with one CTA of kW = 8 warps per SM (half of the
+// register file, leaving room for kernels of other streams on the same SMs); every
+// warp runs its own
+// pipeline over its own items, with no block-wide barrier after set-up. Items come
+// in (K, V) pairs of the same (slot, layer, head, row chunk); a warp takes pairs
+// warp id + m * total warps and does the K item, then the V item, so rotation work
+// and pure copies alternate within every warp. Lane 0 keeps up to kStages items in
+// flight as 1-D TMA bulk loads into the warp's stages (completion on one mbarrier
+// per stage); all lanes wait for an item, move it from shared memory to its place
+// in the output (rotating K rows of slots at a nonzero offset; kPaged: each row's
+// place comes from the block table), and lane 0 refills the stage with the warp's
+// next item. Every wait is bounded: on timeout the warp records an error, waits
+// (bounded) for its own copies in flight and returns.
+template <bool kPaged, int kW, int kStages = kStagesDefault, int kMinBlocks = 16 / kW>
+__global__ void __launch_bounds__(kW * 32, kMinBlocks)
+render_kernel(const __grid_constant__ RenderParams p) {
+    constexpr int kThreads = kW * 32;
+    extern __shared__ __align__(128) uint8_t smem[];
+    // item j of a warp: its data in stage j % kStages, its Item in entry j % kRing (one
+    // entry more than stages, so that a pair's V Item can be written with its K Item)
+    constexpr int kRing = kStages + 1;
+    __shared__ __align__(8) uint64_t full[kW][kStages];
+    __shared__ Item items[kW][kRing];
+    __shared__ PairWalk walks[kW];   // lane 0's position along its warp's pairs
+    float4 *tab = reinterpret_cast<float4 *>(smem + (size_t)kW * kStages * kItemBytes);
+    float *kt = reinterpret_cast<float *>(tab + kMaxTablePairs);
+    float *nst = kt + kMaxTablePairs;
+
+    const int half = p.head_dim >> 1;
+    const int n_table = p.num_slots * half;
+    for (int i = threadIdx.x; i < n_table; i += kThreads) {
+        const float2 cc = split16(p.cs[2 * i]), ss = split16(p.cs[2 * i + 1]);
+        tab[i] = make_float4(cc.x, cc.y, ss.x, ss.y);
+        kt[i] = bound_scale(__fadd_rn(cc.x, cc.y), __fadd_rn(ss.x, ss.y));
+        nst[i] = -__fadd_rn(ss.x, ss.y);
+    }
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) {
+        for (int s = 0; s < kStages; ++s) mbar_init(&full[warp][s], 1);
+        fence_mbar_init();
+    }
+    __syncthreads();
+
+    const uint32_t first = blockIdx.x * kW + warp;
+    const uint32_t stride = gridDim.x * kW;
+    const uint32_t npairs = p.total_chunks / 2;
+    const uint32_t n = npairs > first ? 2 * ((npairs - first + stride - 1) / stride) : 0;
+    const int lane_v = lane & ((p.head_dim >> 4) - 1);
+    uint8_t *wbuf = smem + (size_t)warp * kStages * kItemBytes;
+
+    // Item j: pair j / 2 of the warp (pairs first, first + stride, ...), K if j is even, V if
+    // odd. Lane 0 walks the pairs by additions and writes a pair's two Items at once, the V
+    // Item into entry (j + 1) % kRing, whose previous item (j + 1 - kRing) has been read.
+    if (lane == 0 && n > 0) {
+        PairWalk w;
+        w.pr = first;
+        w.stride = stride;
+        w.npairs = npairs;
+        w.enter<kPaged>(p);
+        walks[warp] = w;
+    }
+    const uint32_t row_bytes = (uint32_t)p.head_dim * 2;
+    auto produce = [&](uint32_t j) {
+        const uint32_t s = j % kStages;
+        Item it;
+        if ((j & 1u) == 0) {
+            PairWalk w = walks[warp];
+            if (j > 0) {
+                w.next<kPaged>(p);
+                walks[warp] = w;
+            }
+            const Pair q = pair_of<kPaged>(p, w);
+            Item v = half_item(q, true);
+            it = half_item(q, false);
+            it.bytes = v.bytes = (uint32_t)q.rows * row_bytes;
+            items[warp][j % kRing] = it;
+            items[warp][(j + 1) % kRing] = v;
+        } else {
+            it = items[warp][j % kRing];
+        }
+        // bounds-checked builds: a source outside the slot's fragment is not copied (the
+        // stage keeps stale bytes, the barrier completes without them)
+        const bool src_ok = CM_IN_BOUNDS(it.src, it.bytes, it.src_base, it.src_size);
+        mbar_arrive_expect_tx(&full[warp][s], src_ok ? it.bytes : 0u);
+        if (j == 0 && p.withhold_warp == first + 1) return;   // injected: the wait runs out
+        if (src_ok) bulk_load(wbuf + (size_t)s * kItemBytes, it.src, it.bytes, &full[warp][s]);
+    };
+
+    uint32_t produced = 0;
+    if (lane == 0)
+        for (; produced < n && produced < (uint32_t)kStages; ++produced) produce(produced);
+
+    uint32_t i = 0;
+    bool aborted = false;
+    for (; i < n; ++i) {
+        const uint32_t s = i % kStages;
+        const bool ok = mbar_wait(&full[warp][s], (i / kStages) & 1u);
+        if (__any_sync(0xFFFFFFFFu, !ok)) {
+            aborted = true;
+            break;
+        }
+        const Item it = items[warp][i % kRing];
+        const uint8_t *buf = wbuf + (size_t)s * kItemBytes;
+        if (it.rotate)
+            rotate_from_smem<kPaged>(p, tab, kt, nst, it, buf, lane, lane_v);
+        else
+            copy_from_smem<kPaged>(p, it, buf, lane);
+        __syncwarp();                          // every lane is done reading stage s
+        if (lane == 0 && produced < n) {
+            fence_proxy_async_smem();
+            produce(produced++);               // item i + kStages into stage s
+        }
+    }
+    if (aborted && lane == 0) {
+        atomicOr(p.error, 1u);
+        for (uint32_t j = i; j < produced; ++j)
+            mbar_wait(&full[warp][j % kStages], (j / kStages) & 1u);
+    }
+}
+
+template <bool kPaged, int kW, int kStages = kStagesDefault, int kMinBlocks = 16 / kW>
+cudaError_t set_smem_attribute() {
+    return cudaFuncSetAttribute(render_kernel<kPaged, kW, kStages, kMinBlocks>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)dyn_smem<kW, kStages>());
+}
+
+// ---------------------------------------------------------------- full-SM render
+
+constexpr int kRegThreads = 256;           // 8 warps per CTA
+constexpr int kRegBlocksPerSm = 3;         // 24 warps per SM
+constexpr uint32_t kRegItemBytes = 1024;   // one work item: 2 vectors per lane
+constexpr int kRegVecs = kRegItemBytes / 16 / 32;
 
 // Paged outputs: where the rows of a pair go, for K and V alike (the two halves differ only
 // in their pool). When the block size is a power of two no smaller than the pair's row
