@@ -288,8 +288,9 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 
 constexpr int kStagesDefault = 3;                   // per warp
 constexpr uint32_t kItemBytes = 4096;               // one work item = one stage
-// (c1, c2, s1, s2) per frequency, then the first-level bound scale k, then -s32
-constexpr size_t kTableBytes = (sizeof(float4) + 2 * sizeof(float)) * kMaxTablePairs;
+// Per frequency: (c1, c2, s1, s2), then the first-level bound scale k, -s32, c32 and s32
+// (one array of kMaxTablePairs each), so that an item's 8 fp32 (cos, sin) are 4 loads
+constexpr size_t kTableBytes = (sizeof(float4) + 4 * sizeof(float)) * kMaxTablePairs;
 // Dynamic shared memory of a CTA of kW warps: the warps' stages, then the (cos, sin) table.
 template <int kW, int kStages = kStagesDefault>
 constexpr size_t dyn_smem() { return (size_t)kW * kStages * kItemBytes + kTableBytes; }
@@ -423,7 +424,8 @@ __device__ __forceinline__ void copy_from_smem(const RenderParams &p, const Item
 // the same for every q, so its 8 (cos, sin) values are loaded once per item.
 template <bool kPaged>
 __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const float4 *tab,
-                                                 const float *kt, const float *nst, const Item &it,
+                                                 const float *kt, const float *nst, const float *c32,
+                                                 const float *s32, const Item &it,
                                                  const uint8_t *buf, int lane, int lane_v) {
     const int vecs_per_row = p.head_dim >> 3;
     const int half_vecs = p.head_dim >> 4;
@@ -433,10 +435,11 @@ __device__ __forceinline__ void rotate_from_smem(const RenderParams &p, const fl
     if (kPaged) pr = paged_rows(p, it);
     float c[8], s[8];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
-        const float4 t = tab[cs_index + e];
-        c[e] = __fadd_rn(t.x, t.y);   // fp32 cos (within one ulp of the fp64 value)
-        s[e] = __fadd_rn(t.z, t.w);
+    for (int h = 0; h < 2; ++h) {
+        const float4 cv = *reinterpret_cast<const float4 *>(c32 + cs_index + 4 * h);
+        const float4 sv = *reinterpret_cast<const float4 *>(s32 + cs_index + 4 * h);
+        c[4 * h] = cv.x, c[4 * h + 1] = cv.y, c[4 * h + 2] = cv.z, c[4 * h + 3] = cv.w;
+        s[4 * h] = sv.x, s[4 * h + 1] = sv.y, s[4 * h + 2] = sv.z, s[4 * h + 3] = sv.w;
     }
     const uint4 *src = reinterpret_cast<const uint4 *>(buf);
 #pragma unroll 1
@@ -626,14 +629,18 @@ render_kernel(const __grid_constant__ RenderParams p) {
     float4 *tab = reinterpret_cast<float4 *>(smem + (size_t)kW * kStages * kItemBytes);
     float *kt = reinterpret_cast<float *>(tab + kMaxTablePairs);
     float *nst = kt + kMaxTablePairs;
+    float *c32 = nst + kMaxTablePairs;
+    float *s32 = c32 + kMaxTablePairs;
 
     const int half = p.head_dim >> 1;
     const int n_table = p.num_slots * half;
     for (int i = threadIdx.x; i < n_table; i += kThreads) {
         const float2 cc = split16(p.cs[2 * i]), ss = split16(p.cs[2 * i + 1]);
         tab[i] = make_float4(cc.x, cc.y, ss.x, ss.y);
-        kt[i] = bound_scale(__fadd_rn(cc.x, cc.y), __fadd_rn(ss.x, ss.y));
-        nst[i] = -__fadd_rn(ss.x, ss.y);
+        c32[i] = __fadd_rn(cc.x, cc.y);   // fp32 cos (within one ulp of the fp64 value)
+        s32[i] = __fadd_rn(ss.x, ss.y);
+        kt[i] = bound_scale(c32[i], s32[i]);
+        nst[i] = -s32[i];
     }
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (lane == 0) {
@@ -703,7 +710,7 @@ render_kernel(const __grid_constant__ RenderParams p) {
         const Item it = items[warp][i % kRing];
         const uint8_t *buf = wbuf + (size_t)s * kItemBytes;
         if (it.rotate)
-            rotate_from_smem<kPaged>(p, tab, kt, nst, it, buf, lane, lane_v);
+            rotate_from_smem<kPaged>(p, tab, kt, nst, c32, s32, it, buf, lane, lane_v);
         else
             copy_from_smem<kPaged>(p, it, buf, lane);
         __syncwarp();                          // every lane is done reading stage s
