@@ -501,6 +501,13 @@ __global__ void compare_kernel(const uint4 *__restrict__ a, const uint4 *__restr
 
 CM_DEFINE_BOUNDS_READER(take_hash_bounds_violations)
 
+int leaf_hash_blocks_per_sm() {
+    int n = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, leaf_hash_kernel, kLeafThreads, 0) != cudaSuccess)
+        return 0;
+    return n;
+}
+
 cudaError_t launch_leaf_hash_group(const LeafGroup &in, cudaStream_t stream, LeafPhases phases) {
     if (in.count > (uint32_t)kMaxLeafGroup) return cudaErrorInvalidValue;
     if (in.count == 0) return cudaSuccess;

@@ -56,6 +56,8 @@ struct LeafGroup {
 // norm keys alone read only K[l*], 1/(2L) of the bytes).
 enum class LeafPhases { kBoth, kLeaves, kNormKeys };
 cudaError_t launch_leaf_hash_group(const LeafGroup &g, cudaStream_t stream, LeafPhases phases);
+// Leaf-hash blocks that fit on one SM at once (occupancy of leaf_hash_kernel), or 0 on error.
+int leaf_hash_blocks_per_sm();
 
 // Level 0 of one fragment (a group of one).
 cudaError_t launch_leaf_hash(const LeafLaunch &a, cudaStream_t stream);

@@ -120,6 +120,7 @@ struct cm_context {
     int32_t routing_layer = -1;
     bool verify = false;
     int num_sms = 0;
+    int leaf_blocks_per_sm = 0;   // leaf-hash blocks resident on one SM at once
     unsigned int *d_error = nullptr;   // set by a kernel whose bounded wait timed out
     std::mutex mu;
     // hashing scratch (device): leaf digests, inner levels, Q[t], compare flag
@@ -1073,6 +1074,7 @@ cm_status cm_context_create(int32_t device, double rope_theta, int32_t routing_l
         CM_CUDA_TRY(cudaDeviceGetAttribute(&ctx->num_sms, cudaDevAttrMultiProcessorCount, device),
                     "multiprocessor count");
         CM_CUDA_TRY(cm::render_prepare(), "render kernel attributes");
+        ctx->leaf_blocks_per_sm = cm::leaf_hash_blocks_per_sm();
         CM_CUDA_TRY(cudaMalloc(&ctx->d_error, sizeof(unsigned int)), "error word allocation");
         CM_CUDA_TRY(cudaMemset(ctx->d_error, 0, sizeof(unsigned int)), "error word reset");
         *out = ctx.release();
@@ -1501,12 +1503,27 @@ cm_status ingest_render_impl(cm_set *const *sets, const cm_fragment *frags, int3
         if (e != cudaSuccess && prior == CM_OK) return cuda_fail(e, "side stream ordering");
         return prior;
     };
+    // The norm keys decide when the render can start. A leaf grid that leaves a block's room
+    // on every SM (one partial wave) is launched first: the hash starts a few launches
+    // earlier and the norm-key blocks still start at once beside it. A larger grid would
+    // take every SM and hold back norm keys launched after it until its first wave retires.
+    uint64_t leaf_blocks = 0;
+    for (const DigestPlan::Frag &l : plan.f) leaf_blocks += ceil_div(l.sizes[0], (uint64_t)cm::kLeafBlockThreads);
+    const bool digest_first =
+        ctx->leaf_blocks_per_sm > 1 &&
+        leaf_blocks <= (uint64_t)(ctx->leaf_blocks_per_sm - 1) * (uint64_t)ctx->num_sms;
+    if (digest_first) {
+        st = enqueue_digest(ctx, plan, fp.data(), fp.size(), cs, false);
+        if (st != CM_OK) return join(st);
+    }
     st = enqueue_norm_keys(ctx, fp.data(), fp.size(), ctx->side, q_dev, q_host, q_off, q_bytes);
     if (st != CM_OK) return join(st);
     cudaError_t e = cudaEventRecord(ctx->side_keys, ctx->side);
     if (e != cudaSuccess) return join(cuda_fail(e, "side stream ordering"));
-    st = enqueue_digest(ctx, plan, fp.data(), fp.size(), cs, false);
-    if (st != CM_OK) return join(st);
+    if (!digest_first) {
+        st = enqueue_digest(ctx, plan, fp.data(), fp.size(), cs, false);
+        if (st != CM_OK) return join(st);
+    }
     e = cudaEventSynchronize(ctx->side_keys);
     if (e != cudaSuccess) return join(cuda_fail(e, "norm-key synchronisation"));
     std::vector<std::vector<uint64_t>> Qd((size_t)n);
