@@ -603,17 +603,16 @@ __device__ __forceinline__ Item half_item(const Pair &q, bool v) {
 }
 
 // Half-SM render: a persistent kernel with one CTA of kW = 8 warps per SM (half of the
-// register file, leaving room for kernels of other streams on the same SMs); every
-// warp runs its own
-// pipeline over its own items, with no block-wide barrier after set-up. Items come
-// in (K, V) pairs of the same (slot, layer, head, row chunk); a warp takes pairs
-// warp id + m * total warps and does the K item, then the V item, so rotation work
-// and pure copies alternate within every warp. Lane 0 keeps up to kStages items in
-// flight as 1-D TMA bulk loads into the warp's stages (completion on one mbarrier
-// per stage); all lanes wait for an item, move it from shared memory to its place
-// in the output (rotating K rows of slots at a nonzero offset; kPaged: each row's
-// place comes from the block table), and lane 0 refills the stage with the warp's
-// next item. Every wait is bounded: on timeout the warp records an error, waits
+// register file, leaving room for kernels of other streams on the same SMs; kW = 4 with 6
+// stages beside the leaf hash); every warp runs its own pipeline over its own items, with
+// no block-wide barrier after set-up. Items come in (K, V) pairs of the same (slot, layer,
+// head, row chunk); a warp takes pairs warp id + m * total warps and does the K item,
+// then the V item, so rotation work and pure copies alternate within every warp. Lane 0
+// keeps up to kStages items in flight as 1-D TMA bulk loads into the warp's stages
+// (completion on one mbarrier per stage); all lanes wait for an item, move it from shared
+// memory to its place in the output (rotating K rows of slots at a nonzero offset; kPaged:
+// each row's place comes from the block table), and lane 0 refills the stage with the
+// warp's next item. Every wait is bounded: on timeout the warp records an error, waits
 // (bounded) for its own copies in flight and returns.
 template <bool kPaged, int kW, int kStages = kStagesDefault, int kMinBlocks = 16 / kW>
 __global__ void __launch_bounds__(kW * 32, kMinBlocks)
