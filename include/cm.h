@@ -240,8 +240,9 @@ cm_status cm_render(const cm_set *set, void *k_out, void *v_out, int64_t capacit
  *     cm_union(target, s) for every set s of `sets` other than target, in order of first
  *         appearance (the replicas' states merged into target, Eq. setunion);
  *     cm_render(target, k_out, v_out, capacity_tokens, stream, out_seq_len, out_order);
- * Overlap: the routing-layer norm keys (Eq. rho) of the deliveries are computed first
- * (one pass over K[l*], 1/(2L) of the bytes, and a synchronisation). Byte-identical
+ * Overlap: the routing-layer norm keys (Eq. rho) of the deliveries are computed as the
+ * call starts, beside the content address (one pass over K[l*], 1/(2L) of the bytes, and
+ * a synchronisation). Byte-identical
  * fragments have equal norm keys, so members of the prospective set (the target's
  * fragments, the other sets', every delivery) whose integer tail sums S, lengths and
  * per-token norm keys all agree are taken for one fragment; if the remaining S are
